@@ -1,0 +1,383 @@
+#!/usr/bin/env python
+"""Benchmark of the pruned prefill (Zero-Shot Adjustable Acceleration) on GB300.
+
+Default workload: the Llama-3.2-1B-shaped decoder (16 layers, d=2048, 32/8
+heads, SwiGLU 8192, vocab 128256), bf16, random-init N(0, 0.02) weights,
+batch 8 x 512 uniform random tokens.  One step = one pruned prefill of the
+whole batch at the headline acceleration factor (--accel, default 4), i.e.
+every row of the path: plan, embed, per layer RMSNorm / QKV+RoPE / attention /
+O+residual / RMSNorm / SwiGLU MLP + residual / column mass / score / top-k /
+gather, then the LM head on the kept rows.
+
+Prints ONE JSON line (rank 0).  value = prefill tokens/s (B*L input tokens per
+forward, all ranks) timed with CUDA events on the launch stream, L2 flushed
+(256 MiB write) between timed steps.  Extra keys: the accel sweep (tokens/s,
+speedup over the same library's unpruned forward, modelled FLOP reduction),
+the roofline of the dominant kernel from the library's per-kernel trace, an
+end-to-end number through zsaa_forward_host with pinned host buffers, the CPU
+oracle timed on the host cores, and SM clocks sampled during the timed region.
+
+--impl reference times the CPU oracle (the reference arm for this build) on
+a bounded sample of the same workload: one sequence per step.
+Multi-GPU (torchrun): every rank runs its own batch (sequences are
+independent; no collective on the data path), value = all ranks' tokens /
+max over ranks of the timed span.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    except OSError:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples every 200 ms while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-f", self.path], stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        try:
+            with open(self.path) as f:
+                for line in f:
+                    parts = [x.strip() for x in line.split(",")]
+                    if len(parts) >= 9:
+                        rows.append(parts)
+        except OSError:
+            pass
+        finally:
+            try:
+                os.unlink(self.path)
+            except OSError:
+                pass
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no nvidia-smi samples"]}
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        smax = [num(r[2]) for r in rows if num(r[2]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = [n for i, n in enumerate(names) if any(r[5 + i].lower() == "active" for r in rows)]
+        power = [num(r[3]) for r in rows if num(r[3]) is not None]
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": reasons, "samples": len(rows), "power_w_max": max(power) if power else None}
+
+
+def oracle_config(shape):
+    from oracle import zsaa_oracle as O
+    return O.OracleConfig(
+        n_layers=shape.n_layers, d_model=shape.d_model, n_heads=shape.n_heads,
+        n_kv_heads=shape.n_kv_heads, head_dim=shape.head_dim, ffn_dim=shape.ffn_dim,
+        vocab=shape.vocab, n_classes=shape.n_classes, rope_theta=shape.rope_theta,
+        rms_eps=shape.rms_eps, dtype=shape.dtype, prune_layers=shape.prune_layers(),
+        plan_mode=shape.plan_mode)
+
+
+def cpu_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads") for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    return os.cpu_count()
+
+
+def time_oracle(shape, weights_np, tokens, accel, budget_s, max_seqs):
+    """Oracle forward on sequences one at a time until budget_s elapses."""
+    from oracle import zsaa_oracle as O
+    ocfg = oracle_config(shape)
+    t0 = time.perf_counter()
+    n = 0
+    while n < max_seqs:
+        O.forward(ocfg, weights_np, tokens[n: n + 1], accel=accel)
+        n += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    return n, time.perf_counter() - t0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="1b", choices=["1b", "1b_cls", "8b"])
+    ap.add_argument("--accel", type=float, default=4.0)
+    ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle work for cpu_baseline")
+    ap.add_argument("--no-extras", action="store_true", help="headline timing only")
+    args = ap.parse_args()
+
+    import numpy as np
+    import torch
+
+    from paper_2509_01190_gb300 import inputs as I
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    wl = I.WORKLOADS[args.workload]
+    shape, B, L = wl["shape"], wl["B"], wl["L"]
+    workload_name = f"{shape.name} B={B} L={L} accel={args.accel:g}"
+
+    if args.impl == "reference":
+        # reference arm: the CPU oracle, one sequence per step, rank 0 only
+        if rank != 0:
+            return
+        g = torch.Generator().manual_seed(I.WEIGHT_SEED)  # noqa: F841  (weights drawn below on CPU)
+        weights = I.make_weights(shape, device="cpu")
+        wnp = I.weights_to_numpy(weights)
+        tokens = I.make_tokens(max(B, args.steps + args.warmup), L, shape.vocab)
+        from oracle import zsaa_oracle as O
+        ocfg = oracle_config(shape)
+        for w in range(args.warmup):
+            O.forward(ocfg, wnp, tokens[w: w + 1], accel=args.accel)
+        times = []
+        for s in range(args.steps):
+            t0 = time.perf_counter()
+            O.forward(ocfg, wnp, tokens[(args.warmup + s) % len(tokens)][None], accel=args.accel)
+            times.append(time.perf_counter() - t0)
+        tot = sum(times)
+        val = args.steps * L / tot
+        line = {"impl": "reference", "metric": "prefill_tokens_per_s", "value": val, "unit": "tokens/s",
+                "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": 1e3 * tot / args.steps, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                "config": {"workload": workload_name + " (CPU oracle, 1 sequence per step)",
+                           "global_batch": 1, "seq_len": L, "accel": args.accel},
+                "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": cpu_threads(), "kind": "oracle",
+                                 "sample": f"1 of {B} sequences per step, float64 NumPy oracle"},
+                "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return
+
+    from paper_2509_01190_gb300 import zsaa
+
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", init_method="env://")
+    else:
+        dist = None
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", torch.cuda.current_device())
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        torch.cuda.synchronize()
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    def max_over_ranks(x):
+        if dist is None:
+            return x
+        t = torch.tensor([x], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    weights = I.make_weights(shape, device=dev)
+    tokens = I.make_tokens(B, L, shape.vocab, seed=I.TOKEN_SEED + rank)
+    tok_dev = torch.from_numpy(tokens).to(dev)
+    cfg = zsaa.config_from_shape(shape)
+    model = zsaa.Model(cfg, weights, B, L)
+    sched1, _ = zsaa.zsaa_plan(model, L, 1.0)
+    max_out = B * (shape.n_classes if shape.n_classes else L * shape.vocab)
+    logits = torch.empty(max_out, device=dev, dtype=torch.float32)
+    flush = torch.empty(256 * 1024 * 1024 // 4, device=dev, dtype=torch.float32)
+
+    def run(accel):
+        zsaa.zsaa_forward(model, tok_dev, B, L, accel, logits, None, stream=stream)
+
+    def timed(accel, steps, warmup, sampler=None):
+        for _ in range(warmup):
+            run(accel)
+        zsaa.zsaa_sync(model)
+        barrier()
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+        ctx = sampler if sampler is not None else None
+        if ctx:
+            ctx.__enter__()
+        try:
+            for a, b in evs:
+                flush.zero_()
+                a.record(stream)
+                run(accel)
+                b.record(stream)
+            torch.cuda.synchronize()
+        finally:
+            if ctx:
+                ctx.__exit__(None, None, None)
+        zsaa.zsaa_sync(model)
+        ms = sum(a.elapsed_time(b) for a, b in evs)
+        barrier()
+        return max_over_ranks(ms) / steps
+
+    # ---- headline
+    sampler = ClockSampler(local) if rank == 0 else None
+    ms_head = timed(args.accel, args.steps, args.warmup, sampler)
+    sched, alpha = zsaa.zsaa_plan(model, L, args.accel)
+    value = world * B * L / (ms_head / 1e3)
+    clocks = sampler.summary() if sampler else None
+
+    line = {"metric": "prefill_tokens_per_s", "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_head, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if shape.dtype == "bf16" else "f32",
+            "data": "synthetic (seeded N(0,0.02) weights, uniform token ids)",
+            "config": {"workload": workload_name, "model": shape.name, "global_batch": B * world,
+                       "seq_len": L, "accel": args.accel, "alpha": alpha, "schedule": sched,
+                       "parallelism": f"replicas x{world} (independent sequences, no collective)",
+                       "l2": "flushed between timed steps (256 MiB write); weights 2.5 GB > L2"},
+            "clocks": clocks}
+
+    if not args.no_extras:
+        from oracle import zsaa_oracle as O
+        ocfg = oracle_config(shape)
+        full_cost = O.model_cost(ocfg, sched1)
+        # ---- accel sweep (speedup over the same library's unpruned forward)
+        sweep = {}
+        base_ms = None
+        for a in sorted(set(wl["accels"]) | {args.accel}):
+            ms = ms_head if a == args.accel else timed(a, args.steps, 3)
+            s_a, al_a = zsaa.zsaa_plan(model, L, a)
+            if a == 1.0:
+                base_ms = ms
+            sweep[f"{a:g}"] = {"ms": ms, "tokens_per_s": world * B * L / (ms / 1e3), "alpha": al_a,
+                               "final_rows": s_a[-1],
+                               "modelled_flop_reduction": full_cost / O.model_cost(ocfg, s_a)}
+        for k, v in sweep.items():
+            v["speedup_vs_unpruned"] = (base_ms / v["ms"]) if base_ms else None
+        line["sweep"] = sweep
+
+        # ---- per-kernel trace of the headline forward (separate traced steps)
+        zsaa.zsaa_trace_begin(model)
+        n_tr = 3
+        for _ in range(n_tr):
+            flush.zero_()
+            run(args.accel)
+        rows = zsaa.zsaa_trace_end(model)
+        zsaa.zsaa_sync(model)
+        tot_ms = sum(r["ms"] for r in rows)
+        kern = {}
+        for r in rows:
+            kern[r["name"]] = {"launches_per_step": r["launches"] / n_tr, "ms_per_step": r["ms"] / n_tr,
+                               "share": r["ms"] / tot_ms if tot_ms else None,
+                               "tflops": (r["flops"] / (r["ms"] / 1e3) / 1e12) if r["ms"] and r["flops"] else None,
+                               "gbs": (r["bytes"] / (r["ms"] / 1e3) / 1e9) if r["ms"] else None}
+        line["kernels"] = kern
+        launches = sum(r["launches"] for r in rows) // n_tr
+        line["gpu_launches"] = launches * args.steps
+        peaks, src = load_peaks()
+        gemms = [r for r in rows if r["name"].startswith("gemm")]
+        dom = max(gemms, key=lambda r: r["ms"]) if gemms else max(rows, key=lambda r: r["ms"])
+        if dom["flops"] > 0:
+            ach = dom["flops"] / (dom["ms"] / 1e3) / 1e12
+            peak = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+            line["roofline"] = {"bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
+                                "frac": ach / peak, "traffic": None, "kernel": dom["name"],
+                                "per_launch_ms": dom["ms"] / dom["launches"],
+                                "peak_source": f"{src} bf16_tflops_sustained (kernel inside a long step)"}
+        else:
+            ach = dom["bytes"] / (dom["ms"] / 1e3) / 1e9
+            peak = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+            line["roofline"] = {"bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
+                                "frac": ach / peak, "traffic": None, "kernel": dom["name"],
+                                "peak_source": f"{src} hbm_gbs"}
+        gemm_f = sum(r["flops"] for r in gemms)
+        gemm_ms = sum(r["ms"] for r in gemms)
+        if gemm_ms:
+            line["roofline"]["all_gemms_tflops"] = gemm_f / (gemm_ms / 1e3) / 1e12
+            line["roofline"]["all_gemms_share"] = gemm_ms / tot_ms
+
+        # ---- end to end through the host-buffer entry point
+        n_fin = sched[-1]
+        n_logit = B * (shape.n_classes if shape.n_classes else n_fin * shape.vocab)
+        tok_h = torch.from_numpy(tokens).pin_memory()
+        log_h = torch.empty(n_logit, dtype=torch.float32).pin_memory()
+        for _ in range(2):
+            zsaa.zsaa_forward_host(model, tok_h, B, L, args.accel, log_h, None, stream=stream)
+        barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            flush.zero_()
+            zsaa.zsaa_forward_host(model, tok_h, B, L, args.accel, log_h, None, stream=stream)
+        torch.cuda.synchronize()
+        e2e_s = max_over_ranks(time.perf_counter() - t0) / args.steps
+        line["e2e"] = {"value": world * B * L / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": B * L * 4,
+                       "d2h_bytes_per_step": n_logit * 4, "ms_per_step": e2e_s * 1e3,
+                       "note": "zsaa_forward_host: pinned host tokens in, host float32 logits out; "
+                               "the 256 MiB L2 flush runs inside this span"}
+
+        # ---- CPU oracle on the host cores (rank 0, N=1 only)
+        if rank == 0 and world == 1:
+            wnp = I.weights_to_numpy(weights)
+            n, secs = time_oracle(shape, wnp, tokens, args.accel, args.cpu_budget, B)
+            line["cpu_baseline"] = {"value": n * L / secs, "unit": "tokens/s", "cores": cpu_threads(),
+                                    "kind": "oracle",
+                                    "sample": f"{n} of {B} sequences x {L} tokens at accel {args.accel:g}, "
+                                              f"float64 NumPy oracle, {secs:.1f} s"}
+    if rank == 0:
+        print(json.dumps(line))
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,252 @@
+/*
+ * zsaa.h -- C ABI of the GB300 pruned-prefill library (Zero-Shot Adjustable
+ * Acceleration, arXiv 2509.01190).
+ *
+ * The library runs the prefill forward pass of a pre-norm decoder (RMSNorm,
+ * grouped-query attention with RoPE, SwiGLU MLP; Appendix A) in which, after
+ * each pruning layer, every position is scored by its soft-score contribution
+ * (Sec. 3.2-3.3), the top N_l positions are kept and compacted into a dense
+ * [B, N_l, d] buffer, and the following layers run on those rows only.  N_l
+ * follows Eq. 2 with a preservation rate alpha chosen per call from an
+ * acceleration factor (Sec. 3.4).
+ *
+ * Conventions for every call:
+ *  - Pointers documented "device" are CUDA device pointers; "host" pointers
+ *    are ordinary CPU memory.  The library never frees caller memory.
+ *  - Work is enqueued on the given stream and is asynchronous unless stated.
+ *    Argument errors are found before anything is enqueued and return
+ *    ZSAA_ERR_INVALID_ARG with nothing launched.
+ *  - Device-side failures (a bounded wait that ran out) set a status word that
+ *    zsaa_sync / zsaa_device_status report; kernels never trap.
+ *  - No C++ exception crosses this boundary.  zsaa_last_error() returns a
+ *    thread-local message for the last failing call on the calling thread.
+ *  - Matrices are row-major.  Linear weights are [out_features, in_features]
+ *    (each output feature's weights contiguous), the layout the GEMMs read as
+ *    K-major operands.  bf16 buffers hold IEEE bfloat16 bit patterns.
+ */
+#ifndef ZSAA_H
+#define ZSAA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#pragma GCC visibility push(default)
+#endif
+
+/* Same type as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st* zsaa_stream;
+
+typedef enum {
+  ZSAA_OK = 0,
+  ZSAA_ERR_INVALID_ARG = 1,
+  ZSAA_ERR_OOM = 2,
+  ZSAA_ERR_CUDA = 3,
+  ZSAA_ERR_TIMEOUT = 4,
+  ZSAA_ERR_UNSUPPORTED = 5
+} zsaa_status;
+
+/* Storage type of weights and activations. */
+enum { ZSAA_F32 = 0, ZSAA_BF16 = 1 };
+
+/* Position score (Sec. 3.2: soft-score times V is each V row's contribution).
+ * SOFTSCORE_VNORM: s_j = sum_g C[g,j] * ||v_{g,j}||_2 ; SOFTSCORE: sum_g C[g,j]
+ * where C[g,j] sums soft-score column j over all queries and over the query
+ * heads of KV group g. */
+enum { ZSAA_SCORE_SOFTSCORE_VNORM = 0, ZSAA_SCORE_SOFTSCORE = 1 };
+
+/* Acceleration factor -> preservation rate (Sec. 3.4).  COST: the largest
+ * alpha (60-step bisection on [0,1]) whose modelled per-sequence FLOPs are at
+ * most 1/accel of the unpruned ones.  RATE: alpha = 1/accel. */
+enum { ZSAA_PLAN_COST = 0, ZSAA_PLAN_RATE = 1 };
+
+/* Flags of zsaa_score_select_ex. */
+enum { ZSAA_FLAG_FORCE_KEEP_LAST = 1 };
+
+/* Decoder shape and pruning options (Appendix A, Table 1; Eq. 2). */
+typedef struct {
+  int n_layers;     /* 1..64 */
+  int d_model;      /* multiple of 64 */
+  int n_heads;      /* query heads */
+  int n_kv_heads;   /* KV heads; n_heads % n_kv_heads == 0 */
+  int head_dim;     /* 32, 64 or 128 (bf16: 64 or 128) */
+  int ffn_dim;      /* multiple of 64 */
+  int vocab;        /* embedding rows */
+  int n_classes;    /* 0: LM head over the vocabulary; >0: classifier on the last kept row */
+  float rope_theta; /* RoPE base; frequency i of a head is theta^(-2i/head_dim) */
+  float rms_eps;    /* RMSNorm epsilon */
+  int dtype;        /* ZSAA_F32 or ZSAA_BF16 */
+  int tau;          /* Eq. 2 floor on kept rows (the paper uses 5, Sec. 4.2) */
+  uint64_t prune_mask;  /* bit l-1 set: layer l compacts its output rows */
+  int force_keep_last;  /* 1: the last position is always kept (counts toward N_l) */
+  int score_mode;       /* ZSAA_SCORE_* */
+  int plan_mode;        /* ZSAA_PLAN_* */
+} zsaa_config;
+
+/* Borrowed device weights; they must outlive the model.  layers points to a
+ * HOST array of n_layers*9 device pointers, per layer in this order:
+ *   attn_norm [d], wq [Hq*hd, d], wk [Hkv*hd, d], wv [Hkv*hd, d],
+ *   wo [d, Hq*hd], mlp_norm [d], wg [F, d], wu [F, d], wd [d, F].
+ * embed is [vocab, d]; final_norm [d]; head is [vocab, d] (may equal embed)
+ * or [n_classes, d].  The pointer array itself is copied at create time. */
+typedef struct {
+  const void* embed;
+  const void* const* layers;
+  const void* final_norm;
+  const void* head;
+} zsaa_weights;
+
+typedef struct zsaa_model zsaa_model;
+
+/* Test and inspection hooks of zsaa_forward_ex.  All pointers are device
+ * pointers or NULL.  Per-pruning-layer arrays are concatenated in layer order
+ * over the layers whose bit is set in prune_mask (and that run):
+ *   forced_idx : [B, N_l] int32 ascending indices into that layer's N_{l-1}
+ *                rows, replacing the top-k choice (Sec. 3.3) there;
+ *   scores_out : [B, N_{l-1}] float32 position scores of that layer;
+ *   idx_out    : [B, N_l] int32 kept indices of that layer.
+ * hidden_out : [B, N_last, d] residual rows leaving the last layer run.
+ * n_layers_run: 0 runs all layers; m > 0 runs layers 1..m, then the head. */
+typedef struct {
+  const int32_t* forced_idx;
+  float* scores_out;
+  int32_t* idx_out;
+  void* hidden_out;
+  int n_layers_run;
+} zsaa_forward_opts;
+
+/* Eq. 2 schedule for a config without a model (host only, no GPU needed).
+ * n_sched receives N_0..N_{n_layers} (n_layers+1 ints, host); *alpha_out the
+ * preservation rate.  accel >= 1; L >= 1. */
+zsaa_status zsaa_plan_config(const zsaa_config* cfg, int L, double accel, int* n_sched,
+                             double* alpha_out);
+
+/* Validate the config, build GEMM tensor maps over the borrowed weights and
+ * allocate workspace for batches up to max_B x max_L (device memory owned by
+ * the model).  On error *out is NULL. */
+zsaa_status zsaa_model_create(const zsaa_config* cfg, const zsaa_weights* w, int max_B,
+                              int max_L, zsaa_model** out);
+
+/* Free the model's workspace (not the weights).  Waits for the device. */
+void zsaa_model_destroy(zsaa_model* m);
+
+/* zsaa_plan_config for the model's config. */
+zsaa_status zsaa_plan(const zsaa_model* m, int L, double accel, int* n_sched, double* alpha_out);
+
+/* Pruned prefill of B sequences of L tokens (Sec. 3.3-3.4).
+ *   token_ids   : device [B, L] int32 in [0, vocab)
+ *   logits_out  : device float32 [B, N_final, vocab] (LM head; N_final is the
+ *                 last entry of the schedule) or [B, n_classes]
+ *   kept_pos_out: device int32 [B, N_final] original positions of the rows
+ *                 the logits belong to, or NULL
+ * 1 <= B <= max_B, 1 <= L <= max_L, accel >= 1. */
+zsaa_status zsaa_forward(zsaa_model* m, const int32_t* token_ids, int B, int L, double accel,
+                         float* logits_out, int32_t* kept_pos_out, zsaa_stream stream);
+
+/* zsaa_forward with the hooks of zsaa_forward_opts (opts may be NULL). */
+zsaa_status zsaa_forward_ex(zsaa_model* m, const int32_t* token_ids, int B, int L, double accel,
+                            float* logits_out, int32_t* kept_pos_out,
+                            const zsaa_forward_opts* opts, zsaa_stream stream);
+
+/* zsaa_forward on HOST buffers: copies token_ids (host [B, L]) in, runs, copies
+ * logits (host float32, same shape as zsaa_forward) and kept positions (host or
+ * NULL) out, and returns after the stream has finished.  Device staging is
+ * owned by the model (allocated on first use). */
+zsaa_status zsaa_forward_host(zsaa_model* m, const int32_t* token_ids, int B, int L,
+                              double accel, float* logits_out, int32_t* kept_pos_out,
+                              zsaa_stream stream);
+
+/* Isolated score + select + compaction (Sec. 3.3 with unit column mass and one
+ * group, so the score of a row is its L2 norm):
+ *   hidden      : device bf16 [B, L, d]
+ *   idx_out     : device int32 [B, k], ascending kept indices per sequence
+ *   gathered_out: device bf16 [B, k, d] kept rows, or NULL
+ * 1 <= k <= L; d % 8 == 0.  Ties keep the lower index.  Scratch for the scores
+ * is allocated stream-ordered from the device's default memory pool. */
+zsaa_status zsaa_score_select(const void* hidden, int B, int L, int d, int k, int32_t* idx_out,
+                              void* gathered_out, zsaa_stream stream);
+
+/* zsaa_score_select with options: dtype ZSAA_BF16 or ZSAA_F32 rows; flags
+ * ZSAA_FLAG_*; scores_in (device float32 [B, L]) replaces the computed scores
+ * when not NULL; scores_out (device float32 [B, L]) receives the scores used.
+ * NaN scores rank below every number. */
+zsaa_status zsaa_score_select_ex(const void* hidden, int B, int L, int d, int dtype, int k,
+                                 int flags, const float* scores_in, float* scores_out,
+                                 int32_t* idx_out, void* gathered_out, zsaa_stream stream);
+
+/* Single steps of the path, for per-kernel checks and timing.  All pointers
+ * device; shapes as stated.
+ * zsaa_op_linear: out[M,N] = epilogue(A[M,K] W[N,K]^T); dtype ZSAA_BF16 uses
+ * the tensor-core GEMM, ZSAA_F32 the fp32 CUDA-core GEMM.  epilogue:
+ *   0 store (out has dtype; bf16 rounds once),
+ *   1 residual: out = resid + acc (resid may alias out),
+ *   2 SwiGLU: out[M,N] = silu(A W^T) * (A W2^T), W and W2 both [N,K],
+ *   3 store float32 (out is float32 whatever dtype),
+ *   4 RoPE: columns [0, rope_cols) are heads of rope_hd dims rotated at
+ *     positions pos[M] (each in [0, 16384)) with base rope_theta
+ *     (rotate-half pairing: dims c and c + rope_hd/2), then bf16 store.
+ * K % 64 == 0 and N % 16 == 0 for bf16; RoPE only for bf16. */
+zsaa_status zsaa_op_linear(const void* A, const void* W, const void* W2, const void* resid,
+                           void* out, int M, int N, int K, int dtype, int epilogue,
+                           const int32_t* pos, int rope_cols, int rope_hd, float rope_theta,
+                           zsaa_stream stream);
+
+/* zsaa_op_attention: causal grouped-query attention (Eq. 1) over a packed
+ * qkv [B*N, (Hq + 2 Hkv) hd] buffer (per row: Hq query heads, then Hkv key
+ * heads, then Hkv value heads).  out [B*N, Hq*hd]; lse float32 [B, Hq, N]
+ * gets log2 of the softmax normaliser of the scaled logits (log2 domain). */
+zsaa_status zsaa_op_attention(const void* qkv, int B, int N, int Hq, int Hkv, int hd, int dtype,
+                              void* out, float* lse, zsaa_stream stream);
+
+/* zsaa_op_colmass: C[B, Hkv, N] float32, C[b,g,j] = sum over the query heads
+ * of group g and queries i >= j of the soft-score P[i,j] (Sec. 3.2), using
+ * the lse that zsaa_op_attention wrote. */
+zsaa_status zsaa_op_colmass(const void* qkv, const float* lse, int B, int N, int Hq, int Hkv,
+                            int hd, int dtype, float* colmass, zsaa_stream stream);
+
+/* Per-kernel timing of the forward pass.  After zsaa_trace_begin every
+ * kernel the model launches is bracketed by CUDA events recorded on the launch
+ * stream (this adds a small gap between launches, so traced forwards are not
+ * for headline timing).  zsaa_trace_end waits for the device, stops recording
+ * and fills up to max_rows rows (host array), one per kernel class in first
+ * launch order: launches, summed device milliseconds, and the algorithmic
+ * FLOPs (2 per multiply-add; causal attention counts only j <= i) and HBM
+ * bytes (each tensor read or written once) of those launches. */
+typedef struct {
+  char name[32];
+  int launches;
+  double ms;
+  double flops;
+  double bytes;
+} zsaa_trace_row;
+
+zsaa_status zsaa_trace_begin(zsaa_model* m);
+zsaa_status zsaa_trace_end(zsaa_model* m, zsaa_trace_row* rows, int max_rows, int* n_rows);
+
+/* Wait for the stream and report the model's device status word (then clear
+ * it): ZSAA_OK, or ZSAA_ERR_TIMEOUT if a kernel gave up a bounded wait. */
+zsaa_status zsaa_sync(zsaa_model* m, zsaa_stream stream);
+
+/* Status word shared by the calls that have no model (zsaa_score_select*,
+ * zsaa_op_*): synchronises the device, returns it and clears it. */
+zsaa_status zsaa_device_status(void);
+
+/* Message of the last failing call on this thread ("" if none). */
+const char* zsaa_last_error(void);
+
+/* Library version string. */
+const char* zsaa_version(void);
+
+#if defined(__GNUC__)
+#pragma GCC visibility pop
+#endif
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ZSAA_H */

@@ -1,0 +1,477 @@
+// Row-wise kernels of the pruned prefill: embedding gather, RMSNorm, position
+// scores (Sec. 3.2-3.3), per-sequence top-k selection, row compaction, fp32
+// RoPE and the classifier head.  All are HBM-bound: one warp per row, 16-byte
+// vector accesses, fp32 arithmetic.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace zsaa {
+
+namespace {
+
+constexpr int kWarpsPerBlock = 8;
+
+inline int row_blocks(int rows) { return (rows + kWarpsPerBlock - 1) / kWarpsPerBlock; }
+
+// ---------------------------------------------------------------- embedding
+
+// h[r, :] = E[tok[r], :], pos[r] = r mod L  (a row is d * elem bytes, copied as uint4)
+// A token id outside [0, vocab) sets kStatusBadIndex and embeds row 0.
+__global__ void embed_kernel(const uint4* __restrict__ E, const int32_t* __restrict__ tok, int rows,
+                             int L, int vocab, int vec_per_row, uint4* __restrict__ h,
+                             int32_t* __restrict__ pos, int* status) {
+  const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= rows) return;
+  int t = tok[r];
+  if (t < 0 || t >= vocab) {
+    if (lane == 0 && status != nullptr) atomicOr(status, kStatusBadIndex);
+    t = 0;
+  }
+  const uint4* src = E + static_cast<size_t>(t) * vec_per_row;
+  uint4* dst = h + static_cast<size_t>(r) * vec_per_row;
+  for (int v = lane; v < vec_per_row; v += 32) dst[v] = __ldg(src + v);
+  if (lane == 0) pos[r] = r % L;
+}
+
+// ---------------------------------------------------------------- RMSNorm
+
+template <typename T>
+__global__ void rmsnorm_kernel(const T* __restrict__ h, const T* __restrict__ w, int rows, int d,
+                               float eps, T* __restrict__ x) {
+  const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= rows) return;
+  const T* hr = h + static_cast<size_t>(r) * d;
+  T* xr = x + static_cast<size_t>(r) * d;
+  float ss = 0.f;
+  for (int i = lane; i < d; i += 32) {
+    float v = to_f(hr[i]);
+    ss += v * v;
+  }
+  ss = warp_sum(ss);
+  const float inv = rsqrtf(ss / static_cast<float>(d) + eps);
+  for (int i = lane; i < d; i += 32) xr[i] = from_f<T>(to_f(hr[i]) * inv * to_f(w[i]));
+}
+
+// bf16 rows, 8 elements per 16-byte vector.
+__global__ void rmsnorm_bf16_vec_kernel(const uint4* __restrict__ h, const uint4* __restrict__ w,
+                                        int rows, int vec_per_row, float eps,
+                                        uint4* __restrict__ x) {
+  const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= rows) return;
+  const uint4* hr = h + static_cast<size_t>(r) * vec_per_row;
+  uint4* xr = x + static_cast<size_t>(r) * vec_per_row;
+  float ss = 0.f;
+  for (int v = lane; v < vec_per_row; v += 32) {
+    uint4 u = hr[v];
+    const uint32_t p[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      float a = bf16lo(p[q]), b = bf16hi(p[q]);
+      ss += a * a + b * b;
+    }
+  }
+  ss = warp_sum(ss);
+  const float inv = rsqrtf(ss / static_cast<float>(vec_per_row * 8) + eps);
+  for (int v = lane; v < vec_per_row; v += 32) {
+    uint4 u = hr[v], wv = __ldg(w + v);
+    const uint32_t p[4] = {u.x, u.y, u.z, u.w};
+    const uint32_t q4[4] = {wv.x, wv.y, wv.z, wv.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      o[q] = pack_bf16x2(bf16lo(p[q]) * inv * bf16lo(q4[q]), bf16hi(p[q]) * inv * bf16hi(q4[q]));
+    xr[v] = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+// ---------------------------------------------------------------- scores
+
+// s[r] = ||h[r, :]||_2 for bf16 rows (the score with unit column mass, one group).
+template <int UNROLL>
+__global__ void row_norm_bf16_kernel(const uint4* __restrict__ h, int rows, int vec_per_row,
+                                     float* __restrict__ s) {
+  const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= rows) return;
+  const uint4* hr = h + static_cast<size_t>(r) * vec_per_row;
+  float ss = 0.f;
+  int v = lane;
+  for (; v + 32 * (UNROLL - 1) < vec_per_row; v += 32 * UNROLL) {
+    uint4 u[UNROLL];
+#pragma unroll
+    for (int q = 0; q < UNROLL; ++q) u[q] = __ldcs(hr + v + 32 * q);
+#pragma unroll
+    for (int q = 0; q < UNROLL; ++q) {
+      const uint32_t p[4] = {u[q].x, u[q].y, u[q].z, u[q].w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        float a = bf16lo(p[e]), b = bf16hi(p[e]);
+        ss = fmaf(a, a, ss);
+        ss = fmaf(b, b, ss);
+      }
+    }
+  }
+  for (; v < vec_per_row; v += 32) {
+    uint4 u = __ldcs(hr + v);
+    const uint32_t p[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      float a = bf16lo(p[e]), b = bf16hi(p[e]);
+      ss = fmaf(a, a, ss);
+      ss = fmaf(b, b, ss);
+    }
+  }
+  ss = warp_sum(ss);
+  if (lane == 0) s[r] = sqrtf(ss);
+}
+
+__global__ void row_norm_f32_kernel(const float* __restrict__ h, int rows, int d,
+                                    float* __restrict__ s) {
+  const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= rows) return;
+  const float* hr = h + static_cast<size_t>(r) * d;
+  float ss = 0.f;
+  for (int i = lane; i < d; i += 32) ss = fmaf(hr[i], hr[i], ss);
+  ss = warp_sum(ss);
+  if (lane == 0) s[r] = sqrtf(ss);
+}
+
+// s[b, j] = sum_g C[b, g, j] * ||v[b, j, g, :]||  (mode 0) or sum_g C[b, g, j] (mode 1)
+template <typename T>
+__global__ void score_colmass_kernel(const T* __restrict__ qkv, int ld, int v_off,
+                                     const float* __restrict__ C, int B, int N, int G, int hd,
+                                     int mode, float* __restrict__ s) {
+  const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= B * N) return;
+  const int b = r / N, j = r % N;
+  const T* v = qkv + static_cast<size_t>(r) * ld + v_off;
+  float acc = 0.f;
+  for (int g = 0; g < G; ++g) {
+    const float c = C[(static_cast<size_t>(b) * G + g) * N + j];
+    if (mode == ZSAA_SCORE_SOFTSCORE) {
+      acc += c;
+    } else {
+      float ss = 0.f;
+      for (int e = lane; e < hd; e += 32) {
+        float x = to_f(v[g * hd + e]);
+        ss = fmaf(x, x, ss);
+      }
+      ss = warp_sum(ss);
+      acc = fmaf(c, sqrtf(ss), acc);
+    }
+  }
+  if (lane == 0) s[r] = acc;
+}
+
+// ---------------------------------------------------------------- top-k select
+
+// Order-preserving map float -> uint32 (larger float -> larger key).  NaN maps
+// to 0, below every number; -0 is folded onto +0.
+__device__ __forceinline__ uint32_t order_key(float f) {
+  uint32_t u = __float_as_uint(f);
+  if (f != f) return 0u;
+  if (u == 0x80000000u) u = 0u;
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+constexpr int kSelThreads = 1024;
+
+// One block per sequence.  Radix select (4 passes of 8 bits) finds the key T of
+// the need-th best candidate and how many candidates equal to T are taken;
+// then an index-ordered ballot/prefix scan writes the kept indices ascending.
+// Ties (equal keys) keep lower indices first.  With force_last the last index
+// is kept and the other k-1 come from indices [0, N-1).
+__global__ void __launch_bounds__(kSelThreads)
+    select_topk_kernel(const float* __restrict__ scores, int N, int k, int force_last,
+                       int32_t* __restrict__ idx_out) {
+  const int b = blockIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  constexpr int nwarps = kSelThreads / 32;
+  const float* s = scores + static_cast<size_t>(b) * N;
+  int32_t* out = idx_out + static_cast<size_t>(b) * k;
+  const int n_cand = force_last ? N - 1 : N;
+  const int need = force_last ? k - 1 : k;
+
+  __shared__ uint32_t hist[256];
+  __shared__ uint32_t sh_digit, sh_remaining;
+  __shared__ int wgt[nwarps], weq[nwarps];
+  __shared__ int tile_gt, tile_eq;
+
+  uint32_t prefix = 0, mask = 0, remaining = static_cast<uint32_t>(need);
+  if (need > 0) {
+    for (int pass = 0; pass < 4; ++pass) {
+      const int shift = 24 - 8 * pass;
+      for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0;
+      __syncthreads();
+      for (int j = tid; j < n_cand; j += kSelThreads) {
+        const uint32_t key = order_key(s[j]);
+        if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+      }
+      __syncthreads();
+      if (warp == 0) {
+        uint32_t c[8], local = 0;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          c[q] = hist[lane * 8 + q];
+          local += c[q];
+        }
+        uint32_t suf = local;  // inclusive suffix sum over lanes
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          uint32_t v = __shfl_down_sync(0xffffffffu, suf, o);
+          if (lane + o < 32) suf += v;
+        }
+        uint32_t acc = suf - local;  // candidates in bins of higher lanes
+#pragma unroll
+        for (int q = 7; q >= 0; --q) {
+          if (acc < remaining && acc + c[q] >= remaining) {
+            sh_digit = static_cast<uint32_t>(lane * 8 + q);
+            sh_remaining = remaining - acc;
+          }
+          acc += c[q];
+        }
+      }
+      __syncthreads();
+      prefix |= sh_digit << shift;
+      mask |= 255u << shift;
+      remaining = sh_remaining;
+      __syncthreads();
+    }
+  }
+  const uint32_t T = prefix;
+  const uint32_t lt_mask = (1u << lane) - 1u;
+  int base_gt = 0, base_eq = 0;
+  for (int j0 = 0; j0 < n_cand && need > 0; j0 += kSelThreads) {
+    const int j = j0 + tid;
+    const bool in = j < n_cand;
+    const uint32_t key = in ? order_key(s[j]) : 0u;
+    const bool gt = in && key > T;
+    const bool eq = in && key == T;
+    const uint32_t bgt = __ballot_sync(0xffffffffu, gt), beq = __ballot_sync(0xffffffffu, eq);
+    if (lane == 0) {
+      wgt[warp] = __popc(bgt);
+      weq[warp] = __popc(beq);
+    }
+    __syncthreads();
+    if (warp == 0) {  // exclusive scan of the per-warp counts
+      int a = wgt[lane], e = weq[lane];
+      int ia = a, ie = e;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        int va = __shfl_up_sync(0xffffffffu, ia, o), ve = __shfl_up_sync(0xffffffffu, ie, o);
+        if (lane >= o) {
+          ia += va;
+          ie += ve;
+        }
+      }
+      wgt[lane] = ia - a;
+      weq[lane] = ie - e;
+      if (lane == 31) {
+        tile_gt = ia;
+        tile_eq = ie;
+      }
+    }
+    __syncthreads();
+    const int gt_before = base_gt + wgt[warp] + __popc(bgt & lt_mask);
+    const int eq_before = base_eq + weq[warp] + __popc(beq & lt_mask);
+    const int rem = static_cast<int>(remaining);
+    if (gt || (eq && eq_before < rem)) out[gt_before + min(eq_before, rem)] = j;
+    base_gt += tile_gt;
+    base_eq += tile_eq;
+    __syncthreads();
+  }
+  if (force_last && tid == 0) out[k - 1] = N - 1;
+}
+
+// ---------------------------------------------------------------- gather
+
+// dst[b*k + r, :] = src[b*N + idx[b*k + r], :]; pos_out likewise.  One warp per row.
+// An index outside [0, N) sets kStatusBadIndex and copies row 0 instead.
+template <int UNROLL>
+__global__ void gather_rows_kernel(const uint4* __restrict__ src, int N, int k, int vec_per_row,
+                                   const int32_t* __restrict__ idx, uint4* __restrict__ dst,
+                                   const int32_t* __restrict__ pos_in, int32_t* __restrict__ pos_out,
+                                   int total, int* status) {
+  const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= total) return;
+  const int b = r / k;
+  int j = idx[r];
+  if (j < 0 || j >= N) {
+    if (lane == 0 && status != nullptr) atomicOr(status, kStatusBadIndex);
+    j = 0;
+  }
+  const size_t srow = static_cast<size_t>(b) * N + j;
+  const uint4* s = src + srow * vec_per_row;
+  uint4* d = dst + static_cast<size_t>(r) * vec_per_row;
+  int v = lane;
+  for (; v + 32 * (UNROLL - 1) < vec_per_row; v += 32 * UNROLL) {
+    uint4 u[UNROLL];
+#pragma unroll
+    for (int q = 0; q < UNROLL; ++q) u[q] = s[v + 32 * q];
+#pragma unroll
+    for (int q = 0; q < UNROLL; ++q) __stcs(d + v + 32 * q, u[q]);
+  }
+  for (; v < vec_per_row; v += 32) __stcs(d + v, s[v]);
+  if (pos_out != nullptr && lane == 0) pos_out[r] = pos_in[srow];
+}
+
+// ---------------------------------------------------------------- RoPE (fp32 path)
+
+// Rotate pairs (c, c + hd/2) of every head in columns [0, rope_cols) of each row.
+__global__ void rope_f32_kernel(float* __restrict__ qkv, int rows, int ld, int rope_cols, int hd,
+                                const int32_t* __restrict__ pos, const float* __restrict__ cos_t,
+                                const float* __restrict__ sin_t) {
+  const int r = blockIdx.y;
+  const int half = hd / 2;
+  const int pairs = rope_cols / 2;
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= rows || t >= pairs) return;
+  const int head = t / half, c = t % half;
+  const int p = pos[r];
+  float* x = qkv + static_cast<size_t>(r) * ld + head * hd;
+  const float cs = cos_t[static_cast<size_t>(p) * half + c];
+  const float sn = sin_t[static_cast<size_t>(p) * half + c];
+  const float x1 = x[c], x2 = x[c + half];
+  x[c] = x1 * cs - x2 * sn;
+  x[c + half] = x2 * cs + x1 * sn;
+}
+
+// ---------------------------------------------------------------- classifier head
+
+// out[b, c] = sum_i xn[i] * W[c, i], xn = storage(rmsnorm(h[b, N-1]) * w)
+template <typename T>
+__global__ void cls_head_kernel(const T* __restrict__ h, int N, int d,
+                                const T* __restrict__ norm_w, float eps, const T* __restrict__ W,
+                                int n_classes, float* __restrict__ out) {
+  extern __shared__ float xs[];  // d floats
+  __shared__ float red[32];
+  const int b = blockIdx.x;
+  const T* row = h + (static_cast<size_t>(b) * N + (N - 1)) * d;
+  float ss = 0.f;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) {
+    float v = to_f(row[i]);
+    ss += v * v;
+  }
+  ss = warp_sum(ss);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    float v = threadIdx.x < blockDim.x / 32 ? red[threadIdx.x] : 0.f;
+    v = warp_sum(v);
+    if (threadIdx.x == 0) red[0] = v;
+  }
+  __syncthreads();
+  const float inv = rsqrtf(red[0] / static_cast<float>(d) + eps);
+  for (int i = threadIdx.x; i < d; i += blockDim.x)
+    xs[i] = to_f(from_f<T>(to_f(row[i]) * inv * to_f(norm_w[i])));
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int c = warp; c < n_classes; c += blockDim.x / 32) {
+    const T* wr = W + static_cast<size_t>(c) * d;
+    float acc = 0.f;
+    for (int i = lane; i < d; i += 32) acc = fmaf(xs[i], to_f(wr[i]), acc);
+    acc = warp_sum(acc);
+    if (lane == 0) out[static_cast<size_t>(b) * n_classes + c] = acc;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_embed(int dtype, const void* E, const int32_t* tok, int rows, int L, int vocab,
+                         int d, void* h, int32_t* pos, int* status, cudaStream_t s) {
+  const int esz = dtype == ZSAA_BF16 ? 2 : 4;
+  const int vec = d * esz / 16;
+  embed_kernel<<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
+      static_cast<const uint4*>(E), tok, rows, L, vocab, vec, static_cast<uint4*>(h), pos, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rmsnorm(int dtype, const void* h, const void* w, int rows, int d, float eps,
+                           void* x, cudaStream_t s) {
+  if (dtype == ZSAA_BF16 && d % 8 == 0) {
+    rmsnorm_bf16_vec_kernel<<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
+        static_cast<const uint4*>(h), static_cast<const uint4*>(w), rows, d / 8, eps,
+        static_cast<uint4*>(x));
+  } else if (dtype == ZSAA_BF16) {
+    rmsnorm_kernel<bf16><<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
+        static_cast<const bf16*>(h), static_cast<const bf16*>(w), rows, d, eps,
+        static_cast<bf16*>(x));
+  } else {
+    rmsnorm_kernel<float><<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
+        static_cast<const float*>(h), static_cast<const float*>(w), rows, d, eps,
+        static_cast<float*>(x));
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_row_norm(int dtype, const void* h, int rows, int d, float* scores,
+                            cudaStream_t s) {
+  if (dtype == ZSAA_BF16) {
+    row_norm_bf16_kernel<8><<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
+        static_cast<const uint4*>(h), rows, d / 8, scores);
+  } else {
+    row_norm_f32_kernel<<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
+        static_cast<const float*>(h), rows, d, scores);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_score_colmass(int dtype, const void* qkv, int ld, int v_off, const float* C,
+                                 int B, int N, int G, int hd, int mode, float* scores,
+                                 cudaStream_t s) {
+  const int rows = B * N;
+  if (dtype == ZSAA_BF16)
+    score_colmass_kernel<bf16><<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
+        static_cast<const bf16*>(qkv), ld, v_off, C, B, N, G, hd, mode, scores);
+  else
+    score_colmass_kernel<float><<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
+        static_cast<const float*>(qkv), ld, v_off, C, B, N, G, hd, mode, scores);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_select(const float* scores, int B, int N, int k, int force_last, int32_t* idx,
+                          cudaStream_t s) {
+  select_topk_kernel<<<B, kSelThreads, 0, s>>>(scores, N, k, force_last, idx);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const void* src, int B, int N, int k, int row_bytes, const int32_t* idx,
+                          void* dst, const int32_t* pos_in, int32_t* pos_out, int* status,
+                          cudaStream_t s) {
+  const int total = B * k;
+  gather_rows_kernel<4><<<row_blocks(total), 32 * kWarpsPerBlock, 0, s>>>(
+      static_cast<const uint4*>(src), N, k, row_bytes / 16, idx, static_cast<uint4*>(dst),
+      pos_in, pos_out, total, status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rope_f32(float* qkv, int rows, int ld, int rope_cols, int hd,
+                            const int32_t* pos, const float* cos_t, const float* sin_t,
+                            cudaStream_t s) {
+  const int pairs = rope_cols / 2;
+  dim3 grid((pairs + 127) / 128, rows);
+  rope_f32_kernel<<<grid, 128, 0, s>>>(qkv, rows, ld, rope_cols, hd, pos, cos_t, sin_t);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_cls_head(int dtype, const void* h, int B, int N, int d, const void* norm_w,
+                            float eps, const void* W, int n_classes, float* out, cudaStream_t s) {
+  const size_t smem = static_cast<size_t>(d) * sizeof(float);
+  if (dtype == ZSAA_BF16)
+    cls_head_kernel<bf16><<<B, 256, smem, s>>>(static_cast<const bf16*>(h), N, d,
+                                               static_cast<const bf16*>(norm_w), eps,
+                                               static_cast<const bf16*>(W), n_classes, out);
+  else
+    cls_head_kernel<float><<<B, 256, smem, s>>>(static_cast<const float*>(h), N, d,
+                                                static_cast<const float*>(norm_w), eps,
+                                                static_cast<const float*>(W), n_classes, out);
+  return cudaGetLastError();
+}
+
+}  // namespace zsaa

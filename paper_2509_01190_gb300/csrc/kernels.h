@@ -1,0 +1,77 @@
+// Host-side launchers of the library's kernels (internal; not part of the C ABI).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace zsaa {
+
+// ---- row kernels (k_rows.cu)
+cudaError_t launch_embed(int dtype, const void* E, const int32_t* tok, int rows, int L, int vocab,
+                         int d, void* h, int32_t* pos, int* status, cudaStream_t s);
+cudaError_t launch_rmsnorm(int dtype, const void* h, const void* w, int rows, int d, float eps,
+                           void* x, cudaStream_t s);
+cudaError_t launch_row_norm(int dtype, const void* h, int rows, int d, float* scores,
+                            cudaStream_t s);
+cudaError_t launch_score_colmass(int dtype, const void* qkv, int ld, int v_off, const float* C,
+                                 int B, int N, int G, int hd, int mode, float* scores,
+                                 cudaStream_t s);
+cudaError_t launch_select(const float* scores, int B, int N, int k, int force_last, int32_t* idx,
+                          cudaStream_t s);
+cudaError_t launch_gather(const void* src, int B, int N, int k, int row_bytes, const int32_t* idx,
+                          void* dst, const int32_t* pos_in, int32_t* pos_out, int* status,
+                          cudaStream_t s);
+cudaError_t launch_rope_f32(float* qkv, int rows, int ld, int rope_cols, int hd,
+                            const int32_t* pos, const float* cos_t, const float* sin_t,
+                            cudaStream_t s);
+cudaError_t launch_cls_head(int dtype, const void* h, int B, int N, int d, const void* norm_w,
+                            float eps, const void* W, int n_classes, float* out, cudaStream_t s);
+
+// ---- GEMMs (k_gemm_tc.cu, k_gemm_simt.cu)
+enum Epilogue : int { kEpiStore = 0, kEpiResid = 1, kEpiSwiGLU = 2, kEpiStoreF32 = 3, kEpiRope = 4 };
+
+struct GemmParams {
+  int M, N, K;
+  void* out;            // [M, ldo] (N columns used; SwiGLU: N = output columns)
+  int ldo;
+  const void* resid;    // kEpiResid: [M, ldo]
+  const int32_t* pos;   // kEpiRope: position of each row
+  const float* cos_t;   // kEpiRope: [positions, hd/2]
+  const float* sin_t;
+  int rope_cols;        // kEpiRope: columns [0, rope_cols) are rotated
+  int hd;               // kEpiRope: head size
+  int* status;          // device status word
+};
+
+// bf16 tensor-core GEMM: out = epi(A[M,K] * W^T).  W is given as up to three
+// row blocks (w0: rows [0, n1), w1: rows [n1, n2), w2: rows [n2, N)) so the
+// QKV projection reads separate Wq/Wk/Wv; SwiGLU passes gate in w0 and up in
+// w1 with n1 = N.
+struct TcWeights {
+  const void* w0;
+  const void* w1;
+  const void* w2;
+  int n1, n2;
+};
+cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
+                           const GemmParams& p, cudaStream_t s);
+
+// fp32 CUDA-core GEMM, same epilogues (kEpiRope is applied by launch_rope_f32).
+cudaError_t launch_gemm_f32(const float* A, int lda, const float* W, const float* W2, int epi,
+                            const GemmParams& p, cudaStream_t s);
+
+// ---- attention (k_attn.cu)
+cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, int Hkv, int hd,
+                             void* out, float* lse, cudaStream_t s);
+cudaError_t launch_colmass(int dtype, const void* qkv, const float* lse, int B, int N, int Hq,
+                           int Hkv, int hd, float* C, cudaStream_t s);
+
+// ---- driver entry point for tensor maps (zsaa_api.cu)
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn get_encode_tiled();
+
+}  // namespace zsaa

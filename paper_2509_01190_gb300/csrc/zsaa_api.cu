@@ -1,0 +1,866 @@
+// C ABI of the pruned-prefill library: planner (Eq. 2, Sec. 3.4), model
+// workspace, and the stream-ordered forward pass that chains the kernels.
+//
+// Forward pass of one call (Sec. 3.3): embed -> for each layer l on N_{l-1}
+// rows: RMSNorm, QKV GEMM with RoPE at original positions, causal GQA
+// attention, O GEMM + residual, RMSNorm, gate/up GEMM with SwiGLU, down GEMM
+// + residual; if layer l prunes and N_l < N_{l-1}: column mass, scores, top-k,
+// gather of the residual rows and their positions -> final RMSNorm + head.
+// The schedule is computed on the host before any launch; there is no
+// host/device synchronisation inside a forward.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <unordered_map>
+#include <vector>
+
+#include "common.cuh"
+#include "kernels.h"
+
+using namespace zsaa;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+zsaa_status fail(zsaa_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return st;
+}
+
+#define ZCK(expr)                                                                        \
+  do {                                                                                   \
+    cudaError_t e_ = (expr);                                                             \
+    if (e_ != cudaSuccess)                                                               \
+      return fail(ZSAA_ERR_CUDA, "%s failed: %s (%s:%d)", #expr, cudaGetErrorString(e_), \
+                  __FILE__, __LINE__);                                                   \
+  } while (0)
+
+// ---------------------------------------------------------------- planner
+
+bool prunes(const zsaa_config& c, int layer) { return (c.prune_mask >> (layer - 1)) & 1ull; }
+
+// Eq. 2: N_l = min(N_{l-1}, max(floor(alpha N_{l-1}), min(tau, N_{l-1}))) after a pruning layer.
+void eq2_schedule(const zsaa_config& c, int L, double alpha, int* out) {
+  out[0] = L;
+  for (int l = 1; l <= c.n_layers; ++l) {
+    const int prev = out[l - 1];
+    if (prunes(c, l)) {
+      long long nl = static_cast<long long>(std::floor(alpha * static_cast<double>(prev)));
+      const long long floor_rows = prev < c.tau ? prev : c.tau;
+      if (nl < floor_rows) nl = floor_rows;
+      out[l] = static_cast<int>(nl < prev ? nl : prev);
+    } else {
+      out[l] = prev;
+    }
+  }
+}
+
+// Modelled FLOPs of one sequence: linear layers + causal attention + head.
+long long model_cost(const zsaa_config& c, const int* sched) {
+  const long long d = c.d_model, hd = c.head_dim, dq = static_cast<long long>(c.n_heads) * hd;
+  const long long f = 2 * d * (dq + 2LL * c.n_kv_heads * hd) + 2 * dq * d + 6 * d * c.ffn_dim;
+  long long total = 0;
+  for (int l = 0; l < c.n_layers; ++l) {
+    const long long n = sched[l];
+    total += n * f + 2 * n * n * dq;
+  }
+  if (c.n_classes > 0)
+    total += 2 * d * c.n_classes;
+  else
+    total += static_cast<long long>(sched[c.n_layers]) * 2 * d * c.vocab;
+  return total;
+}
+
+zsaa_status plan_impl(const zsaa_config& c, int L, double accel, int* sched, double* alpha_out) {
+  if (!(accel >= 1.0)) return fail(ZSAA_ERR_INVALID_ARG, "accel must be >= 1 (got %g)", accel);
+  if (L < 1) return fail(ZSAA_ERR_INVALID_ARG, "L must be >= 1");
+  double alpha = 1.0;
+  if (c.plan_mode == ZSAA_PLAN_RATE) {
+    alpha = 1.0 / accel;
+  } else if (accel != 1.0) {
+    std::vector<int> s(c.n_layers + 1);
+    eq2_schedule(c, L, 1.0, s.data());
+    const double target = static_cast<double>(model_cost(c, s.data())) / accel;
+    double lo = 0.0, hi = 1.0;
+    for (int it = 0; it < 60; ++it) {
+      const double mid = 0.5 * (lo + hi);
+      eq2_schedule(c, L, mid, s.data());
+      if (static_cast<double>(model_cost(c, s.data())) <= target)
+        lo = mid;
+      else
+        hi = mid;
+    }
+    alpha = lo;
+  }
+  eq2_schedule(c, L, alpha, sched);
+  if (alpha_out) *alpha_out = alpha;
+  return ZSAA_OK;
+}
+
+zsaa_status validate_config(const zsaa_config& c) {
+  if (c.n_layers < 1 || c.n_layers > 64) return fail(ZSAA_ERR_INVALID_ARG, "n_layers must be 1..64");
+  if (c.dtype != ZSAA_F32 && c.dtype != ZSAA_BF16) return fail(ZSAA_ERR_INVALID_ARG, "bad dtype");
+  if (c.n_heads < 1 || c.n_kv_heads < 1 || c.n_heads % c.n_kv_heads != 0)
+    return fail(ZSAA_ERR_INVALID_ARG, "n_heads must be a positive multiple of n_kv_heads");
+  if (c.head_dim < 2 || c.head_dim % 2 != 0 || c.head_dim > 128)
+    return fail(ZSAA_ERR_INVALID_ARG, "head_dim must be even and <= 128");
+  if (c.d_model < 8 || c.d_model % 8 != 0 || c.ffn_dim < 1 || c.vocab < 1)
+    return fail(ZSAA_ERR_INVALID_ARG, "bad d_model / ffn_dim / vocab");
+  if (c.tau < 1) return fail(ZSAA_ERR_INVALID_ARG, "tau must be >= 1");
+  if (c.n_classes < 0) return fail(ZSAA_ERR_INVALID_ARG, "n_classes must be >= 0");
+  if (c.score_mode != ZSAA_SCORE_SOFTSCORE_VNORM && c.score_mode != ZSAA_SCORE_SOFTSCORE)
+    return fail(ZSAA_ERR_INVALID_ARG, "bad score_mode");
+  if (c.plan_mode != ZSAA_PLAN_COST && c.plan_mode != ZSAA_PLAN_RATE)
+    return fail(ZSAA_ERR_INVALID_ARG, "bad plan_mode");
+  if (c.n_layers < 64 && (c.prune_mask >> c.n_layers) != 0)
+    return fail(ZSAA_ERR_INVALID_ARG, "prune_mask names layers beyond n_layers");
+  if (c.dtype == ZSAA_BF16) {
+    const int dq = c.n_heads * c.head_dim;
+    if (c.head_dim != 64 && c.head_dim != 128)
+      return fail(ZSAA_ERR_UNSUPPORTED, "bf16 models need head_dim 64 or 128");
+    if (c.d_model % 64 || dq % 64 || c.ffn_dim % 64)
+      return fail(ZSAA_ERR_UNSUPPORTED, "bf16 models need d_model, heads*head_dim, ffn_dim % 64 == 0");
+    if ((c.n_kv_heads * c.head_dim) % 64)
+      return fail(ZSAA_ERR_UNSUPPORTED, "bf16 models need kv_heads*head_dim % 64 == 0");
+    if (c.n_classes == 0 && c.vocab % 16)
+      return fail(ZSAA_ERR_UNSUPPORTED, "bf16 LM head needs vocab % 16 == 0");
+  } else if (c.d_model % 4) {
+    return fail(ZSAA_ERR_UNSUPPORTED, "f32 models need d_model % 4 == 0");
+  }
+  return ZSAA_OK;
+}
+
+// ---------------------------------------------------------------- device helpers
+
+EncodeTiledFn g_encode = nullptr;
+std::once_flag g_encode_once;
+
+std::mutex g_status_mu;
+std::unordered_map<int, int*> g_status_by_dev;  // shared status word of model-less calls
+
+int* shared_status() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
+  std::lock_guard<std::mutex> lk(g_status_mu);
+  auto it = g_status_by_dev.find(dev);
+  if (it != g_status_by_dev.end()) return it->second;
+  int* p = nullptr;
+  if (cudaMalloc(&p, sizeof(int)) != cudaSuccess) return nullptr;
+  if (cudaMemset(p, 0, sizeof(int)) != cudaSuccess) return nullptr;
+  g_status_by_dev[dev] = p;
+  return p;
+}
+
+// RoPE tables of zsaa_op_linear, cached per (device, theta, head size):
+// positions 0 .. kOpRopePositions-1.
+constexpr int kOpRopePositions = 16384;
+struct RopeTable {
+  float* cos_t;
+  float* sin_t;
+};
+std::mutex g_rope_mu;
+std::unordered_map<std::string, RopeTable> g_rope_tables;
+
+bool op_rope_table(float theta, int hd, RopeTable* out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  char key[96];
+  snprintf(key, sizeof(key), "%d/%.9g/%d", dev, static_cast<double>(theta), hd);
+  std::lock_guard<std::mutex> lk(g_rope_mu);
+  auto it = g_rope_tables.find(key);
+  if (it != g_rope_tables.end()) {
+    *out = it->second;
+    return true;
+  }
+  const int half = hd / 2;
+  std::vector<float> c(static_cast<size_t>(kOpRopePositions) * half), sv(c.size());
+  for (int q = 0; q < kOpRopePositions; ++q)
+    for (int i = 0; i < half; ++i) {
+      const double a = static_cast<double>(q) *
+                       std::pow(static_cast<double>(theta), -2.0 * i / static_cast<double>(hd));
+      c[static_cast<size_t>(q) * half + i] = static_cast<float>(std::cos(a));
+      sv[static_cast<size_t>(q) * half + i] = static_cast<float>(std::sin(a));
+    }
+  RopeTable t{nullptr, nullptr};
+  if (cudaMalloc(&t.cos_t, c.size() * 4) != cudaSuccess) return false;
+  if (cudaMalloc(&t.sin_t, c.size() * 4) != cudaSuccess) return false;
+  if (cudaMemcpy(t.cos_t, c.data(), c.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess) return false;
+  if (cudaMemcpy(t.sin_t, sv.data(), c.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess) return false;
+  g_rope_tables[key] = t;
+  *out = t;
+  return true;
+}
+
+}  // namespace
+
+namespace zsaa {
+EncodeTiledFn get_encode_tiled() {
+  std::call_once(g_encode_once, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<EncodeTiledFn>(fn);
+  });
+  return g_encode;
+}
+}  // namespace zsaa
+
+// ---------------------------------------------------------------- model
+
+struct zsaa_model {
+  zsaa_config cfg;
+  int max_B = 0, max_L = 0;
+  int device = 0;
+  const void* embed = nullptr;
+  const void* final_norm = nullptr;
+  const void* head = nullptr;
+  std::vector<const void*> layers;  // n_layers * 9
+  size_t esz = 2;
+  int ld_qkv = 0, dq = 0, dkv = 0;
+  // workspace
+  void* h[2] = {nullptr, nullptr};
+  void* x = nullptr;
+  void* qkv = nullptr;
+  void* attn = nullptr;
+  void* act = nullptr;
+  float* lse = nullptr;
+  float* colmass = nullptr;
+  float* scores = nullptr;
+  int32_t* idx = nullptr;
+  int32_t* pos[2] = {nullptr, nullptr};
+  float* rope_cos = nullptr;
+  float* rope_sin = nullptr;
+  int* status = nullptr;
+  // host-buffer staging (zsaa_forward_host)
+  int32_t* stage_tok = nullptr;
+  float* stage_logits = nullptr;
+  int32_t* stage_pos = nullptr;
+  size_t stage_logits_cap = 0;
+  // tracing (zsaa_trace_begin / _end)
+  struct TraceRec {
+    int cls;
+    cudaEvent_t a, b;
+    double flops, bytes;
+  };
+  bool tracing = false;
+  std::vector<TraceRec> trace;
+  std::vector<cudaEvent_t> ev_pool;
+  size_t ev_used = 0;
+  std::vector<std::string> trace_names;
+};
+
+namespace {
+
+const void* LW(const zsaa_model* m, int layer, int slot) {
+  return m->layers[static_cast<size_t>(layer) * 9 + slot];
+}
+enum { kAttnNorm = 0, kWq, kWk, kWv, kWo, kMlpNorm, kWg, kWu, kWd };
+
+// Brackets one kernel launch with events while the model is tracing.
+class TraceScope {
+ public:
+  TraceScope(zsaa_model* m, const char* name, double flops, double bytes, cudaStream_t s)
+      : m_(m), s_(s) {
+    if (!m->tracing) return;
+    int cls = -1;
+    for (size_t i = 0; i < m->trace_names.size(); ++i)
+      if (m->trace_names[i] == name) cls = static_cast<int>(i);
+    if (cls < 0) {
+      cls = static_cast<int>(m->trace_names.size());
+      m->trace_names.push_back(name);
+    }
+    rec_.cls = cls;
+    rec_.flops = flops;
+    rec_.bytes = bytes;
+    rec_.a = event();
+    rec_.b = event();
+    if (rec_.a && rec_.b && cudaEventRecord(rec_.a, s) == cudaSuccess) active_ = true;
+  }
+  ~TraceScope() {
+    if (active_ && cudaEventRecord(rec_.b, s_) == cudaSuccess) m_->trace.push_back(rec_);
+  }
+
+ private:
+  cudaEvent_t event() {
+    if (m_->ev_used == m_->ev_pool.size()) {
+      cudaEvent_t e = nullptr;
+      if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+      m_->ev_pool.push_back(e);
+    }
+    return m_->ev_pool[m_->ev_used++];
+  }
+  zsaa_model* m_;
+  cudaStream_t s_;
+  zsaa_model::TraceRec rec_{};
+  bool active_ = false;
+};
+
+void free_model(zsaa_model* m) {
+  if (m == nullptr) return;
+  for (cudaEvent_t e : m->ev_pool) cudaEventDestroy(e);
+  void* ptrs[] = {m->h[0], m->h[1], m->x, m->qkv, m->attn, m->act, m->lse, m->colmass,
+                  m->scores, m->idx, m->pos[0], m->pos[1], m->rope_cos, m->rope_sin,
+                  m->status, m->stage_tok, m->stage_logits, m->stage_pos};
+  for (void* p : ptrs)
+    if (p) cudaFree(p);
+  delete m;
+}
+
+// out[M, N] = epi(A W^T) on the model's dtype path.
+zsaa_status linear(zsaa_model* m, const void* A, int lda, const TcWeights& W, int epi,
+                   GemmParams p, cudaStream_t s) {
+  p.status = m->status;
+  if (m->cfg.dtype == ZSAA_BF16) {
+    ZCK(launch_gemm_tc(A, lda, W, epi, p, s));
+  } else {
+    if (epi == kEpiRope) return fail(ZSAA_ERR_UNSUPPORTED, "f32 RoPE epilogue");
+    ZCK(launch_gemm_f32(static_cast<const float*>(A), lda, static_cast<const float*>(W.w0),
+                        static_cast<const float*>(W.w1), epi, p, s));
+  }
+  return ZSAA_OK;
+}
+
+zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double accel,
+                        float* logits, int32_t* kept_pos, const zsaa_forward_opts* opts,
+                        cudaStream_t s) {
+  const zsaa_config& c = m->cfg;
+  if (tok == nullptr || logits == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null token or logits pointer");
+  if (B < 1 || B > m->max_B || L < 1 || L > m->max_L)
+    return fail(ZSAA_ERR_INVALID_ARG, "B=%d L=%d outside [1,%d] x [1,%d]", B, L, m->max_B, m->max_L);
+  const int n_run = (opts && opts->n_layers_run > 0) ? opts->n_layers_run : c.n_layers;
+  if (n_run > c.n_layers) return fail(ZSAA_ERR_INVALID_ARG, "n_layers_run > n_layers");
+  std::vector<int> sched(c.n_layers + 1);
+  double alpha = 1.0;
+  zsaa_status st = plan_impl(c, L, accel, sched.data(), &alpha);
+  if (st != ZSAA_OK) return st;
+
+  const int d = c.d_model, hd = c.head_dim, Hq = c.n_heads, Hkv = c.n_kv_heads;
+  const int dt = c.dtype;
+  int cur = 0;
+  const double es = static_cast<double>(m->esz);
+#define TRACE(name, fl, by) TraceScope trace_scope_(m, name, fl, by, s)
+  {
+    TRACE("embed", 0.0, static_cast<double>(B) * L * (d * es + 8.0));
+    ZCK(launch_embed(dt, m->embed, tok, B * L, L, c.vocab, d, m->h[cur], m->pos[cur], m->status, s));
+  }
+  size_t off_forced = 0, off_scores = 0, off_idx = 0;
+  int N = L;
+  for (int l = 1; l <= n_run; ++l) {
+    const int li = l - 1;
+    const int M = B * N;
+    void* h = m->h[cur];
+    const double Md = static_cast<double>(M);
+    // attention branch
+    {
+      TRACE("rmsnorm", 0.0, 2.0 * Md * d * es);
+      ZCK(launch_rmsnorm(dt, h, LW(m, li, kAttnNorm), M, d, c.rms_eps, m->x, s));
+    }
+    GemmParams p{};
+    p.M = M;
+    p.K = d;
+    p.out = m->qkv;
+    p.ldo = m->ld_qkv;
+    if (dt == ZSAA_BF16) {
+      p.N = m->ld_qkv;
+      p.pos = m->pos[cur];
+      p.cos_t = m->rope_cos;
+      p.sin_t = m->rope_sin;
+      p.rope_cols = m->dq + m->dkv;
+      p.hd = hd;
+      TcWeights W{LW(m, li, kWq), LW(m, li, kWk), LW(m, li, kWv), m->dq, m->dq + m->dkv};
+      TRACE("gemm_qkv_rope", 2.0 * Md * m->ld_qkv * d, (Md * d + static_cast<double>(m->ld_qkv) * d + Md * m->ld_qkv) * es);
+      st = linear(m, m->x, d, W, kEpiRope, p, s);
+      if (st != ZSAA_OK) return st;
+    } else {
+      TRACE("gemm_qkv_f32", 2.0 * Md * m->ld_qkv * d, (Md * d + static_cast<double>(m->ld_qkv) * d + Md * m->ld_qkv) * es);
+      const int cols[3] = {m->dq, m->dkv, m->dkv};
+      const int slots[3] = {kWq, kWk, kWv};
+      int c0 = 0;
+      for (int t = 0; t < 3; ++t) {
+        GemmParams q = p;
+        q.N = cols[t];
+        q.out = static_cast<float*>(m->qkv) + c0;
+        TcWeights W{LW(m, li, slots[t]), nullptr, nullptr, cols[t], cols[t]};
+        st = linear(m, m->x, d, W, kEpiStore, q, s);
+        if (st != ZSAA_OK) return st;
+        c0 += cols[t];
+      }
+      ZCK(launch_rope_f32(static_cast<float*>(m->qkv), M, m->ld_qkv, m->dq + m->dkv, hd,
+                          m->pos[cur], m->rope_cos, m->rope_sin, s));
+    }
+    {
+      const double pairs = static_cast<double>(B) * Hq * (static_cast<double>(N) * (N + 1) / 2.0);
+      TRACE("attention", 4.0 * pairs * hd, Md * (m->ld_qkv + m->dq) * es + static_cast<double>(B) * Hq * N * 4.0);
+      ZCK(launch_attention(dt, m->qkv, B, N, Hq, Hkv, hd, m->attn, m->lse, s));
+    }
+    {
+      GemmParams q{};
+      q.M = M;
+      q.N = d;
+      q.K = m->dq;
+      q.out = h;
+      q.ldo = d;
+      q.resid = h;
+      TcWeights W{LW(m, li, kWo), nullptr, nullptr, d, d};
+      TRACE("gemm_o_resid", 2.0 * Md * d * m->dq, (Md * m->dq + static_cast<double>(d) * m->dq + 2.0 * Md * d) * es);
+      st = linear(m, m->attn, m->dq, W, kEpiResid, q, s);
+      if (st != ZSAA_OK) return st;
+    }
+    // MLP branch
+    {
+      TRACE("rmsnorm", 0.0, 2.0 * Md * d * es);
+      ZCK(launch_rmsnorm(dt, h, LW(m, li, kMlpNorm), M, d, c.rms_eps, m->x, s));
+    }
+    {
+      GemmParams q{};
+      q.M = M;
+      q.N = c.ffn_dim;
+      q.K = d;
+      q.out = m->act;
+      q.ldo = c.ffn_dim;
+      TcWeights W{LW(m, li, kWg), LW(m, li, kWu), nullptr, c.ffn_dim, c.ffn_dim};
+      const double F = c.ffn_dim;
+      TRACE("gemm_gate_up_swiglu", 4.0 * Md * F * d, (Md * d + 2.0 * F * d + Md * F) * es);
+      st = linear(m, m->x, d, W, kEpiSwiGLU, q, s);
+      if (st != ZSAA_OK) return st;
+    }
+    {
+      GemmParams q{};
+      q.M = M;
+      q.N = d;
+      q.K = c.ffn_dim;
+      q.out = h;
+      q.ldo = d;
+      q.resid = h;
+      TcWeights W{LW(m, li, kWd), nullptr, nullptr, d, d};
+      const double F = c.ffn_dim;
+      TRACE("gemm_down_resid", 2.0 * Md * d * F, (Md * F + F * d + 2.0 * Md * d) * es);
+      st = linear(m, m->act, c.ffn_dim, W, kEpiResid, q, s);
+      if (st != ZSAA_OK) return st;
+    }
+    // elimination after the layer (Sec. 3.3)
+    if (prunes(c, l)) {
+      const int k = sched[l];
+      const bool want_scores = opts && opts->scores_out;
+      const bool forced = opts && opts->forced_idx;
+      const bool want_idx = opts && opts->idx_out;
+      if (k < N || want_scores || want_idx) {
+        float* sc = want_scores ? opts->scores_out + off_scores : m->scores;
+        {
+          const double pairs = static_cast<double>(B) * Hq * (static_cast<double>(N) * (N + 1) / 2.0);
+          TRACE("colmass", 2.0 * pairs * hd,
+                Md * (m->dq + m->dkv) * es + static_cast<double>(B) * (Hq + Hkv) * N * 4.0);
+          ZCK(launch_colmass(dt, m->qkv, m->lse, B, N, Hq, Hkv, hd, m->colmass, s));
+        }
+        {
+          TRACE("score", 0.0, Md * m->dkv * es + Md * (Hkv + 1) * 4.0);
+          ZCK(launch_score_colmass(dt, m->qkv, m->ld_qkv, m->dq + m->dkv, m->colmass, B, N, Hkv, hd,
+                                   c.score_mode, sc, s));
+        }
+        const int32_t* idx = m->idx;
+        if (forced) {
+          idx = opts->forced_idx + off_forced;
+        } else {  // with k == N (only when idx_out is requested) this yields 0..N-1
+          TRACE("select", 0.0, Md * 4.0 + static_cast<double>(B) * k * 4.0);
+          ZCK(launch_select(sc, B, N, k, c.force_keep_last, m->idx, s));
+        }
+        if (want_idx)
+          ZCK(cudaMemcpyAsync(opts->idx_out + off_idx, idx, sizeof(int32_t) * B * k,
+                              cudaMemcpyDeviceToDevice, s));
+        if (k < N) {
+          TRACE("gather", 0.0, static_cast<double>(B) * k * (2.0 * d * es + 12.0));
+          ZCK(launch_gather(h, B, N, k, static_cast<int>(d * m->esz), idx, m->h[cur ^ 1],
+                            m->pos[cur], m->pos[cur ^ 1], m->status, s));
+          cur ^= 1;
+        }
+      }
+      off_forced += static_cast<size_t>(B) * k;
+      off_idx += static_cast<size_t>(B) * k;
+      off_scores += static_cast<size_t>(B) * N;
+      N = k;
+    }
+  }
+  // head
+  const int M = B * N;
+  if (opts && opts->hidden_out)
+    ZCK(cudaMemcpyAsync(opts->hidden_out, m->h[cur], M * d * m->esz, cudaMemcpyDeviceToDevice, s));
+  if (c.n_classes > 0) {
+    TRACE("cls_head", 2.0 * B * d * c.n_classes, (static_cast<double>(B) * d + static_cast<double>(c.n_classes) * d) * es);
+    ZCK(launch_cls_head(dt, m->h[cur], B, N, d, m->final_norm, c.rms_eps, m->head, c.n_classes,
+                        logits, s));
+  } else {
+    {
+      TRACE("rmsnorm", 0.0, 2.0 * static_cast<double>(M) * d * es);
+      ZCK(launch_rmsnorm(dt, m->h[cur], m->final_norm, M, d, c.rms_eps, m->x, s));
+    }
+    GemmParams q{};
+    q.M = M;
+    q.N = c.vocab;
+    q.K = d;
+    q.out = logits;
+    q.ldo = c.vocab;
+    TcWeights W{m->head, nullptr, nullptr, c.vocab, c.vocab};
+    const double V = c.vocab, Mh = M;
+    TRACE("gemm_lm_head", 2.0 * Mh * V * d, (Mh * d + V * d) * es + Mh * V * 4.0);
+    st = linear(m, m->x, d, W, dt == ZSAA_BF16 ? kEpiStoreF32 : kEpiStore, q, s);
+    if (st != ZSAA_OK) return st;
+  }
+  if (kept_pos)
+    ZCK(cudaMemcpyAsync(kept_pos, m->pos[cur], sizeof(int32_t) * M, cudaMemcpyDeviceToDevice, s));
+#undef TRACE
+  return ZSAA_OK;
+}
+
+zsaa_status score_select_impl(const void* hidden, int B, int L, int d, int dtype, int k, int flags,
+                              const float* scores_in, float* scores_out, int32_t* idx_out,
+                              void* gathered_out, cudaStream_t s) {
+  if (hidden == nullptr || idx_out == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null hidden or idx_out");
+  if (B < 1 || L < 1 || d < 1) return fail(ZSAA_ERR_INVALID_ARG, "B, L, d must be >= 1");
+  if (k < 1 || k > L) return fail(ZSAA_ERR_INVALID_ARG, "k=%d outside [1, L=%d]", k, L);
+  if (dtype != ZSAA_BF16 && dtype != ZSAA_F32) return fail(ZSAA_ERR_INVALID_ARG, "bad dtype");
+  const int esz = dtype == ZSAA_BF16 ? 2 : 4;
+  if ((static_cast<size_t>(d) * esz) % 16 != 0)
+    return fail(ZSAA_ERR_INVALID_ARG, "row bytes d*%d must be a multiple of 16", esz);
+  if ((reinterpret_cast<uintptr_t>(hidden) | reinterpret_cast<uintptr_t>(gathered_out)) % 16)
+    return fail(ZSAA_ERR_INVALID_ARG, "hidden and gathered_out must be 16-byte aligned");
+  if (static_cast<long long>(B) * L > (1LL << 31) - 1)
+    return fail(ZSAA_ERR_INVALID_ARG, "B*L too large");
+  const int force_last = (flags & ZSAA_FLAG_FORCE_KEEP_LAST) ? 1 : 0;
+  float* scratch = nullptr;
+  const float* sc = scores_in;
+  if (sc == nullptr) {
+    float* dst = scores_out;
+    if (dst == nullptr) {
+      ZCK(cudaMallocAsync(reinterpret_cast<void**>(&scratch), sizeof(float) * B * L, s));
+      dst = scratch;
+    }
+    ZCK(launch_row_norm(dtype, hidden, B * L, d, dst, s));
+    sc = dst;
+  } else if (scores_out != nullptr) {
+    ZCK(cudaMemcpyAsync(scores_out, scores_in, sizeof(float) * B * L, cudaMemcpyDeviceToDevice, s));
+  }
+  cudaError_t e = launch_select(sc, B, L, k, force_last, idx_out, s);
+  if (e == cudaSuccess && gathered_out != nullptr)
+    e = launch_gather(hidden, B, L, k, d * esz, idx_out, gathered_out, nullptr, nullptr, nullptr, s);
+  if (scratch) {
+    cudaError_t e2 = cudaFreeAsync(scratch, s);
+    if (e == cudaSuccess) e = e2;
+  }
+  ZCK(e);
+  return ZSAA_OK;
+}
+
+zsaa_status read_status(int* word, cudaStream_t s, bool whole_device) {
+  if (whole_device)
+    ZCK(cudaDeviceSynchronize());
+  else
+    ZCK(cudaStreamSynchronize(s));
+  int v = 0;
+  ZCK(cudaMemcpy(&v, word, sizeof(int), cudaMemcpyDeviceToHost));
+  if (v != 0) {
+    ZCK(cudaMemset(word, 0, sizeof(int)));
+    if (v & kStatusTimeout)
+      return fail(ZSAA_ERR_TIMEOUT, "a kernel gave up a bounded wait (status 0x%x)", v);
+    return fail(ZSAA_ERR_INVALID_ARG, "a token id or forced index was out of range (status 0x%x)", v);
+  }
+  return ZSAA_OK;
+}
+
+}  // namespace
+
+// ================================================================ C ABI
+
+extern "C" {
+
+const char* zsaa_last_error(void) { return g_last_error.c_str(); }
+
+const char* zsaa_version(void) { return "zsaa 0.1 (sm_103a)"; }
+
+zsaa_status zsaa_plan_config(const zsaa_config* cfg, int L, double accel, int* n_sched,
+                             double* alpha_out) {
+  if (cfg == nullptr || n_sched == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null argument");
+  zsaa_status st = validate_config(*cfg);
+  if (st != ZSAA_OK) return st;
+  return plan_impl(*cfg, L, accel, n_sched, alpha_out);
+}
+
+zsaa_status zsaa_model_create(const zsaa_config* cfg, const zsaa_weights* w, int max_B, int max_L,
+                              zsaa_model** out) {
+  if (out == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null out");
+  *out = nullptr;
+  if (cfg == nullptr || w == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null config or weights");
+  zsaa_status st = validate_config(*cfg);
+  if (st != ZSAA_OK) return st;
+  if (max_B < 1 || max_L < 1) return fail(ZSAA_ERR_INVALID_ARG, "max_B and max_L must be >= 1");
+  if (w->embed == nullptr || w->layers == nullptr || w->final_norm == nullptr || w->head == nullptr)
+    return fail(ZSAA_ERR_INVALID_ARG, "null weight pointer");
+  const size_t esz = cfg->dtype == ZSAA_BF16 ? 2 : 4;
+  for (int i = 0; i < cfg->n_layers * 9; ++i) {
+    const void* p = w->layers[i];
+    if (p == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null layer weight %d", i);
+    if (reinterpret_cast<uintptr_t>(p) % 16) return fail(ZSAA_ERR_INVALID_ARG, "layer weight %d not 16-byte aligned", i);
+  }
+  const long long rows = static_cast<long long>(max_B) * max_L;
+  if (rows > (1LL << 30)) return fail(ZSAA_ERR_INVALID_ARG, "max_B*max_L too large");
+
+  zsaa_model* m = new zsaa_model();
+  m->cfg = *cfg;
+  m->max_B = max_B;
+  m->max_L = max_L;
+  cudaGetDevice(&m->device);
+  m->embed = w->embed;
+  m->final_norm = w->final_norm;
+  m->head = w->head;
+  m->layers.assign(w->layers, w->layers + cfg->n_layers * 9);
+  m->esz = esz;
+  m->dq = cfg->n_heads * cfg->head_dim;
+  m->dkv = cfg->n_kv_heads * cfg->head_dim;
+  m->ld_qkv = m->dq + 2 * m->dkv;
+
+  const size_t d = cfg->d_model, F = cfg->ffn_dim;
+  bool ok = true;
+  auto alloc = [&](void** p, size_t bytes) {
+    if (ok && cudaMalloc(p, bytes + 16) != cudaSuccess) ok = false;
+  };
+  alloc(&m->h[0], rows * d * esz);
+  alloc(&m->h[1], rows * d * esz);
+  alloc(&m->x, rows * d * esz);
+  alloc(&m->qkv, rows * m->ld_qkv * esz);
+  alloc(&m->attn, rows * m->dq * esz);
+  alloc(&m->act, rows * F * esz);
+  alloc(reinterpret_cast<void**>(&m->lse), rows * cfg->n_heads * sizeof(float));
+  alloc(reinterpret_cast<void**>(&m->colmass), rows * cfg->n_kv_heads * sizeof(float));
+  alloc(reinterpret_cast<void**>(&m->scores), rows * sizeof(float));
+  alloc(reinterpret_cast<void**>(&m->idx), rows * sizeof(int32_t));
+  alloc(reinterpret_cast<void**>(&m->pos[0]), rows * sizeof(int32_t));
+  alloc(reinterpret_cast<void**>(&m->pos[1]), rows * sizeof(int32_t));
+  const int half = cfg->head_dim / 2;
+  alloc(reinterpret_cast<void**>(&m->rope_cos), static_cast<size_t>(max_L) * half * sizeof(float));
+  alloc(reinterpret_cast<void**>(&m->rope_sin), static_cast<size_t>(max_L) * half * sizeof(float));
+  alloc(reinterpret_cast<void**>(&m->status), sizeof(int));
+  if (!ok) {
+    cudaGetLastError();
+    free_model(m);
+    return fail(ZSAA_ERR_OOM, "workspace allocation failed for max_B=%d max_L=%d", max_B, max_L);
+  }
+  // RoPE table: angle(p, i) = p * theta^(-2i/hd), evaluated in double.
+  std::vector<float> cs(static_cast<size_t>(max_L) * half), sn(cs.size());
+  for (int p = 0; p < max_L; ++p)
+    for (int i = 0; i < half; ++i) {
+      const double inv = std::pow(static_cast<double>(cfg->rope_theta),
+                                  -2.0 * static_cast<double>(i) / static_cast<double>(cfg->head_dim));
+      const double a = static_cast<double>(p) * inv;
+      cs[static_cast<size_t>(p) * half + i] = static_cast<float>(std::cos(a));
+      sn[static_cast<size_t>(p) * half + i] = static_cast<float>(std::sin(a));
+    }
+  cudaError_t e = cudaMemcpy(m->rope_cos, cs.data(), cs.size() * sizeof(float), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemcpy(m->rope_sin, sn.data(), sn.size() * sizeof(float), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemset(m->status, 0, sizeof(int));
+  if (e != cudaSuccess) {
+    free_model(m);
+    return fail(ZSAA_ERR_CUDA, "workspace initialisation failed: %s", cudaGetErrorString(e));
+  }
+  if (cfg->dtype == ZSAA_BF16 && get_encode_tiled() == nullptr) {
+    free_model(m);
+    return fail(ZSAA_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+  }
+  *out = m;
+  return ZSAA_OK;
+}
+
+void zsaa_model_destroy(zsaa_model* m) {
+  if (m == nullptr) return;
+  cudaDeviceSynchronize();
+  free_model(m);
+}
+
+zsaa_status zsaa_plan(const zsaa_model* m, int L, double accel, int* n_sched, double* alpha_out) {
+  if (m == nullptr || n_sched == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null argument");
+  return plan_impl(m->cfg, L, accel, n_sched, alpha_out);
+}
+
+zsaa_status zsaa_forward(zsaa_model* m, const int32_t* token_ids, int B, int L, double accel,
+                         float* logits_out, int32_t* kept_pos_out, zsaa_stream stream) {
+  if (m == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null model");
+  return run_forward(m, token_ids, B, L, accel, logits_out, kept_pos_out, nullptr,
+                     reinterpret_cast<cudaStream_t>(stream));
+}
+
+zsaa_status zsaa_forward_ex(zsaa_model* m, const int32_t* token_ids, int B, int L, double accel,
+                            float* logits_out, int32_t* kept_pos_out, const zsaa_forward_opts* opts,
+                            zsaa_stream stream) {
+  if (m == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null model");
+  return run_forward(m, token_ids, B, L, accel, logits_out, kept_pos_out, opts,
+                     reinterpret_cast<cudaStream_t>(stream));
+}
+
+zsaa_status zsaa_forward_host(zsaa_model* m, const int32_t* token_ids, int B, int L, double accel,
+                              float* logits_out, int32_t* kept_pos_out, zsaa_stream stream) {
+  if (m == nullptr || token_ids == nullptr || logits_out == nullptr)
+    return fail(ZSAA_ERR_INVALID_ARG, "null argument");
+  if (B < 1 || B > m->max_B || L < 1 || L > m->max_L)
+    return fail(ZSAA_ERR_INVALID_ARG, "B=%d L=%d outside [1,%d] x [1,%d]", B, L, m->max_B, m->max_L);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  std::vector<int> sched(m->cfg.n_layers + 1);
+  zsaa_status st = plan_impl(m->cfg, L, accel, sched.data(), nullptr);
+  if (st != ZSAA_OK) return st;
+  const int n_final = sched[m->cfg.n_layers];
+  const size_t n_logits = m->cfg.n_classes > 0 ? static_cast<size_t>(B) * m->cfg.n_classes
+                                               : static_cast<size_t>(B) * n_final * m->cfg.vocab;
+  const size_t rows = static_cast<size_t>(m->max_B) * m->max_L;
+  if (m->stage_tok == nullptr) {
+    ZCK(cudaMalloc(&m->stage_tok, rows * sizeof(int32_t)));
+    ZCK(cudaMalloc(&m->stage_pos, rows * sizeof(int32_t)));
+  }
+  if (m->stage_logits_cap < n_logits) {
+    if (m->stage_logits) ZCK(cudaFree(m->stage_logits));
+    m->stage_logits = nullptr;
+    m->stage_logits_cap = 0;
+    ZCK(cudaMalloc(&m->stage_logits, n_logits * sizeof(float)));
+    m->stage_logits_cap = n_logits;
+  }
+  ZCK(cudaMemcpyAsync(m->stage_tok, token_ids, sizeof(int32_t) * B * L, cudaMemcpyHostToDevice, s));
+  st = run_forward(m, m->stage_tok, B, L, accel, m->stage_logits, m->stage_pos, nullptr, s);
+  if (st != ZSAA_OK) return st;
+  ZCK(cudaMemcpyAsync(logits_out, m->stage_logits, n_logits * sizeof(float), cudaMemcpyDeviceToHost, s));
+  if (kept_pos_out)
+    ZCK(cudaMemcpyAsync(kept_pos_out, m->stage_pos, sizeof(int32_t) * B * n_final,
+                        cudaMemcpyDeviceToHost, s));
+  ZCK(cudaStreamSynchronize(s));
+  return ZSAA_OK;
+}
+
+zsaa_status zsaa_score_select(const void* hidden, int B, int L, int d, int k, int32_t* idx_out,
+                              void* gathered_out, zsaa_stream stream) {
+  return score_select_impl(hidden, B, L, d, ZSAA_BF16, k, 0, nullptr, nullptr, idx_out,
+                           gathered_out, reinterpret_cast<cudaStream_t>(stream));
+}
+
+zsaa_status zsaa_score_select_ex(const void* hidden, int B, int L, int d, int dtype, int k,
+                                 int flags, const float* scores_in, float* scores_out,
+                                 int32_t* idx_out, void* gathered_out, zsaa_stream stream) {
+  return score_select_impl(hidden, B, L, d, dtype, k, flags, scores_in, scores_out, idx_out,
+                           gathered_out, reinterpret_cast<cudaStream_t>(stream));
+}
+
+zsaa_status zsaa_op_linear(const void* A, const void* W, const void* W2, const void* resid,
+                           void* out, int M, int N, int K, int dtype, int epilogue,
+                           const int32_t* pos, int rope_cols, int rope_hd, float rope_theta,
+                           zsaa_stream stream) {
+  if (A == nullptr || W == nullptr || out == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null argument");
+  if (M < 1 || N < 1 || K < 1) return fail(ZSAA_ERR_INVALID_ARG, "M, N, K must be >= 1");
+  if (epilogue < 0 || epilogue > 4) return fail(ZSAA_ERR_INVALID_ARG, "bad epilogue");
+  if (epilogue == kEpiSwiGLU && W2 == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "SwiGLU needs W2");
+  if (epilogue == kEpiResid && resid == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "residual needs resid");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  GemmParams p{};
+  p.M = M;
+  p.N = N;
+  p.K = K;
+  p.out = out;
+  p.ldo = N;
+  p.resid = resid;
+  p.status = shared_status();
+  if (p.status == nullptr) return fail(ZSAA_ERR_CUDA, "status word allocation failed");
+  if (dtype == ZSAA_BF16) {
+    if (K % 64 || N % 16) return fail(ZSAA_ERR_UNSUPPORTED, "bf16 GEMM needs K %% 64 == 0 and N %% 16 == 0");
+    if (epilogue == kEpiRope) {
+      if (pos == nullptr || rope_hd < 32 || rope_hd % 32 || rope_cols % rope_hd || rope_cols > N)
+        return fail(ZSAA_ERR_INVALID_ARG, "bad RoPE arguments");
+      RopeTable t;
+      if (!op_rope_table(rope_theta, rope_hd, &t)) return fail(ZSAA_ERR_CUDA, "RoPE table setup failed");
+      p.pos = pos;
+      p.cos_t = t.cos_t;
+      p.sin_t = t.sin_t;
+      p.rope_cols = rope_cols;
+      p.hd = rope_hd;
+    }
+    TcWeights Wt{W, W2, nullptr, N, N};
+    ZCK(launch_gemm_tc(A, K, Wt, epilogue, p, s));
+  } else if (dtype == ZSAA_F32) {
+    if (epilogue == kEpiRope) return fail(ZSAA_ERR_UNSUPPORTED, "f32 GEMM has no RoPE epilogue");
+    ZCK(launch_gemm_f32(static_cast<const float*>(A), K, static_cast<const float*>(W),
+                        static_cast<const float*>(W2), epilogue, p, s));
+  } else {
+    return fail(ZSAA_ERR_INVALID_ARG, "bad dtype");
+  }
+  return ZSAA_OK;
+}
+
+zsaa_status zsaa_op_attention(const void* qkv, int B, int N, int Hq, int Hkv, int hd, int dtype,
+                              void* out, float* lse, zsaa_stream stream) {
+  if (qkv == nullptr || out == nullptr || lse == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null argument");
+  if (B < 1 || N < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv) return fail(ZSAA_ERR_INVALID_ARG, "bad shape");
+  if (dtype == ZSAA_BF16 && hd != 64 && hd != 128) return fail(ZSAA_ERR_UNSUPPORTED, "bf16 attention needs hd 64 or 128");
+  if (dtype == ZSAA_F32 && (hd < 1 || hd > 128)) return fail(ZSAA_ERR_UNSUPPORTED, "f32 attention needs hd <= 128");
+  ZCK(launch_attention(dtype, qkv, B, N, Hq, Hkv, hd, out, lse, reinterpret_cast<cudaStream_t>(stream)));
+  return ZSAA_OK;
+}
+
+zsaa_status zsaa_op_colmass(const void* qkv, const float* lse, int B, int N, int Hq, int Hkv,
+                            int hd, int dtype, float* colmass, zsaa_stream stream) {
+  if (qkv == nullptr || lse == nullptr || colmass == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null argument");
+  if (B < 1 || N < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv) return fail(ZSAA_ERR_INVALID_ARG, "bad shape");
+  if (dtype == ZSAA_BF16 && hd != 64 && hd != 128) return fail(ZSAA_ERR_UNSUPPORTED, "bf16 column mass needs hd 64 or 128");
+  ZCK(launch_colmass(dtype, qkv, lse, B, N, Hq, Hkv, hd, colmass, reinterpret_cast<cudaStream_t>(stream)));
+  return ZSAA_OK;
+}
+
+zsaa_status zsaa_trace_begin(zsaa_model* m) {
+  if (m == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null model");
+  m->trace.clear();
+  m->ev_used = 0;
+  m->trace_names.clear();
+  m->tracing = true;
+  return ZSAA_OK;
+}
+
+zsaa_status zsaa_trace_end(zsaa_model* m, zsaa_trace_row* rows, int max_rows, int* n_rows) {
+  if (m == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null model");
+  m->tracing = false;
+  ZCK(cudaDeviceSynchronize());
+  std::vector<zsaa_trace_row> agg(m->trace_names.size());
+  for (size_t i = 0; i < agg.size(); ++i) {
+    memset(&agg[i], 0, sizeof(zsaa_trace_row));
+    snprintf(agg[i].name, sizeof(agg[i].name), "%s", m->trace_names[i].c_str());
+  }
+  for (const auto& r : m->trace) {
+    float ms = 0.f;
+    ZCK(cudaEventElapsedTime(&ms, r.a, r.b));
+    zsaa_trace_row& a = agg[r.cls];
+    a.launches += 1;
+    a.ms += ms;
+    a.flops += r.flops;
+    a.bytes += r.bytes;
+  }
+  const int n = static_cast<int>(agg.size());
+  if (n_rows) *n_rows = n;
+  for (int i = 0; i < n && i < max_rows && rows != nullptr; ++i) rows[i] = agg[i];
+  m->trace.clear();
+  m->ev_used = 0;
+  return ZSAA_OK;
+}
+
+zsaa_status zsaa_sync(zsaa_model* m, zsaa_stream stream) {
+  if (m == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null model");
+  return read_status(m->status, reinterpret_cast<cudaStream_t>(stream), false);
+}
+
+zsaa_status zsaa_device_status(void) {
+  int* w = shared_status();
+  if (w == nullptr) return fail(ZSAA_ERR_CUDA, "status word allocation failed");
+  return read_status(w, nullptr, true);
+}
+
+}  // extern "C"

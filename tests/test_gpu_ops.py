@@ -1,0 +1,203 @@
+"""Per-kernel parity on the GPU, through the C ABI: GEMM epilogues (tensor-core
+bf16 and CUDA-core fp32), causal attention (Eq. 1) and the soft-score column
+mass, each against the oracle's step (or a float64 matmul for a bare GEMM) on
+seeded inputs spanning several tiles and a ragged tail."""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import zsaa_oracle as O
+from tests.helpers import accum_bound, bf16_ulp_close, need_gpu
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def z(zlib):
+    need_gpu()
+    return zlib
+
+
+def _rand(shape, seed, scale=1.0, dtype=torch.bfloat16):
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+    return (torch.randn(*shape, generator=g, device="cuda") * scale).to(dtype)
+
+
+def _np(t):
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 64, 64), (300, 384, 256), (128, 256, 128), (517, 1024, 512),
+                                   (40, 2048, 2048)])
+def test_linear_bf16_store_and_f32(z, M, N, K):
+    A = _rand((M, K), 1)
+    W = _rand((N, K), 2)
+    ref = _np(A) @ _np(W).T
+    out = torch.empty(M, N, device="cuda", dtype=torch.bfloat16)
+    z.zsaa_op_linear(A, W, None, None, out, M, N, K, z.ZSAA_BF16, z.EPI_STORE)
+    out32 = torch.empty(M, N, device="cuda", dtype=torch.float32)
+    z.zsaa_op_linear(A, W, None, None, out32, M, N, K, z.ZSAA_BF16, z.EPI_STORE_F32)
+    torch.cuda.synchronize()
+    z.zsaa_device_status()
+    tol = accum_bound(_np(A), _np(W))
+    assert np.all(bf16_ulp_close(_np(out), O.bf16_round(ref), 1, tol))
+    # the worst-case bound is loose; nearly every element must also be within 1 ulp
+    assert np.mean(bf16_ulp_close(_np(out), O.bf16_round(ref), 1)) > 0.995
+    assert np.all(np.abs(_np(out32) - ref) <= tol + 1e-6 * np.abs(ref))
+
+
+def test_linear_bf16_large_n_lm_head(z):
+    M, N, K = 37, 128256, 256
+    A = _rand((M, K), 3)
+    W = _rand((N, K), 4, 0.02)
+    out = torch.empty(M, N, device="cuda", dtype=torch.float32)
+    z.zsaa_op_linear(A, W, None, None, out, M, N, K, z.ZSAA_BF16, z.EPI_STORE_F32)
+    torch.cuda.synchronize()
+    ref = _np(A) @ _np(W).T
+    assert np.all(np.abs(_np(out) - ref) <= accum_bound(_np(A), _np(W)) + 1e-6 * np.abs(ref))
+
+
+@pytest.mark.parametrize("M,N,K", [(200, 256, 128), (5, 512, 1024), (1000, 2048, 256)])
+def test_linear_bf16_residual_in_place(z, M, N, K):
+    A = _rand((M, K), 5, 0.1)
+    W = _rand((N, K), 6, 0.1)
+    H = _rand((M, N), 7)
+    h0 = _np(H)
+    z.zsaa_op_linear(A, W, None, H, H, M, N, K, z.ZSAA_BF16, z.EPI_RESID)
+    torch.cuda.synchronize()
+    ref = O.bf16_round(h0 + _np(A) @ _np(W).T)
+    assert np.all(bf16_ulp_close(_np(H), ref, 1, accum_bound(_np(A), _np(W))))
+
+
+@pytest.mark.parametrize("M,F,K", [(130, 384, 256), (7, 1024, 512), (600, 2048, 128)])
+def test_linear_bf16_swiglu(z, M, F, K):
+    A = _rand((M, K), 8)
+    Wg = _rand((F, K), 9, 0.1)
+    Wu = _rand((F, K), 10, 0.1)
+    out = torch.empty(M, F, device="cuda", dtype=torch.bfloat16)
+    z.zsaa_op_linear(A, Wg, Wu, None, out, M, F, K, z.ZSAA_BF16, z.EPI_SWIGLU)
+    torch.cuda.synchronize()
+    g = _np(A) @ _np(Wg).T
+    u = _np(A) @ _np(Wu).T
+    ref = O.bf16_round(O.silu(g) * u)
+    # d(silu(g) u) = silu'(g) u dg + silu(g) du, |silu'| <= 1.1
+    tol = 1.1 * np.abs(u) * accum_bound(_np(A), _np(Wg)) + np.abs(O.silu(g)) * accum_bound(_np(A), _np(Wu))
+    assert np.all(bf16_ulp_close(_np(out), ref, 2, tol))
+
+
+@pytest.mark.parametrize("hd,Hq,Hkv", [(64, 4, 2), (128, 2, 1)])
+def test_linear_bf16_rope(z, hd, Hq, Hkv):
+    M, K = 333, 256
+    N = (Hq + 2 * Hkv) * hd
+    rope_cols = (Hq + Hkv) * hd
+    A = _rand((M, K), 11)
+    W = _rand((N, K), 12, 0.1)
+    pos = torch.randint(0, 4096, (M,), generator=torch.Generator().manual_seed(3)).to(torch.int32).cuda()
+    out = torch.empty(M, N, device="cuda", dtype=torch.bfloat16)
+    z.zsaa_op_linear(A, W, None, None, out, M, N, K, z.ZSAA_BF16, z.EPI_ROPE, pos=pos,
+                     rope_cols=rope_cols, rope_hd=hd, rope_theta=500000.0)
+    torch.cuda.synchronize()
+    acc = _np(A) @ _np(W).T
+    cos, sin = O.rope_angles(pos.cpu().numpy(), hd, 500000.0)
+    qk = O.apply_rope(acc[:, :rope_cols].reshape(M, Hq + Hkv, hd), cos, sin).reshape(M, rope_cols)
+    ref = O.bf16_round(np.concatenate([qk, acc[:, rope_cols:]], axis=1))
+    # each rotated value mixes two accumulators; the float32 table adds ~1e-7 relative
+    b = accum_bound(_np(A), _np(W))
+    bq = b[:, :rope_cols].reshape(M, Hq + Hkv, hd)
+    half = hd // 2
+    pair = np.concatenate([bq[..., :half] + bq[..., half:], bq[..., :half] + bq[..., half:]], axis=-1)
+    tol = np.concatenate([pair.reshape(M, rope_cols), b[:, rope_cols:]], axis=1) + 1e-6 * np.abs(acc)
+    assert np.all(bf16_ulp_close(_np(out), ref, 2, tol))
+
+
+@pytest.mark.parametrize("epi", ["store", "resid", "swiglu"])
+def test_linear_f32(z, epi):
+    M, N, K = 77, 130, 96
+    A = _rand((M, K), 13, dtype=torch.float32)
+    W = _rand((N, K), 14, dtype=torch.float32)
+    W2 = _rand((N, K), 15, dtype=torch.float32)
+    H = _rand((M, N), 16, dtype=torch.float32)
+    h0 = _np(H)
+    e = {"store": z.EPI_STORE, "resid": z.EPI_RESID, "swiglu": z.EPI_SWIGLU}[epi]
+    out = H if epi == "resid" else torch.empty(M, N, device="cuda", dtype=torch.float32)
+    z.zsaa_op_linear(A, W, W2 if epi == "swiglu" else None, H if epi == "resid" else None, out,
+                     M, N, K, z.ZSAA_F32, e)
+    torch.cuda.synchronize()
+    acc = _np(A) @ _np(W).T
+    u = _np(A) @ _np(W2).T
+    ref = {"store": acc, "resid": h0 + acc, "swiglu": O.silu(acc) * u}[epi]
+    b = accum_bound(_np(A), _np(W))
+    tol = {"store": b, "resid": b, "swiglu": 1.1 * np.abs(u) * b
+           + np.abs(O.silu(acc)) * accum_bound(_np(A), _np(W2))}[epi]
+    assert np.all(np.abs(_np(out) - ref) <= tol + 2e-7 * np.abs(ref))
+
+
+def _qkv(B, N, Hq, Hkv, hd, seed, dtype):
+    return _rand((B * N, (Hq + 2 * Hkv) * hd), seed, 1.0, dtype)
+
+
+def _oracle_attention(qkv, B, N, Hq, Hkv, hd):
+    x = _np(qkv).reshape(B, N, Hq + 2 * Hkv, hd)
+    per = Hq // Hkv
+    outs, lses, Ps = [], [], []
+    for b in range(B):
+        q, k, v = x[b, :, :Hq], x[b, :, Hq:Hq + Hkv], x[b, :, Hq + Hkv:]
+        o = np.empty((N, Hq, hd))
+        P = np.empty((Hq, N, N))
+        lse = np.empty((Hq, N))
+        for h in range(Hq):
+            g = h // per
+            P[h] = O.attention_probs(q[:, h], k[:, g])
+            o[:, h] = P[h] @ v[:, g]
+            s = (q[:, h] @ k[:, g].T) / math.sqrt(hd)
+            s = np.where(np.tril(np.ones((N, N), bool)), s, -np.inf)
+            mx = s.max(axis=1)
+            lse[h] = (mx + np.log(np.exp(s - mx[:, None]).sum(axis=1))) / math.log(2.0)
+        outs.append(o.reshape(N, Hq * hd))
+        lses.append(lse)
+        Ps.append(P)
+    return np.stack(outs), np.stack(lses), Ps, x
+
+
+@pytest.mark.parametrize("B,N,Hq,Hkv,hd", [(2, 1, 4, 2, 64), (2, 65, 4, 2, 64), (1, 200, 4, 1, 128),
+                                           (2, 130, 8, 2, 128), (1, 64, 2, 2, 64)])
+def test_attention_and_colmass_bf16(z, B, N, Hq, Hkv, hd):
+    qkv = _qkv(B, N, Hq, Hkv, hd, 20 + N, torch.bfloat16)
+    out = torch.empty(B * N, Hq * hd, device="cuda", dtype=torch.bfloat16)
+    lse = torch.empty(B, Hq, N, device="cuda", dtype=torch.float32)
+    z.zsaa_op_attention(qkv, B, N, Hq, Hkv, hd, z.ZSAA_BF16, out, lse)
+    torch.cuda.synchronize()
+    ref_o, ref_lse, Ps, _ = _oracle_attention(qkv, B, N, Hq, Hkv, hd)
+    got = _np(out).reshape(B, N, Hq * hd)
+    err = np.abs(got - ref_o)
+    assert err.max() < 2e-2 and err.mean() < 2e-3, (err.max(), err.mean())
+    np.testing.assert_allclose(_np(lse), ref_lse, rtol=1e-5, atol=1e-4)
+    # column mass from the oracle's lse, so it is checked on its own
+    C = torch.empty(B, Hkv, N, device="cuda", dtype=torch.float32)
+    lse_in = torch.from_numpy(ref_lse.astype(np.float32)).cuda()
+    z.zsaa_op_colmass(qkv, lse_in, B, N, Hq, Hkv, hd, z.ZSAA_BF16, C)
+    torch.cuda.synchronize()
+    refC = np.stack([O.column_mass(Ps[b], Hkv) for b in range(B)])
+    np.testing.assert_allclose(_np(C), refC, rtol=2e-4, atol=1e-5)
+    # every query row sums to one: each group's columns total (Hq/Hkv) * N
+    np.testing.assert_allclose(_np(C).sum(axis=2), (Hq // Hkv) * N, rtol=1e-4)
+
+
+@pytest.mark.parametrize("B,N,Hq,Hkv,hd", [(2, 64, 4, 4, 32), (1, 37, 4, 2, 32)])
+def test_attention_and_colmass_f32(z, B, N, Hq, Hkv, hd):
+    qkv = _qkv(B, N, Hq, Hkv, hd, 40 + N, torch.float32)
+    out = torch.empty(B * N, Hq * hd, device="cuda", dtype=torch.float32)
+    lse = torch.empty(B, Hq, N, device="cuda", dtype=torch.float32)
+    z.zsaa_op_attention(qkv, B, N, Hq, Hkv, hd, z.ZSAA_F32, out, lse)
+    torch.cuda.synchronize()
+    ref_o, ref_lse, Ps, _ = _oracle_attention(qkv, B, N, Hq, Hkv, hd)
+    np.testing.assert_allclose(_np(out).reshape(B, N, Hq * hd), ref_o, rtol=1e-5, atol=1e-5)
+    C = torch.empty(B, Hkv, N, device="cuda", dtype=torch.float32)
+    z.zsaa_op_colmass(qkv, lse, B, N, Hq, Hkv, hd, z.ZSAA_F32, C)
+    torch.cuda.synchronize()
+    refC = np.stack([O.column_mass(Ps[b], Hkv) for b in range(B)])
+    np.testing.assert_allclose(_np(C), refC, rtol=1e-5, atol=1e-6)
