@@ -110,13 +110,25 @@ typedef struct zsaa_model zsaa_model;
  *   scores_out : [B, N_{l-1}] float32 position scores of that layer;
  *   idx_out    : [B, N_l] int32 kept indices of that layer.
  * hidden_out : [B, N_last, d] residual rows leaving the last layer run.
- * n_layers_run: 0 runs all layers; m > 0 runs layers 1..m, then the head. */
+ * n_layers_run: 0 runs through the last layer; m > 0 stops after layer m,
+ *               then the head runs on the rows leaving layer m.
+ * hidden_in  : [B, L, d] residual rows to start from instead of embedding
+ *              token_ids (token_ids is then ignored and may be NULL); the
+ *              pass starts at layer first_layer (1 .. n_layers + 1; n_layers
+ *              + 1 runs only the head).  pos_in [B, L] gives the rows'
+ *              original positions (NULL: 0..L-1).  The preservation rate is
+ *              planned for sequences of plan_L tokens (0: L) and Eq. 2 is
+ *              applied from N_{first_layer-1} = L. */
 typedef struct {
   const int32_t* forced_idx;
   float* scores_out;
   int32_t* idx_out;
   void* hidden_out;
   int n_layers_run;
+  const void* hidden_in;
+  const int32_t* pos_in;
+  int first_layer;
+  int plan_L;
 } zsaa_forward_opts;
 
 /* Eq. 2 schedule for a config without a model (host only, no GPU needed).

@@ -338,7 +338,8 @@ def head(cfg: OracleConfig, weights, h: np.ndarray, store: _Store) -> np.ndarray
 
 
 def forward(cfg: OracleConfig, weights, tokens: np.ndarray, accel: Optional[float] = None,
-            alpha: Optional[float] = None, forced_idx: Optional[Dict[int, np.ndarray]] = None):
+            alpha: Optional[float] = None, forced_idx: Optional[Dict[int, np.ndarray]] = None,
+            collect: bool = False):
     """Pruned prefill of a batch of token sequences [B, L].
 
     The preservation schedule comes from ``accel`` (via ``plan``) or from
@@ -348,7 +349,9 @@ def forward(cfg: OracleConfig, weights, tokens: np.ndarray, accel: Optional[floa
 
     Returns a dict with ``logits`` ([B, N_n, V] or [B, n_classes]),
     ``kept_pos`` [B, N_n], ``schedule``, ``alpha`` and per pruning layer
-    ``idx`` [B, k] and ``scores`` [B, N_{l-1}].
+    ``idx`` [B, k] and ``scores`` [B, N_{l-1}].  With ``collect`` it also has
+    ``layer_inputs`` {l: (h [B, N_{l-1}, d], pos [B, N_{l-1}])} and
+    ``final_hidden`` [B, N_n, d] (the residual rows entering the head).
     """
     tokens = np.asarray(tokens)
     B, L = tokens.shape
@@ -363,11 +366,15 @@ def forward(cfg: OracleConfig, weights, tokens: np.ndarray, accel: Optional[floa
     logits, kept_pos = [], []
     idx_all: Dict[int, list] = {}
     scores_all: Dict[int, list] = {}
+    inputs_all: Dict[int, list] = {}
+    finals = []
     for b in range(B):
         h = store(emb[tokens[b]])
         pos = np.arange(L)
         for layer in range(1, cfg.n_layers + 1):
             lw = weights["layers"][layer - 1]
+            if collect:
+                inputs_all.setdefault(layer, []).append((h, pos))
             h, P, v = attention_block(cfg, lw, h, pos, store)
             h = mlp_block(cfg, lw, h, store)
             k_keep = sched[layer]
@@ -386,7 +393,8 @@ def forward(cfg: OracleConfig, weights, tokens: np.ndarray, accel: Optional[floa
                 pos = pos[idx]
         logits.append(head(cfg, weights, h, store))
         kept_pos.append(pos)
-    return {
+        finals.append(h)
+    out = {
         "logits": np.stack(logits),
         "kept_pos": np.stack(kept_pos),
         "schedule": sched,
@@ -394,6 +402,11 @@ def forward(cfg: OracleConfig, weights, tokens: np.ndarray, accel: Optional[floa
         "idx": {k: np.stack(v) for k, v in idx_all.items()},
         "scores": {k: np.stack(v) for k, v in scores_all.items()},
     }
+    if collect:
+        out["layer_inputs"] = {k: (np.stack([a for a, _ in v]), np.stack([p for _, p in v]))
+                               for k, v in inputs_all.items()}
+        out["final_hidden"] = np.stack(finals)
+    return out
 
 
 def forward_masked(cfg: OracleConfig, weights, tokens: np.ndarray, sched: Sequence[int]):

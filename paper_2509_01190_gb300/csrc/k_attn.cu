@@ -12,7 +12,8 @@
 //   P[i,j], recomputed from q, k and lse2 (no N x N matrix is stored).
 //
 // bf16 path: FlashAttention-style tiles on mma.sync m16n8k16 (64 queries x 64
-// keys per step, 4 warps x 16 rows), online softmax in fp32.  The column-mass
+// keys per step, 4 warps x 16 rows), online softmax in fp32; the probabilities
+// enter P V as a hi/lo pair of bf16 matrices.  The column-mass
 // pass sweeps key blocks outer / query blocks inner so each CTA owns its
 // columns and sums them in registers (deterministic, no atomics).
 // fp32 path: plain CUDA-core kernels (one warp per row / column).
@@ -150,17 +151,22 @@ __global__ void __launch_bounds__(128)
       o[i][2] *= al_hi;
       o[i][3] *= al_hi;
     }
-    uint32_t pf[4][4];
+    // P as a pair of bf16 matrices, P = P_hi + P_lo, so P V keeps ~16 bits of P
+    // (one bf16 P would cost ~0.1% relative error in every output).
+    uint32_t ph[4][4], pl[4][4];
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt) {
       const float p0 = exp2f(s[nt][0] - base_lo), p1 = exp2f(s[nt][1] - base_lo);
       const float p2 = exp2f(s[nt][2] - base_hi), p3 = exp2f(s[nt][3] - base_hi);
       l_lo += p0 + p1;
       l_hi += p2 + p3;
-      pf[nt >> 1][(nt & 1) * 2 + 0] = pack_bf16x2(p0, p1);
-      pf[nt >> 1][(nt & 1) * 2 + 1] = pack_bf16x2(p2, p3);
+      const uint32_t h01 = pack_bf16x2(p0, p1), h23 = pack_bf16x2(p2, p3);
+      ph[nt >> 1][(nt & 1) * 2 + 0] = h01;
+      ph[nt >> 1][(nt & 1) * 2 + 1] = h23;
+      pl[nt >> 1][(nt & 1) * 2 + 0] = pack_bf16x2(p0 - bf16lo(h01), p1 - bf16hi(h01));
+      pl[nt >> 1][(nt & 1) * 2 + 1] = pack_bf16x2(p2 - bf16lo(h23), p3 - bf16hi(h23));
     }
-    // O += P V
+    // O += P_hi V + P_lo V
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
 #pragma unroll
@@ -169,8 +175,10 @@ __global__ void __launch_bounds__(128)
         const int r = j * 16 + (mi & 1) * 8 + (lane & 7);
         uint32_t b0, b1, b2, b3;
         ldsm_x4_t(sV + swz<ROWB>(r, dp * 2 + (mi >> 1)), b0, b1, b2, b3);
-        mma_bf16_16816(o[2 * dp], pf[j], b0, b1);
-        mma_bf16_16816(o[2 * dp + 1], pf[j], b2, b3);
+        mma_bf16_16816(o[2 * dp], ph[j], b0, b1);
+        mma_bf16_16816(o[2 * dp + 1], ph[j], b2, b3);
+        mma_bf16_16816(o[2 * dp], pl[j], b0, b1);
+        mma_bf16_16816(o[2 * dp + 1], pl[j], b2, b3);
       }
     }
     __syncthreads();

@@ -335,28 +335,57 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
                         float* logits, int32_t* kept_pos, const zsaa_forward_opts* opts,
                         cudaStream_t s) {
   const zsaa_config& c = m->cfg;
-  if (tok == nullptr || logits == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null token or logits pointer");
+  const bool from_hidden = opts && opts->hidden_in;
+  if ((!from_hidden && tok == nullptr) || logits == nullptr)
+    return fail(ZSAA_ERR_INVALID_ARG, "null token or logits pointer");
   if (B < 1 || B > m->max_B || L < 1 || L > m->max_L)
     return fail(ZSAA_ERR_INVALID_ARG, "B=%d L=%d outside [1,%d] x [1,%d]", B, L, m->max_B, m->max_L);
+  const int first = from_hidden ? opts->first_layer : 1;
   const int n_run = (opts && opts->n_layers_run > 0) ? opts->n_layers_run : c.n_layers;
-  if (n_run > c.n_layers) return fail(ZSAA_ERR_INVALID_ARG, "n_layers_run > n_layers");
+  if (first < 1 || first > c.n_layers + 1) return fail(ZSAA_ERR_INVALID_ARG, "first_layer outside [1, n_layers+1]");
+  if (n_run > c.n_layers || n_run < first - 1) return fail(ZSAA_ERR_INVALID_ARG, "bad n_layers_run");
+  const int plan_L = (from_hidden && opts->plan_L > 0) ? opts->plan_L : L;
   std::vector<int> sched(c.n_layers + 1);
   double alpha = 1.0;
-  zsaa_status st = plan_impl(c, L, accel, sched.data(), &alpha);
+  zsaa_status st = plan_impl(c, plan_L, accel, sched.data(), &alpha);
   if (st != ZSAA_OK) return st;
+  if (from_hidden) {  // Eq. 2 continued from the rows given
+    sched[first - 1] = L;
+    for (int l = first; l <= c.n_layers; ++l) {
+      int tmp[2];
+      zsaa_config one = c;
+      one.n_layers = 1;
+      one.prune_mask = prunes(c, l) ? 1ull : 0ull;
+      eq2_schedule(one, sched[l - 1], alpha, tmp);
+      sched[l] = tmp[1];
+    }
+  }
 
   const int d = c.d_model, hd = c.head_dim, Hq = c.n_heads, Hkv = c.n_kv_heads;
   const int dt = c.dtype;
   int cur = 0;
   const double es = static_cast<double>(m->esz);
 #define TRACE(name, fl, by) TraceScope trace_scope_(m, name, fl, by, s)
-  {
+  if (from_hidden) {
+    ZCK(cudaMemcpyAsync(m->h[cur], opts->hidden_in, static_cast<size_t>(B) * L * d * m->esz,
+                        cudaMemcpyDeviceToDevice, s));
+    if (opts->pos_in) {
+      ZCK(cudaMemcpyAsync(m->pos[cur], opts->pos_in, sizeof(int32_t) * B * L,
+                          cudaMemcpyDeviceToDevice, s));
+    } else {
+      std::vector<int32_t> iota(static_cast<size_t>(B) * L);
+      for (size_t i = 0; i < iota.size(); ++i) iota[i] = static_cast<int32_t>(i % L);
+      ZCK(cudaMemcpyAsync(m->pos[cur], iota.data(), iota.size() * sizeof(int32_t),
+                          cudaMemcpyHostToDevice, s));
+      ZCK(cudaStreamSynchronize(s));
+    }
+  } else {
     TRACE("embed", 0.0, static_cast<double>(B) * L * (d * es + 8.0));
     ZCK(launch_embed(dt, m->embed, tok, B * L, L, c.vocab, d, m->h[cur], m->pos[cur], m->status, s));
   }
   size_t off_forced = 0, off_scores = 0, off_idx = 0;
   int N = L;
-  for (int l = 1; l <= n_run; ++l) {
+  for (int l = first; l <= n_run; ++l) {
     const int li = l - 1;
     const int M = B * N;
     void* h = m->h[cur];

@@ -53,7 +53,8 @@ class zsaa_weights(C.Structure):
 
 class zsaa_forward_opts(C.Structure):
     _fields_ = [("forced_idx", C.c_void_p), ("scores_out", C.c_void_p), ("idx_out", C.c_void_p),
-                ("hidden_out", C.c_void_p), ("n_layers_run", C.c_int)]
+                ("hidden_out", C.c_void_p), ("n_layers_run", C.c_int), ("hidden_in", C.c_void_p),
+                ("pos_in", C.c_void_p), ("first_layer", C.c_int), ("plan_L", C.c_int)]
 
 
 class zsaa_trace_row(C.Structure):
@@ -220,9 +221,10 @@ def zsaa_forward(model: Model, token_ids, B: int, L: int, accel: float, logits_o
 
 def zsaa_forward_ex(model: Model, token_ids, B: int, L: int, accel: float, logits_out,
                     kept_pos_out=None, forced_idx=None, scores_out=None, idx_out=None,
-                    hidden_out=None, n_layers_run: int = 0, stream=None):
+                    hidden_out=None, n_layers_run: int = 0, hidden_in=None, pos_in=None,
+                    first_layer: int = 1, plan_L: int = 0, stream=None):
     opts = zsaa_forward_opts(_ptr(forced_idx), _ptr(scores_out), _ptr(idx_out), _ptr(hidden_out),
-                             n_layers_run)
+                             n_layers_run, _ptr(hidden_in), _ptr(pos_in), first_layer, plan_L)
     _check(lib().zsaa_forward_ex(model.handle, _ptr(token_ids), B, L, float(accel),
                                  _ptr(logits_out), _ptr(kept_pos_out), C.byref(opts),
                                  _stream(stream)))
