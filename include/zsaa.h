@@ -190,6 +190,25 @@ zsaa_status zsaa_score_select_ex(const void* hidden, int B, int L, int d, int dt
                                  int flags, const float* scores_in, float* scores_out,
                                  int32_t* idx_out, void* gathered_out, zsaa_stream stream);
 
+/* zsaa_score_select for callers that cannot allocate device memory while they
+ * run (the paper has no counterpart; this is a property of the library).
+ * Serving loops that reserve their memory budget up front, latency-critical
+ * code that must avoid the allocator's locks and implicit synchronisation, and
+ * hosts whose framework owns every device allocation cannot let a call take
+ * scratch from the memory pool, as zsaa_score_select does for its B*L scores.
+ * This call allocates nothing: the scores live in a fixed array of 1,048,576
+ * floats (4 MiB) that the library holds on every GPU where its device code is
+ * loaded, until the process exits.
+ *   Arguments, layouts and results are those of zsaa_score_select.
+ *   B*L above 1,048,576 is rejected with ZSAA_ERR_INVALID_ARG before any work.
+ *   The first call on a device looks up the array's device address with that
+ *   device current; make that first call before any stream capture.
+ *   All calls share the one array: calls whose work can overlap on the GPU
+ *   (different streams, or different host threads) race on it and must be
+ *   ordered by the caller. */
+zsaa_status zsaa_score_select_noalloc(const void* hidden, int B, int L, int d, int k,
+                                      int32_t* idx_out, void* gathered_out, zsaa_stream stream);
+
 /* Single steps of the path, for per-kernel checks and timing.  All pointers
  * device; shapes as stated.
  * zsaa_op_linear: out[M,N] = epilogue(A[M,K] W[N,K]^T); dtype ZSAA_BF16 uses

@@ -67,6 +67,9 @@ cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, i
 cudaError_t launch_colmass(int dtype, const void* qkv, const float* lse, int B, int N, int Hq,
                            int Hkv, int hd, float* C, cudaStream_t s);
 
+// ---- thread-local message returned by zsaa_last_error (zsaa_api.cu)
+void set_last_error(const char* msg);
+
 // ---- driver entry point for tensor maps (zsaa_api.cu)
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,

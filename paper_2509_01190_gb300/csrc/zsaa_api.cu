@@ -203,6 +203,8 @@ bool op_rope_table(float theta, int hd, RopeTable* out) {
 }  // namespace
 
 namespace zsaa {
+void set_last_error(const char* msg) { g_last_error = msg; }
+
 EncodeTiledFn get_encode_tiled() {
   std::call_once(g_encode_once, [] {
     void* fn = nullptr;

@@ -27,6 +27,7 @@ EXPORTED = [
     "zsaa_forward_ex", "zsaa_forward_host", "zsaa_score_select", "zsaa_score_select_ex",
     "zsaa_op_linear", "zsaa_op_attention", "zsaa_op_colmass", "zsaa_sync", "zsaa_device_status",
     "zsaa_last_error", "zsaa_version", "zsaa_trace_begin", "zsaa_trace_end",
+    "zsaa_score_select_noalloc",
 ]
 
 
@@ -86,6 +87,7 @@ def lib():
             "zsaa_forward_host": ([_P, _P, _I, _I, _D, _P, _P, _P], _I),
             "zsaa_score_select": ([_P, _I, _I, _I, _I, _P, _P, _P], _I),
             "zsaa_score_select_ex": ([_P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _P, _P], _I),
+            "zsaa_score_select_noalloc": ([_P, _I, _I, _I, _I, _P, _P, _P], _I),
             "zsaa_op_linear": ([_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _I, _I, C.c_float, _P], _I),
             "zsaa_op_attention": ([_P, _I, _I, _I, _I, _I, _I, _P, _P, _P], _I),
             "zsaa_op_colmass": ([_P, _P, _I, _I, _I, _I, _I, _I, _P, _P], _I),
@@ -275,6 +277,13 @@ def zsaa_score_select_ex(hidden, B: int, L: int, d: int, dtype: int, k: int, fla
     _check(lib().zsaa_score_select_ex(_ptr(hidden), B, L, d, dtype, k, flags, _ptr(scores_in),
                                       _ptr(scores_out), _ptr(idx_out), _ptr(gathered_out),
                                       _stream(stream)))
+
+
+def zsaa_score_select_noalloc(hidden, B: int, L: int, d: int, k: int, idx_out, gathered_out=None,
+                              stream=None):
+    """zsaa_score_select without device allocation (fixed 4 MiB scratch, B*L <= 2**20)."""
+    _check(lib().zsaa_score_select_noalloc(_ptr(hidden), B, L, d, k, _ptr(idx_out),
+                                           _ptr(gathered_out), _stream(stream)))
 
 
 def zsaa_op_linear(A, W, W2, resid, out, M: int, N: int, K: int, dtype: int, epilogue: int,
