@@ -42,7 +42,12 @@ struct GemmParams {
   int rope_cols;        // kEpiRope: columns [0, rope_cols) are rotated
   int hd;               // kEpiRope: head size
   int* status;          // device status word
+  float* splitk_ws;     // optional fp32 workspace for split-K partial tiles (NULL: no split)
+  size_t splitk_ws_elems;
 };
+
+// Split-K workspace a caller should provide: two waves of 128 x 256 fp32 tiles.
+constexpr size_t kSplitKWorkspaceElems = static_cast<size_t>(2) * 160 * 128 * 256;
 
 // bf16 tensor-core GEMM: out = epi(A[M,K] * W^T).  W is given as up to three
 // row blocks (w0: rows [0, n1), w1: rows [n1, n2), w2: rows [n2, N)) so the

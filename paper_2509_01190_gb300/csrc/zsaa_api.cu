@@ -160,6 +160,22 @@ int* shared_status() {
   return p;
 }
 
+// Split-K workspace of zsaa_op_linear, one per device, allocated on first use.
+std::mutex g_ws_mu;
+std::unordered_map<int, float*> g_op_ws;
+
+float* op_splitk_ws() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
+  std::lock_guard<std::mutex> lk(g_ws_mu);
+  auto it = g_op_ws.find(dev);
+  if (it != g_op_ws.end()) return it->second;
+  float* p = nullptr;
+  if (cudaMalloc(&p, kSplitKWorkspaceElems * sizeof(float)) != cudaSuccess) return nullptr;
+  g_op_ws[dev] = p;
+  return p;
+}
+
 // RoPE tables of zsaa_op_linear, cached per (device, theta, head size):
 // positions 0 .. kOpRopePositions-1.
 constexpr int kOpRopePositions = 16384;
@@ -243,6 +259,7 @@ struct zsaa_model {
   int32_t* pos[2] = {nullptr, nullptr};
   float* rope_cos = nullptr;
   float* rope_sin = nullptr;
+  float* splitk_ws = nullptr;
   int* status = nullptr;
   // host-buffer staging (zsaa_forward_host)
   int32_t* stage_tok = nullptr;
@@ -313,7 +330,7 @@ void free_model(zsaa_model* m) {
   for (cudaEvent_t e : m->ev_pool) cudaEventDestroy(e);
   void* ptrs[] = {m->h[0], m->h[1], m->x, m->qkv, m->attn, m->act, m->lse, m->colmass,
                   m->scores, m->idx, m->pos[0], m->pos[1], m->rope_cos, m->rope_sin,
-                  m->status, m->stage_tok, m->stage_logits, m->stage_pos};
+                  m->splitk_ws, m->status, m->stage_tok, m->stage_logits, m->stage_pos};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   delete m;
@@ -323,6 +340,8 @@ void free_model(zsaa_model* m) {
 zsaa_status linear(zsaa_model* m, const void* A, int lda, const TcWeights& W, int epi,
                    GemmParams p, cudaStream_t s) {
   p.status = m->status;
+  p.splitk_ws = m->splitk_ws;
+  p.splitk_ws_elems = m->splitk_ws ? kSplitKWorkspaceElems : 0;
   if (m->cfg.dtype == ZSAA_BF16) {
     ZCK(launch_gemm_tc(A, lda, W, epi, p, s));
   } else {
@@ -680,6 +699,8 @@ zsaa_status zsaa_model_create(const zsaa_config* cfg, const zsaa_weights* w, int
   alloc(reinterpret_cast<void**>(&m->rope_cos), static_cast<size_t>(max_L) * half * sizeof(float));
   alloc(reinterpret_cast<void**>(&m->rope_sin), static_cast<size_t>(max_L) * half * sizeof(float));
   alloc(reinterpret_cast<void**>(&m->status), sizeof(int));
+  if (cfg->dtype == ZSAA_BF16)
+    alloc(reinterpret_cast<void**>(&m->splitk_ws), kSplitKWorkspaceElems * sizeof(float));
   if (!ok) {
     cudaGetLastError();
     free_model(m);
@@ -818,6 +839,8 @@ zsaa_status zsaa_op_linear(const void* A, const void* W, const void* W2, const v
       p.hd = rope_hd;
     }
     TcWeights Wt{W, W2, nullptr, N, N};
+    p.splitk_ws = op_splitk_ws();
+    p.splitk_ws_elems = p.splitk_ws ? kSplitKWorkspaceElems : 0;
     ZCK(launch_gemm_tc(A, K, Wt, epilogue, p, s));
   } else if (dtype == ZSAA_F32) {
     if (epilogue == kEpiRope) return fail(ZSAA_ERR_UNSUPPORTED, "f32 GEMM has no RoPE epilogue");

@@ -159,6 +159,62 @@ def test_linear_bf16_full_1b_shapes(z, name, M, N, K):
     assert np.mean(bf16_ulp_close(got, ref, 1)) > 0.995, name
 
 
+# Small M with deep K: fewer tiles than SMs, so the GEMM splits K and a
+# finishing kernel sums the fp32 partials in a fixed order (every epilogue).
+@pytest.mark.parametrize("epi", ["store", "store_f32", "resid", "swiglu", "rope"])
+def test_linear_bf16_split_k(z, epi):
+    M, K = 40, 4096
+    A = _rand((M, K), 51)
+    An = _np(A)
+    if epi == "rope":
+        hd, Hq, Hkv = 64, 4, 2
+        N, rope_cols = (Hq + 2 * Hkv) * hd, (Hq + Hkv) * hd
+        W = _rand((N, K), 52, 0.02)
+        pos = torch.arange(100, 100 + M, dtype=torch.int32, device="cuda")
+        out = torch.empty(M, N, device="cuda", dtype=torch.bfloat16)
+        z.zsaa_op_linear(A, W, None, None, out, M, N, K, z.ZSAA_BF16, z.EPI_ROPE, pos=pos,
+                         rope_cols=rope_cols, rope_hd=hd, rope_theta=10000.0)
+        acc = An @ _np(W).T
+        cos, sin = O.rope_angles(pos.cpu().numpy(), hd, 10000.0)
+        qk = O.apply_rope(acc[:, :rope_cols].reshape(M, -1, hd), cos, sin).reshape(M, rope_cols)
+        ref = O.bf16_round(np.concatenate([qk, acc[:, rope_cols:]], axis=1))
+        tol = 2 * accum_bound(An, _np(W)).max(axis=1, keepdims=True)
+    elif epi == "swiglu":
+        F = 1024
+        Wg, Wu = _rand((F, K), 53, 0.02), _rand((F, K), 54, 0.02)
+        out = torch.empty(M, F, device="cuda", dtype=torch.bfloat16)
+        z.zsaa_op_linear(A, Wg, Wu, None, out, M, F, K, z.ZSAA_BF16, z.EPI_SWIGLU)
+        g, u = An @ _np(Wg).T, An @ _np(Wu).T
+        ref = O.bf16_round(O.silu(g) * u)
+        tol = 1.1 * np.abs(u) * accum_bound(An, _np(Wg)) + np.abs(O.silu(g)) * accum_bound(An, _np(Wu))
+    else:
+        N = 2048
+        W = _rand((N, K), 55, 0.02)
+        acc = An @ _np(W).T
+        tol = accum_bound(An, _np(W))
+        if epi == "resid":
+            H = _rand((M, N), 56)
+            h0 = _np(H)
+            z.zsaa_op_linear(A, W, None, H, H, M, N, K, z.ZSAA_BF16, z.EPI_RESID)
+            out, ref = H, O.bf16_round(h0 + acc)
+        elif epi == "store":
+            out = torch.empty(M, N, device="cuda", dtype=torch.bfloat16)
+            z.zsaa_op_linear(A, W, None, None, out, M, N, K, z.ZSAA_BF16, z.EPI_STORE)
+            ref = O.bf16_round(acc)
+        else:
+            out = torch.empty(M, N, device="cuda", dtype=torch.float32)
+            z.zsaa_op_linear(A, W, None, None, out, M, N, K, z.ZSAA_BF16, z.EPI_STORE_F32)
+            ref = acc
+    torch.cuda.synchronize()
+    z.zsaa_device_status()
+    got = _np(out)
+    if epi == "store_f32":
+        assert np.all(np.abs(got - ref) <= tol + 1e-6 * np.abs(ref))
+    else:
+        assert np.all(bf16_ulp_close(got, ref, 2, tol)), epi
+        assert np.mean(bf16_ulp_close(got, ref, 1)) > 0.995, epi
+
+
 @pytest.mark.parametrize("epi", ["store", "resid", "swiglu"])
 def test_linear_f32(z, epi):
     M, N, K = 77, 130, 96
