@@ -270,7 +270,7 @@ def main():
         barrier()
         return max_over_ranks(ms) / steps
 
-    # ---- headline
+    # ---- headline (plain forwards replay from the library's CUDA graphs)
     sampler = ClockSampler(local) if rank == 0 else None
     ms_head = timed(args.accel, args.steps, args.warmup, sampler)
     sched, alpha = zsaa.zsaa_plan(model, L, args.accel)
@@ -305,6 +305,10 @@ def main():
         for k, v in sweep.items():
             v["speedup_vs_unpruned"] = (base_ms / v["ms"]) if base_ms else None
         line["sweep"] = sweep
+        # the same headline forward without graph replay (every launch from the host)
+        zsaa.zsaa_model_set_graphs(model, False)
+        line["ms_per_step_eager"] = timed(args.accel, args.steps, 3)
+        zsaa.zsaa_model_set_graphs(model, True)
 
         # ---- per-kernel trace of the headline forward (separate traced steps)
         zsaa.zsaa_trace_begin(model)

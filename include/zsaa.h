@@ -159,6 +159,15 @@ zsaa_status zsaa_plan(const zsaa_model* m, int L, double accel, int* n_sched, do
 zsaa_status zsaa_forward(zsaa_model* m, const int32_t* token_ids, int B, int L, double accel,
                          float* logits_out, int32_t* kept_pos_out, zsaa_stream stream);
 
+/* zsaa_forward and zsaa_forward_host replay repeated calls from CUDA graphs:
+ * the first call with a given (token_ids, B, L, accel, logits_out,
+ * kept_pos_out) runs eagerly, the second is captured on the given stream and
+ * instantiated, and later ones launch the graph.  The 16 most recent argument
+ * sets are kept per model.  A model is used by one host thread at a time.
+ * zsaa_model_set_graphs(m, 0) turns this off (every call eager); 1 turns it
+ * back on.  zsaa_forward_ex always runs eagerly. */
+zsaa_status zsaa_model_set_graphs(zsaa_model* m, int enable);
+
 /* zsaa_forward with the hooks of zsaa_forward_opts (opts may be NULL). */
 zsaa_status zsaa_forward_ex(zsaa_model* m, const int32_t* token_ids, int B, int L, double accel,
                             float* logits_out, int32_t* kept_pos_out,

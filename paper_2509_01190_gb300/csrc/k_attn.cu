@@ -208,19 +208,26 @@ __global__ void __launch_bounds__(128)
   }
 }
 
-// Column mass: CTA (key block kb, KV head g, batch b).  Warp w owns keys
-// kb*64 + w*16 .. +16 as the A operand; query tiles are the B operand.
+// Column mass: CTA (key block kb, query chunk qc, KV head g * B + b).  Warp w
+// owns keys kb*64 + w*16 .. +16 as the A operand; the query tiles of chunk qc
+// (q_per blocks of 64, only those at or after the key block) are the B
+// operand, for every query head of group g.  The CTA writes its partial column
+// sums, times ||v_j|| of group g when weight_vnorm is set (the score of R1 is
+// linear in the column mass), to parts[qc][b][g][j]; a reduce kernel sums
+// the chunks in a fixed order.
 template <int HD>
 __global__ void __launch_bounds__(128)
     colmass_bf16_kernel(const bf16* __restrict__ qkv, const float* __restrict__ lse2, int N,
-                        int Hq, int Hkv, float* __restrict__ C, float scale_log2) {
+                        int Hq, int Hkv, int B, int q_per, int weight_vnorm,
+                        float* __restrict__ parts, float scale_log2) {
   constexpr int ROWB = HD * 2;
   constexpr int TILE = 64 * ROWB;
   extern __shared__ __align__(128) uint8_t sm[];
   float* sL = reinterpret_cast<float*>(sm + 3 * TILE);  // 2 x 64 lse values
   const uint32_t sK = smem_u32(sm), sQ0 = sK + TILE;
 
-  const int kb = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+  const int kb = blockIdx.x, qc = blockIdx.y;
+  const int g = blockIdx.z % Hkv, b = blockIdx.z / Hkv;
   const int per = Hq / Hkv;
   const size_t ld = static_cast<size_t>(Hq + 2 * Hkv) * HD;
   const bf16* base = qkv + static_cast<size_t>(b) * N * ld;
@@ -229,10 +236,12 @@ __global__ void __launch_bounds__(128)
   const int gid = lane >> 2, tig = lane & 3;
   const int j_lo = kb * 64 + warp * 16 + gid, j_hi = j_lo + 8;
   const int n_qb = (N + 63) / 64;
-  const int steps = per * (n_qb - kb);
+  const int qb0 = max(kb, qc * q_per), qb1 = min(n_qb, (qc + 1) * q_per);
+  const int nq = qb1 > qb0 ? qb1 - qb0 : 0;
+  const int steps = per * nq;
 
   auto issue = [&](int step, int buf) {
-    const int hh = step / (n_qb - kb), qb = kb + step % (n_qb - kb);
+    const int hh = step / nq, qb = qb0 + step % nq;
     const int h = g * per + hh;
     load_tile64<HD>(sQ0 + buf * TILE, base + h * HD, ld, qb * 64, N);
     for (int i = threadIdx.x; i < 64; i += 128) {
@@ -241,69 +250,121 @@ __global__ void __launch_bounds__(128)
     }
   };
 
-  load_tile64<HD>(sK, Kg, ld, kb * 64, N);
-  issue(0, 0);
-  cp_async_commit();
-
-  uint32_t kf[HD / 16][4];
   float acc_lo = 0.f, acc_hi = 0.f;
-  for (int step = 0; step < steps; ++step) {
-    const int buf = step & 1;
-    if (step + 1 < steps) issue(step + 1, buf ^ 1);
+  if (steps > 0) {
+    load_tile64<HD>(sK, Kg, ld, kb * 64, N);
+    issue(0, 0);
     cp_async_commit();
-    cp_async_wait<1>();
-    __syncthreads();
-    if (step == 0) {
+    uint32_t kf[HD / 16][4];
+    for (int step = 0; step < steps; ++step) {
+      const int buf = step & 1;
+      if (step + 1 < steps) issue(step + 1, buf ^ 1);
+      cp_async_commit();
+      cp_async_wait<1>();
+      __syncthreads();
+      if (step == 0) {
 #pragma unroll
-      for (int kk = 0; kk < HD / 16; ++kk) {
-        const int mi = lane >> 3;
-        const int r = warp * 16 + (mi & 1) * 8 + (lane & 7);
-        ldsm_x4(sK + swz<ROWB>(r, kk * 2 + (mi >> 1)), kf[kk][0], kf[kk][1], kf[kk][2], kf[kk][3]);
-      }
-    }
-    const int qb = kb + step % (n_qb - kb);
-    const uint32_t sQ = sQ0 + buf * TILE;
-    float s[8][4];
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-#pragma unroll
-    for (int kk = 0; kk < HD / 16; ++kk) {
-#pragma unroll
-      for (int np = 0; np < 4; ++np) {
-        const int mi = lane >> 3;
-        const int r = np * 16 + (mi >> 1) * 8 + (lane & 7);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4(sQ + swz<ROWB>(r, kk * 2 + (mi & 1)), b0, b1, b2, b3);
-        mma_bf16_16816(s[2 * np], kf[kk], b0, b1);
-        mma_bf16_16816(s[2 * np + 1], kf[kk], b2, b3);
-      }
-    }
-    const float* L = sL + buf * 64;
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt) {
-#pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const int qi = nt * 8 + 2 * tig + e;
-        const int i = qb * 64 + qi;
-        if (i < N) {
-          const float l = L[qi];
-          if (i >= j_lo) acc_lo += exp2f(s[nt][e] * scale_log2 - l);
-          if (i >= j_hi) acc_hi += exp2f(s[nt][2 + e] * scale_log2 - l);
+        for (int kk = 0; kk < HD / 16; ++kk) {
+          const int mi = lane >> 3;
+          const int r = warp * 16 + (mi & 1) * 8 + (lane & 7);
+          ldsm_x4(sK + swz<ROWB>(r, kk * 2 + (mi >> 1)), kf[kk][0], kf[kk][1], kf[kk][2], kf[kk][3]);
         }
       }
+      const int qb = qb0 + step % nq;
+      const uint32_t sQ = sQ0 + buf * TILE;
+      float sacc[8][4];
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt) sacc[nt][0] = sacc[nt][1] = sacc[nt][2] = sacc[nt][3] = 0.f;
+#pragma unroll
+      for (int kk = 0; kk < HD / 16; ++kk) {
+#pragma unroll
+        for (int np = 0; np < 4; ++np) {
+          const int mi = lane >> 3;
+          const int r = np * 16 + (mi >> 1) * 8 + (lane & 7);
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4(sQ + swz<ROWB>(r, kk * 2 + (mi & 1)), b0, b1, b2, b3);
+          mma_bf16_16816(sacc[2 * np], kf[kk], b0, b1);
+          mma_bf16_16816(sacc[2 * np + 1], kf[kk], b2, b3);
+        }
+      }
+      const float* Lq = sL + buf * 64;
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt) {
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int qi = nt * 8 + 2 * tig + e;
+          const int i = qb * 64 + qi;
+          if (i < N) {
+            const float l = Lq[qi];
+            if (i >= j_lo) acc_lo += exp2f(sacc[nt][e] * scale_log2 - l);
+            if (i >= j_hi) acc_hi += exp2f(sacc[nt][2 + e] * scale_log2 - l);
+          }
+        }
+      }
+      __syncthreads();
     }
-    __syncthreads();
+    cp_async_wait<0>();
   }
-  cp_async_wait<0>();
   acc_lo += __shfl_xor_sync(0xffffffffu, acc_lo, 1);
   acc_lo += __shfl_xor_sync(0xffffffffu, acc_lo, 2);
   acc_hi += __shfl_xor_sync(0xffffffffu, acc_hi, 1);
   acc_hi += __shfl_xor_sync(0xffffffffu, acc_hi, 2);
-  if (tig == 0) {
-    float* Cg = C + (static_cast<size_t>(b) * Hkv + g) * N;
-    if (j_lo < N) Cg[j_lo] = acc_lo;
-    if (j_hi < N) Cg[j_hi] = acc_hi;
+  if (weight_vnorm) {
+    // ||v_j|| of group g: the quad (tig = 0..3) splits the hd dims of rows j_lo, j_hi
+    const bf16* Vg = base + (Hq + Hkv + g) * HD;
+    float ss_lo = 0.f, ss_hi = 0.f;
+    constexpr int QD = HD / 4;
+    if (j_lo < N) {
+      const uint4* v = reinterpret_cast<const uint4*>(Vg + static_cast<size_t>(j_lo) * ld + tig * QD);
+#pragma unroll
+      for (int q = 0; q < QD / 8; ++q) {
+        const uint4 u = v[q];
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) ss_lo += bf16lo(w[e]) * bf16lo(w[e]) + bf16hi(w[e]) * bf16hi(w[e]);
+      }
+    }
+    if (j_hi < N) {
+      const uint4* v = reinterpret_cast<const uint4*>(Vg + static_cast<size_t>(j_hi) * ld + tig * QD);
+#pragma unroll
+      for (int q = 0; q < QD / 8; ++q) {
+        const uint4 u = v[q];
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) ss_hi += bf16lo(w[e]) * bf16lo(w[e]) + bf16hi(w[e]) * bf16hi(w[e]);
+      }
+    }
+    ss_lo += __shfl_xor_sync(0xffffffffu, ss_lo, 1);
+    ss_lo += __shfl_xor_sync(0xffffffffu, ss_lo, 2);
+    ss_hi += __shfl_xor_sync(0xffffffffu, ss_hi, 1);
+    ss_hi += __shfl_xor_sync(0xffffffffu, ss_hi, 2);
+    acc_lo *= sqrtf(ss_lo);
+    acc_hi *= sqrtf(ss_hi);
   }
+  if (tig == 0) {
+    float* P = parts + ((static_cast<size_t>(qc) * B + b) * Hkv + g) * N;
+    if (j_lo < N) P[j_lo] = acc_lo;
+    if (j_hi < N) P[j_hi] = acc_hi;
+  }
+}
+
+// out[b][g][j] = sum_qc parts[qc][b][g][j]                      (sum_groups = 0)
+// out[b][j]    = sum_qc sum_g parts[qc][b][g][j]                 (sum_groups = 1)
+__global__ void colmass_reduce_kernel(const float* __restrict__ parts, int n_qc, int B, int G,
+                                      int N, int sum_groups, float* __restrict__ out) {
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  const int total = sum_groups ? B * N : B * G * N;
+  if (idx >= total) return;
+  const size_t plane = static_cast<size_t>(B) * G * N;
+  float acc = 0.f;
+  if (sum_groups) {
+    const int b = idx / N, j = idx % N;
+    for (int qc = 0; qc < n_qc; ++qc)
+      for (int g = 0; g < G; ++g) acc += parts[qc * plane + (static_cast<size_t>(b) * G + g) * N + j];
+  } else {
+    for (int qc = 0; qc < n_qc; ++qc) acc += parts[qc * plane + idx];
+  }
+  out[idx] = acc;
 }
 
 // fp32 attention: one warp per (query i, head h, batch b).
@@ -359,10 +420,10 @@ __global__ void attn_fwd_f32_kernel(const float* __restrict__ qkv, int N, int Hq
   if (lane == 0) lse2[(static_cast<size_t>(b) * Hq + h) * N + i] = lse;
 }
 
-// fp32 column mass: one warp per (key j, KV head g, batch b).
+// fp32 column mass: one warp per (key j, KV head g, batch b); one query chunk.
 __global__ void colmass_f32_kernel(const float* __restrict__ qkv, const float* __restrict__ lse2,
-                                   int N, int Hq, int Hkv, int hd, float* __restrict__ C,
-                                   float scale_log2) {
+                                   int N, int Hq, int Hkv, int hd, int B, int weight_vnorm,
+                                   float* __restrict__ parts, float scale_log2) {
   const int j = blockIdx.x * 4 + (threadIdx.x >> 5);
   const int g = blockIdx.y, b = blockIdx.z, lane = threadIdx.x & 31;
   if (j >= N) return;
@@ -381,7 +442,13 @@ __global__ void colmass_f32_kernel(const float* __restrict__ qkv, const float* _
     }
   }
   acc = warp_sum(acc);
-  if (lane == 0) C[(static_cast<size_t>(b) * Hkv + g) * N + j] = acc;
+  if (weight_vnorm) {
+    const float* v = base + j * ld + (Hq + Hkv + g) * hd;
+    float ss = 0.f;
+    for (int e = lane; e < hd; e += 32) ss = fmaf(v[e], v[e], ss);
+    acc *= sqrtf(warp_sum(ss));
+  }
+  if (lane == 0) parts[(static_cast<size_t>(b) * Hkv + g) * N + j] = acc;
 }
 
 template <typename Kern>
@@ -419,31 +486,69 @@ cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, i
   return cudaGetLastError();
 }
 
-cudaError_t launch_colmass(int dtype, const void* qkv, const float* lse, int B, int N, int Hq,
-                           int Hkv, int hd, float* C, cudaStream_t s) {
+int colmass_chunks(int N) {
+  const int n_qb = (N + 63) / 64;
+  return (n_qb + kColmassQPer - 1) / kColmassQPer;
+}
+
+size_t colmass_parts_elems(int B, int N, int Hkv) {
+  return static_cast<size_t>(colmass_chunks(N)) * B * Hkv * N;
+}
+
+namespace {
+cudaError_t colmass_parts(int dtype, const void* qkv, const float* lse, int B, int N, int Hq,
+                          int Hkv, int hd, int weight_vnorm, float* parts, int* n_qc,
+                          cudaStream_t s) {
   const float scale_log2 = kLog2e / sqrtf(static_cast<float>(hd));
   if (dtype == ZSAA_F32) {
+    *n_qc = 1;
     dim3 grid((N + 3) / 4, Hkv, B);
-    colmass_f32_kernel<<<grid, 128, 0, s>>>(static_cast<const float*>(qkv), lse, N, Hq, Hkv, hd,
-                                            C, scale_log2);
+    colmass_f32_kernel<<<grid, 128, 0, s>>>(static_cast<const float*>(qkv), lse, N, Hq, Hkv, hd, B,
+                                            weight_vnorm, parts, scale_log2);
     return cudaGetLastError();
   }
-  dim3 grid((N + 63) / 64, Hkv, B);
+  *n_qc = colmass_chunks(N);
+  dim3 grid((N + 63) / 64, *n_qc, Hkv * B);
   if (hd == 64) {
     const int smem = 3 * 64 * 128 + 2 * 64 * 4;
     static cudaError_t e = set_smem(colmass_bf16_kernel<64>, smem);
     if (e != cudaSuccess) return e;
     colmass_bf16_kernel<64><<<grid, 128, smem, s>>>(static_cast<const bf16*>(qkv), lse, N, Hq,
-                                                     Hkv, C, scale_log2);
+                                                     Hkv, B, kColmassQPer, weight_vnorm, parts,
+                                                     scale_log2);
   } else if (hd == 128) {
     const int smem = 3 * 64 * 256 + 2 * 64 * 4;
     static cudaError_t e = set_smem(colmass_bf16_kernel<128>, smem);
     if (e != cudaSuccess) return e;
     colmass_bf16_kernel<128><<<grid, 128, smem, s>>>(static_cast<const bf16*>(qkv), lse, N, Hq,
-                                                      Hkv, C, scale_log2);
+                                                      Hkv, B, kColmassQPer, weight_vnorm, parts,
+                                                      scale_log2);
   } else {
     return cudaErrorInvalidValue;
   }
+  return cudaGetLastError();
+}
+}  // namespace
+
+cudaError_t launch_colmass(int dtype, const void* qkv, const float* lse, int B, int N, int Hq,
+                           int Hkv, int hd, float* parts, float* C, cudaStream_t s) {
+  int n_qc = 1;
+  cudaError_t e = colmass_parts(dtype, qkv, lse, B, N, Hq, Hkv, hd, 0, parts, &n_qc, s);
+  if (e != cudaSuccess) return e;
+  const int total = B * Hkv * N;
+  colmass_reduce_kernel<<<(total + 255) / 256, 256, 0, s>>>(parts, n_qc, B, Hkv, N, 0, C);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_position_scores(int dtype, const void* qkv, const float* lse, int B, int N,
+                                   int Hq, int Hkv, int hd, int mode, float* parts,
+                                   float* scores, cudaStream_t s) {
+  int n_qc = 1;
+  cudaError_t e = colmass_parts(dtype, qkv, lse, B, N, Hq, Hkv, hd,
+                                mode == ZSAA_SCORE_SOFTSCORE_VNORM ? 1 : 0, parts, &n_qc, s);
+  if (e != cudaSuccess) return e;
+  const int total = B * N;
+  colmass_reduce_kernel<<<(total + 255) / 256, 256, 0, s>>>(parts, n_qc, B, Hkv, N, 1, scores);
   return cudaGetLastError();
 }
 

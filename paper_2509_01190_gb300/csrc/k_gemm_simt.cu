@@ -73,6 +73,7 @@ __global__ void __launch_bounds__(256)
 
 cudaError_t launch_gemm_f32(const float* A, int lda, const float* W, const float* W2, int epi,
                             const GemmParams& p, cudaStream_t s) {
+  if (p.launches) *p.launches += 1;
   dim3 grid((p.N + TB - 1) / TB, (p.M + TB - 1) / TB);
   if (epi == kEpiSwiGLU)
     gemm_f32_kernel<true><<<grid, 256, 0, s>>>(A, lda, W, W2, p.M, p.N, p.K, epi,

@@ -73,15 +73,20 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
   if (ts.splits > 1) {  // fp32 partial of this split, virtual column layout
     float* ws = ts.ws + (static_cast<size_t>(ks) * p.M + row) * ts.vn + n0;
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 16) {
-      uint32_t r[16];
+    for (int c = 0; c < BN; c += 32) {
+      uint32_t r[32];
       __syncwarp();
-      tmem_ld16(tbase + c, r);
+      tmem_ld16(tbase + c, *reinterpret_cast<uint32_t(*)[16]>(r));
+      tmem_ld16(tbase + c + 16, *reinterpret_cast<uint32_t(*)[16]>(r + 16));
       tmem_ld_wait();
-      if (row_ok && n0 + c < ts.vn) {
-        uint4* dst = reinterpret_cast<uint4*>(ws + c);
 #pragma unroll
-        for (int q = 0; q < 4; ++q) dst[q] = make_uint4(r[4 * q], r[4 * q + 1], r[4 * q + 2], r[4 * q + 3]);
+      for (int h = 0; h < 2; ++h) {
+        if (row_ok && n0 + c + 16 * h < ts.vn) {
+          uint4* dst = reinterpret_cast<uint4*>(ws + c + 16 * h);
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            dst[q] = make_uint4(r[16 * h + 4 * q], r[16 * h + 4 * q + 1], r[16 * h + 4 * q + 2], r[16 * h + 4 * q + 3]);
+        }
       }
     }
     return;
@@ -106,15 +111,20 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
   } else if (EPI == kEpiStoreF32) {
     float* out = static_cast<float*>(p.out);
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 16) {
-      uint32_t r[16];
+    for (int c = 0; c < BN; c += 32) {
+      uint32_t r[32];
       __syncwarp();
-      tmem_ld16(tbase + c, r);
+      tmem_ld16(tbase + c, *reinterpret_cast<uint32_t(*)[16]>(r));
+      tmem_ld16(tbase + c + 16, *reinterpret_cast<uint32_t(*)[16]>(r + 16));
       tmem_ld_wait();
-      if (row_ok && n0 + c < p.N) {
-        uint4* dst = reinterpret_cast<uint4*>(out + static_cast<size_t>(row) * p.ldo + n0 + c);
 #pragma unroll
-        for (int q = 0; q < 4; ++q) dst[q] = make_uint4(r[4 * q], r[4 * q + 1], r[4 * q + 2], r[4 * q + 3]);
+      for (int h = 0; h < 2; ++h) {
+        if (row_ok && n0 + c + 16 * h < p.N) {
+          uint4* dst = reinterpret_cast<uint4*>(out + static_cast<size_t>(row) * p.ldo + n0 + c + 16 * h);
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            dst[q] = make_uint4(r[16 * h + 4 * q], r[16 * h + 4 * q + 1], r[16 * h + 4 * q + 2], r[16 * h + 4 * q + 3]);
+        }
       }
     }
   } else if (EPI == kEpiRope) {
@@ -127,6 +137,16 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
 #pragma unroll 1
       for (int c = 0; c < half; c += 16) {
         uint32_t x1[16], x2[16];
+        float4 cs4[4], sn4[4];
+        if (rot && row_ok) {  // table loads first: their latency overlaps the TMEM load
+          const float4* cp = reinterpret_cast<const float4*>(p.cos_t + static_cast<size_t>(ps) * half + c);
+          const float4* sp = reinterpret_cast<const float4*>(p.sin_t + static_cast<size_t>(ps) * half + c);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            cs4[q] = __ldg(cp + q);
+            sn4[q] = __ldg(sp + q);
+          }
+        }
         __syncwarp();
         tmem_ld16(tbase + hs + c, x1);
         tmem_ld16(tbase + hs + half + c, x2);
@@ -134,11 +154,9 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
         if (row_ok && n0 + hs < p.N) {
           float y1[16], y2[16];
           if (rot) {
-            const float4* cp = reinterpret_cast<const float4*>(p.cos_t + static_cast<size_t>(ps) * half + c);
-            const float4* sp = reinterpret_cast<const float4*>(p.sin_t + static_cast<size_t>(ps) * half + c);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
-              const float4 cs = __ldg(cp + q), sn = __ldg(sp + q);
+              const float4 cs = cs4[q], sn = sn4[q];
               const float cv[4] = {cs.x, cs.y, cs.z, cs.w}, sv[4] = {sn.x, sn.y, sn.z, sn.w};
 #pragma unroll
               for (int e = 0; e < 4; ++e) {
@@ -163,29 +181,49 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
   } else {  // kEpiStore / kEpiResid, bf16 out
     bf16* out = static_cast<bf16*>(p.out);
     const bf16* res = static_cast<const bf16*>(p.resid);
-#pragma unroll 1
-    for (int c = 0; c < BN; c += 16) {
-      uint32_t r[16];
-      __syncwarp();
-      tmem_ld16(tbase + c, r);
-      tmem_ld_wait();
-      if (row_ok && n0 + c < p.N) {
-        const size_t off = static_cast<size_t>(row) * p.ldo + n0 + c;
-        float v[16];
+    const size_t rowoff = static_cast<size_t>(row) * p.ldo + n0;
+    uint4 rc[4], rn[4];
+    auto load_res = [&](int c, uint4 (&r)[4]) {
 #pragma unroll
-        for (int e = 0; e < 16; ++e) v[e] = __uint_as_float(r[e]);
-        if (EPI == kEpiResid) {
-          const uint4* rp = reinterpret_cast<const uint4*>(res + off);
-          const uint4 r0 = rp[0], r1 = rp[1];
-          const uint32_t rr[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            v[2 * e] += bf16lo(rr[e]);
-            v[2 * e + 1] += bf16hi(rr[e]);
-          }
+      for (int h = 0; h < 2; ++h) {
+        if (EPI == kEpiResid && row_ok && n0 + c + 16 * h < p.N) {
+          const uint4* rp = reinterpret_cast<const uint4*>(res + rowoff + c + 16 * h);
+          r[2 * h] = rp[0];
+          r[2 * h + 1] = rp[1];
+        } else {
+          r[2 * h] = r[2 * h + 1] = make_uint4(0u, 0u, 0u, 0u);
         }
-        store_bf16x16(out + off, v);
       }
+    };
+    load_res(0, rc);
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      if (c + 32 < BN) load_res(c + 32, rn);  // in flight while this chunk drains TMEM
+      uint32_t r[32];
+      __syncwarp();
+      tmem_ld16(tbase + c, *reinterpret_cast<uint32_t(*)[16]>(r));
+      tmem_ld16(tbase + c + 16, *reinterpret_cast<uint32_t(*)[16]>(r + 16));
+      tmem_ld_wait();
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        if (row_ok && n0 + c + 16 * h < p.N) {
+          float v[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) v[e] = __uint_as_float(r[16 * h + e]);
+          if (EPI == kEpiResid) {
+            const uint32_t rr[8] = {rc[2 * h].x, rc[2 * h].y, rc[2 * h].z, rc[2 * h].w,
+                                    rc[2 * h + 1].x, rc[2 * h + 1].y, rc[2 * h + 1].z, rc[2 * h + 1].w};
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              v[2 * e] += bf16lo(rr[e]);
+              v[2 * e + 1] += bf16hi(rr[e]);
+            }
+          }
+          store_bf16x16(out + rowoff + c + 16 * h, v);
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) rc[q] = rn[q];
     }
   }
 }
@@ -470,7 +508,9 @@ cudaError_t run_tc(const TcMaps& maps, int n1, int n2, const GemmParams& p, cons
   const int grid = ts.total < num_sms() ? ts.total : num_sms();
   gemm_tc_kernel<BN, EPI><<<grid, kThreads, C::SMEM, s>>>(maps, n1, n2, p, ts);
   cudaError_t e = cudaGetLastError();
+  if (p.launches) *p.launches += 1;
   if (e != cudaSuccess || ts.splits == 1) return e;
+  if (p.launches) *p.launches += 1;
   const int ncols = EPI == kEpiRope ? p.rope_cols / 2 + (p.N - p.rope_cols) : p.N;
   const int chunks = (ncols + 7) / 8;
   dim3 fgrid((chunks + 127) / 128, p.M);

@@ -1,6 +1,6 @@
-// Row-wise kernels of the pruned prefill: embedding gather, RMSNorm, position
-// scores (Sec. 3.2-3.3), per-sequence top-k selection, row compaction, fp32
-// RoPE and the classifier head.  All are HBM-bound: one warp per row, 16-byte
+// Row-wise kernels of the pruned prefill: embedding gather, RMSNorm, row-norm
+// scores of the isolated path (Sec. 3.3 with unit column mass), per-sequence
+// top-k selection, row compaction, fp32 RoPE and the classifier head.  All are HBM-bound: one warp per row, 16-byte
 // vector accesses, fp32 arithmetic.
 #include "common.cuh"
 #include "kernels.h"
@@ -138,34 +138,6 @@ __global__ void row_norm_f32_kernel(const float* __restrict__ h, int rows, int d
   for (int i = lane; i < d; i += 32) ss = fmaf(hr[i], hr[i], ss);
   ss = warp_sum(ss);
   if (lane == 0) s[r] = sqrtf(ss);
-}
-
-// s[b, j] = sum_g C[b, g, j] * ||v[b, j, g, :]||  (mode 0) or sum_g C[b, g, j] (mode 1)
-template <typename T>
-__global__ void score_colmass_kernel(const T* __restrict__ qkv, int ld, int v_off,
-                                     const float* __restrict__ C, int B, int N, int G, int hd,
-                                     int mode, float* __restrict__ s) {
-  const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  if (r >= B * N) return;
-  const int b = r / N, j = r % N;
-  const T* v = qkv + static_cast<size_t>(r) * ld + v_off;
-  float acc = 0.f;
-  for (int g = 0; g < G; ++g) {
-    const float c = C[(static_cast<size_t>(b) * G + g) * N + j];
-    if (mode == ZSAA_SCORE_SOFTSCORE) {
-      acc += c;
-    } else {
-      float ss = 0.f;
-      for (int e = lane; e < hd; e += 32) {
-        float x = to_f(v[g * hd + e]);
-        ss = fmaf(x, x, ss);
-      }
-      ss = warp_sum(ss);
-      acc = fmaf(c, sqrtf(ss), acc);
-    }
-  }
-  if (lane == 0) s[r] = acc;
 }
 
 // ---------------------------------------------------------------- top-k select
@@ -419,19 +391,6 @@ cudaError_t launch_row_norm(int dtype, const void* h, int rows, int d, float* sc
     row_norm_f32_kernel<<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
         static_cast<const float*>(h), rows, d, scores);
   }
-  return cudaGetLastError();
-}
-
-cudaError_t launch_score_colmass(int dtype, const void* qkv, int ld, int v_off, const float* C,
-                                 int B, int N, int G, int hd, int mode, float* scores,
-                                 cudaStream_t s) {
-  const int rows = B * N;
-  if (dtype == ZSAA_BF16)
-    score_colmass_kernel<bf16><<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
-        static_cast<const bf16*>(qkv), ld, v_off, C, B, N, G, hd, mode, scores);
-  else
-    score_colmass_kernel<float><<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
-        static_cast<const float*>(qkv), ld, v_off, C, B, N, G, hd, mode, scores);
   return cudaGetLastError();
 }
 

@@ -14,9 +14,6 @@ cudaError_t launch_rmsnorm(int dtype, const void* h, const void* w, int rows, in
                            void* x, cudaStream_t s);
 cudaError_t launch_row_norm(int dtype, const void* h, int rows, int d, float* scores,
                             cudaStream_t s);
-cudaError_t launch_score_colmass(int dtype, const void* qkv, int ld, int v_off, const float* C,
-                                 int B, int N, int G, int hd, int mode, float* scores,
-                                 cudaStream_t s);
 cudaError_t launch_select(const float* scores, int B, int N, int k, int force_last, int32_t* idx,
                           cudaStream_t s);
 cudaError_t launch_gather(const void* src, int B, int N, int k, int row_bytes, const int32_t* idx,
@@ -44,6 +41,7 @@ struct GemmParams {
   int* status;          // device status word
   float* splitk_ws;     // optional fp32 workspace for split-K partial tiles (NULL: no split)
   size_t splitk_ws_elems;
+  int* launches;        // optional host counter: kernels launched are added to it
 };
 
 // Split-K workspace a caller should provide: two waves of 128 x 256 fp32 tiles.
@@ -69,8 +67,18 @@ cudaError_t launch_gemm_f32(const float* A, int lda, const float* W, const float
 // ---- attention (k_attn.cu)
 cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, int Hkv, int hd,
                              void* out, float* lse, cudaStream_t s);
+// Column mass C[B, Hkv, N] (via query-chunk partials in `parts`, which must
+// hold colmass_parts_elems(B, N, Hkv) floats).
+constexpr int kColmassQPer = 2;  // query blocks of 64 per column-mass CTA
+int colmass_chunks(int N);
+size_t colmass_parts_elems(int B, int N, int Hkv);
 cudaError_t launch_colmass(int dtype, const void* qkv, const float* lse, int B, int N, int Hq,
-                           int Hkv, int hd, float* C, cudaStream_t s);
+                           int Hkv, int hd, float* parts, float* C, cudaStream_t s);
+// Position scores s[B, N] of R1 (mode ZSAA_SCORE_*): column mass weighted by
+// ||v|| per group, summed over groups; same workspace as launch_colmass.
+cudaError_t launch_position_scores(int dtype, const void* qkv, const float* lse, int B, int N,
+                                   int Hq, int Hkv, int hd, int mode, float* parts,
+                                   float* scores, cudaStream_t s);
 
 // ---- thread-local message returned by zsaa_last_error (zsaa_api.cu)
 void set_last_error(const char* msg);

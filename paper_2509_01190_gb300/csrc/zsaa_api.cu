@@ -12,6 +12,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <list>
 #include <mutex>
 #include <string>
 #include <unordered_map>
@@ -253,7 +254,7 @@ struct zsaa_model {
   void* attn = nullptr;
   void* act = nullptr;
   float* lse = nullptr;
-  float* colmass = nullptr;
+  float* colmass = nullptr;  // query-chunk partials of the column mass / scores
   float* scores = nullptr;
   int32_t* idx = nullptr;
   int32_t* pos[2] = {nullptr, nullptr};
@@ -269,6 +270,7 @@ struct zsaa_model {
   // tracing (zsaa_trace_begin / _end)
   struct TraceRec {
     int cls;
+    int kernels;
     cudaEvent_t a, b;
     double flops, bytes;
   };
@@ -277,6 +279,15 @@ struct zsaa_model {
   std::vector<cudaEvent_t> ev_pool;
   size_t ev_used = 0;
   std::vector<std::string> trace_names;
+  // CUDA graphs of plain forwards, keyed by their arguments (most recent first)
+  struct GraphEntry {
+    std::string key;
+    int seen = 0;                 // eager runs so far with this key
+    cudaGraphExec_t exec = nullptr;
+  };
+  bool use_graphs = true;
+  std::list<GraphEntry> graphs;
+  cudaStream_t capture_stream = nullptr;  // graphs are recorded here, launched on the caller's
 };
 
 namespace {
@@ -307,8 +318,10 @@ class TraceScope {
     if (rec_.a && rec_.b && cudaEventRecord(rec_.a, s) == cudaSuccess) active_ = true;
   }
   ~TraceScope() {
+    rec_.kernels = kernels;
     if (active_ && cudaEventRecord(rec_.b, s_) == cudaSuccess) m_->trace.push_back(rec_);
   }
+  int kernels = 1;  // kernels launched inside the scope
 
  private:
   cudaEvent_t event() {
@@ -328,6 +341,9 @@ class TraceScope {
 void free_model(zsaa_model* m) {
   if (m == nullptr) return;
   for (cudaEvent_t e : m->ev_pool) cudaEventDestroy(e);
+  for (auto& g : m->graphs)
+    if (g.exec) cudaGraphExecDestroy(g.exec);
+  if (m->capture_stream) cudaStreamDestroy(m->capture_stream);
   void* ptrs[] = {m->h[0], m->h[1], m->x, m->qkv, m->attn, m->act, m->lse, m->colmass,
                   m->scores, m->idx, m->pos[0], m->pos[1], m->rope_cos, m->rope_sin,
                   m->splitk_ws, m->status, m->stage_tok, m->stage_logits, m->stage_pos};
@@ -338,10 +354,11 @@ void free_model(zsaa_model* m) {
 
 // out[M, N] = epi(A W^T) on the model's dtype path.
 zsaa_status linear(zsaa_model* m, const void* A, int lda, const TcWeights& W, int epi,
-                   GemmParams p, cudaStream_t s) {
+                   GemmParams p, cudaStream_t s, int* kernels = nullptr) {
   p.status = m->status;
   p.splitk_ws = m->splitk_ws;
   p.splitk_ws_elems = m->splitk_ws ? kSplitKWorkspaceElems : 0;
+  p.launches = kernels;
   if (m->cfg.dtype == ZSAA_BF16) {
     ZCK(launch_gemm_tc(A, lda, W, epi, p, s));
   } else {
@@ -430,10 +447,12 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
       p.hd = hd;
       TcWeights W{LW(m, li, kWq), LW(m, li, kWk), LW(m, li, kWv), m->dq, m->dq + m->dkv};
       TRACE("gemm_qkv_rope", 2.0 * Md * m->ld_qkv * d, (Md * d + static_cast<double>(m->ld_qkv) * d + Md * m->ld_qkv) * es);
-      st = linear(m, m->x, d, W, kEpiRope, p, s);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->x, d, W, kEpiRope, p, s, &trace_scope_.kernels);
       if (st != ZSAA_OK) return st;
     } else {
       TRACE("gemm_qkv_f32", 2.0 * Md * m->ld_qkv * d, (Md * d + static_cast<double>(m->ld_qkv) * d + Md * m->ld_qkv) * es);
+      trace_scope_.kernels = 1;  // the RoPE kernel below; the GEMMs add theirs
       const int cols[3] = {m->dq, m->dkv, m->dkv};
       const int slots[3] = {kWq, kWk, kWv};
       int c0 = 0;
@@ -442,7 +461,7 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
         q.N = cols[t];
         q.out = static_cast<float*>(m->qkv) + c0;
         TcWeights W{LW(m, li, slots[t]), nullptr, nullptr, cols[t], cols[t]};
-        st = linear(m, m->x, d, W, kEpiStore, q, s);
+        st = linear(m, m->x, d, W, kEpiStore, q, s, &trace_scope_.kernels);
         if (st != ZSAA_OK) return st;
         c0 += cols[t];
       }
@@ -464,7 +483,8 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
       q.resid = h;
       TcWeights W{LW(m, li, kWo), nullptr, nullptr, d, d};
       TRACE("gemm_o_resid", 2.0 * Md * d * m->dq, (Md * m->dq + static_cast<double>(d) * m->dq + 2.0 * Md * d) * es);
-      st = linear(m, m->attn, m->dq, W, kEpiResid, q, s);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->attn, m->dq, W, kEpiResid, q, s, &trace_scope_.kernels);
       if (st != ZSAA_OK) return st;
     }
     // MLP branch
@@ -482,7 +502,8 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
       TcWeights W{LW(m, li, kWg), LW(m, li, kWu), nullptr, c.ffn_dim, c.ffn_dim};
       const double F = c.ffn_dim;
       TRACE("gemm_gate_up_swiglu", 4.0 * Md * F * d, (Md * d + 2.0 * F * d + Md * F) * es);
-      st = linear(m, m->x, d, W, kEpiSwiGLU, q, s);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->x, d, W, kEpiSwiGLU, q, s, &trace_scope_.kernels);
       if (st != ZSAA_OK) return st;
     }
     {
@@ -496,7 +517,8 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
       TcWeights W{LW(m, li, kWd), nullptr, nullptr, d, d};
       const double F = c.ffn_dim;
       TRACE("gemm_down_resid", 2.0 * Md * d * F, (Md * F + F * d + 2.0 * Md * d) * es);
-      st = linear(m, m->act, c.ffn_dim, W, kEpiResid, q, s);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->act, c.ffn_dim, W, kEpiResid, q, s, &trace_scope_.kernels);
       if (st != ZSAA_OK) return st;
     }
     // elimination after the layer (Sec. 3.3)
@@ -509,14 +531,11 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
         float* sc = want_scores ? opts->scores_out + off_scores : m->scores;
         {
           const double pairs = static_cast<double>(B) * Hq * (static_cast<double>(N) * (N + 1) / 2.0);
-          TRACE("colmass", 2.0 * pairs * hd,
-                Md * (m->dq + m->dkv) * es + static_cast<double>(B) * (Hq + Hkv) * N * 4.0);
-          ZCK(launch_colmass(dt, m->qkv, m->lse, B, N, Hq, Hkv, hd, m->colmass, s));
-        }
-        {
-          TRACE("score", 0.0, Md * m->dkv * es + Md * (Hkv + 1) * 4.0);
-          ZCK(launch_score_colmass(dt, m->qkv, m->ld_qkv, m->dq + m->dkv, m->colmass, B, N, Hkv, hd,
-                                   c.score_mode, sc, s));
+          TRACE("colmass_score", 2.0 * pairs * hd,
+                Md * (m->dq + 2 * m->dkv) * es + static_cast<double>(B) * Hq * N * 4.0 + Md * 4.0);
+          trace_scope_.kernels = 2;
+          ZCK(launch_position_scores(dt, m->qkv, m->lse, B, N, Hq, Hkv, hd, c.score_mode, m->colmass,
+                                     sc, s));
         }
         const int32_t* idx = m->idx;
         if (forced) {
@@ -563,12 +582,71 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
     TcWeights W{m->head, nullptr, nullptr, c.vocab, c.vocab};
     const double V = c.vocab, Mh = M;
     TRACE("gemm_lm_head", 2.0 * Mh * V * d, (Mh * d + V * d) * es + Mh * V * 4.0);
-    st = linear(m, m->x, d, W, dt == ZSAA_BF16 ? kEpiStoreF32 : kEpiStore, q, s);
+    trace_scope_.kernels = 0;
+    st = linear(m, m->x, d, W, dt == ZSAA_BF16 ? kEpiStoreF32 : kEpiStore, q, s, &trace_scope_.kernels);
     if (st != ZSAA_OK) return st;
   }
   if (kept_pos)
     ZCK(cudaMemcpyAsync(kept_pos, m->pos[cur], sizeof(int32_t) * M, cudaMemcpyDeviceToDevice, s));
 #undef TRACE
+  return ZSAA_OK;
+}
+
+// A plain forward (no hooks, not tracing) is replayed from a CUDA graph: the
+// first call with given arguments runs eagerly, the second is captured and
+// instantiated, later ones launch the graph (one launch instead of ~175 and
+// no per-call host work).  At most kMaxGraphs argument sets are kept.
+constexpr size_t kMaxGraphs = 16;
+
+zsaa_status forward_cached(zsaa_model* m, const int32_t* tok, int B, int L, double accel,
+                           float* logits, int32_t* kept_pos, cudaStream_t s) {
+  if (!m->use_graphs || m->tracing)
+    return run_forward(m, tok, B, L, accel, logits, kept_pos, nullptr, s);
+  char key[160];
+  snprintf(key, sizeof(key), "%p/%d/%d/%.17g/%p/%p", static_cast<const void*>(tok), B, L, accel,
+           static_cast<void*>(logits), static_cast<void*>(kept_pos));
+  auto it = m->graphs.begin();
+  for (; it != m->graphs.end(); ++it)
+    if (it->key == key) break;
+  if (it == m->graphs.end()) {
+    m->graphs.push_front(zsaa_model::GraphEntry{key, 0, nullptr});
+    if (m->graphs.size() > kMaxGraphs) {
+      if (m->graphs.back().exec) cudaGraphExecDestroy(m->graphs.back().exec);
+      m->graphs.pop_back();
+    }
+    it = m->graphs.begin();
+  } else if (it != m->graphs.begin()) {
+    m->graphs.splice(m->graphs.begin(), m->graphs, it);
+    it = m->graphs.begin();
+  }
+  if (it->exec != nullptr) {
+    ZCK(cudaGraphLaunch(it->exec, s));
+    return ZSAA_OK;
+  }
+  if (it->seen == 0) {  // first sight: eager (also sets up kernel attributes)
+    zsaa_status st = run_forward(m, tok, B, L, accel, logits, kept_pos, nullptr, s);
+    if (st == ZSAA_OK) it->seen = 1;
+    return st;
+  }
+  // Record on the model's own stream (capture is impossible on the legacy
+  // default stream); recording executes nothing, the launch below does.
+  if (m->capture_stream == nullptr)
+    ZCK(cudaStreamCreateWithFlags(&m->capture_stream, cudaStreamNonBlocking));
+  cudaGraph_t graph = nullptr;
+  ZCK(cudaStreamBeginCapture(m->capture_stream, cudaStreamCaptureModeThreadLocal));
+  zsaa_status st = run_forward(m, tok, B, L, accel, logits, kept_pos, nullptr, m->capture_stream);
+  cudaError_t e = cudaStreamEndCapture(m->capture_stream, &graph);
+  if (st != ZSAA_OK) {
+    if (graph) cudaGraphDestroy(graph);
+    return st;
+  }
+  ZCK(e);
+  cudaGraphExec_t exec = nullptr;
+  e = cudaGraphInstantiate(&exec, graph, 0);
+  cudaGraphDestroy(graph);
+  ZCK(e);
+  it->exec = exec;
+  ZCK(cudaGraphLaunch(exec, s));
   return ZSAA_OK;
 }
 
@@ -690,7 +768,8 @@ zsaa_status zsaa_model_create(const zsaa_config* cfg, const zsaa_weights* w, int
   alloc(&m->attn, rows * m->dq * esz);
   alloc(&m->act, rows * F * esz);
   alloc(reinterpret_cast<void**>(&m->lse), rows * cfg->n_heads * sizeof(float));
-  alloc(reinterpret_cast<void**>(&m->colmass), rows * cfg->n_kv_heads * sizeof(float));
+  alloc(reinterpret_cast<void**>(&m->colmass),
+        colmass_parts_elems(max_B, max_L, cfg->n_kv_heads) * sizeof(float));
   alloc(reinterpret_cast<void**>(&m->scores), rows * sizeof(float));
   alloc(reinterpret_cast<void**>(&m->idx), rows * sizeof(int32_t));
   alloc(reinterpret_cast<void**>(&m->pos[0]), rows * sizeof(int32_t));
@@ -745,8 +824,14 @@ zsaa_status zsaa_plan(const zsaa_model* m, int L, double accel, int* n_sched, do
 zsaa_status zsaa_forward(zsaa_model* m, const int32_t* token_ids, int B, int L, double accel,
                          float* logits_out, int32_t* kept_pos_out, zsaa_stream stream) {
   if (m == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null model");
-  return run_forward(m, token_ids, B, L, accel, logits_out, kept_pos_out, nullptr,
-                     reinterpret_cast<cudaStream_t>(stream));
+  return forward_cached(m, token_ids, B, L, accel, logits_out, kept_pos_out,
+                        reinterpret_cast<cudaStream_t>(stream));
+}
+
+zsaa_status zsaa_model_set_graphs(zsaa_model* m, int enable) {
+  if (m == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null model");
+  m->use_graphs = enable != 0;
+  return ZSAA_OK;
 }
 
 zsaa_status zsaa_forward_ex(zsaa_model* m, const int32_t* token_ids, int B, int L, double accel,
@@ -783,7 +868,7 @@ zsaa_status zsaa_forward_host(zsaa_model* m, const int32_t* token_ids, int B, in
     m->stage_logits_cap = n_logits;
   }
   ZCK(cudaMemcpyAsync(m->stage_tok, token_ids, sizeof(int32_t) * B * L, cudaMemcpyHostToDevice, s));
-  st = run_forward(m, m->stage_tok, B, L, accel, m->stage_logits, m->stage_pos, nullptr, s);
+  st = forward_cached(m, m->stage_tok, B, L, accel, m->stage_logits, m->stage_pos, s);
   if (st != ZSAA_OK) return st;
   ZCK(cudaMemcpyAsync(logits_out, m->stage_logits, n_logits * sizeof(float), cudaMemcpyDeviceToHost, s));
   if (kept_pos_out)
@@ -867,7 +952,14 @@ zsaa_status zsaa_op_colmass(const void* qkv, const float* lse, int B, int N, int
   if (qkv == nullptr || lse == nullptr || colmass == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null argument");
   if (B < 1 || N < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv) return fail(ZSAA_ERR_INVALID_ARG, "bad shape");
   if (dtype == ZSAA_BF16 && hd != 64 && hd != 128) return fail(ZSAA_ERR_UNSUPPORTED, "bf16 column mass needs hd 64 or 128");
-  ZCK(launch_colmass(dtype, qkv, lse, B, N, Hq, Hkv, hd, colmass, reinterpret_cast<cudaStream_t>(stream)));
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  float* parts = nullptr;
+  ZCK(cudaMallocAsync(reinterpret_cast<void**>(&parts),
+                      colmass_parts_elems(B, N, Hkv) * sizeof(float), s));
+  cudaError_t e = launch_colmass(dtype, qkv, lse, B, N, Hq, Hkv, hd, parts, colmass, s);
+  cudaError_t e2 = cudaFreeAsync(parts, s);
+  ZCK(e);
+  ZCK(e2);
   return ZSAA_OK;
 }
 
@@ -893,7 +985,7 @@ zsaa_status zsaa_trace_end(zsaa_model* m, zsaa_trace_row* rows, int max_rows, in
     float ms = 0.f;
     ZCK(cudaEventElapsedTime(&ms, r.a, r.b));
     zsaa_trace_row& a = agg[r.cls];
-    a.launches += 1;
+    a.launches += r.kernels;
     a.ms += ms;
     a.flops += r.flops;
     a.bytes += r.bytes;

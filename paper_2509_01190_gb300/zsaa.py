@@ -27,7 +27,7 @@ EXPORTED = [
     "zsaa_forward_ex", "zsaa_forward_host", "zsaa_score_select", "zsaa_score_select_ex",
     "zsaa_op_linear", "zsaa_op_attention", "zsaa_op_colmass", "zsaa_sync", "zsaa_device_status",
     "zsaa_last_error", "zsaa_version", "zsaa_trace_begin", "zsaa_trace_end",
-    "zsaa_score_select_noalloc",
+    "zsaa_score_select_noalloc", "zsaa_model_set_graphs",
 ]
 
 
@@ -88,6 +88,7 @@ def lib():
             "zsaa_score_select": ([_P, _I, _I, _I, _I, _P, _P, _P], _I),
             "zsaa_score_select_ex": ([_P, _I, _I, _I, _I, _I, _I, _P, _P, _P, _P, _P], _I),
             "zsaa_score_select_noalloc": ([_P, _I, _I, _I, _I, _P, _P, _P], _I),
+            "zsaa_model_set_graphs": ([_P, _I], _I),
             "zsaa_op_linear": ([_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _I, _I, C.c_float, _P], _I),
             "zsaa_op_attention": ([_P, _I, _I, _I, _I, _I, _I, _P, _P, _P], _I),
             "zsaa_op_colmass": ([_P, _P, _I, _I, _I, _I, _I, _I, _P, _P], _I),
@@ -206,6 +207,10 @@ def zsaa_model_create(cfg: zsaa_config, weights: Dict, max_B: int, max_L: int) -
 
 def zsaa_model_destroy(model: Model):
     model.close()
+
+
+def zsaa_model_set_graphs(model: Model, enable: bool):
+    _check(lib().zsaa_model_set_graphs(model.handle, 1 if enable else 0))
 
 
 def zsaa_plan(model: Model, L: int, accel: float) -> Tuple[List[int], float]:
