@@ -9,6 +9,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "../../include/zsaa.h"
 
 namespace zsaa {
@@ -20,6 +22,38 @@ enum : int { kStatusTimeout = 1, kStatusBadIndex = 2 };
 
 // A bounded wait gives up after this many nanoseconds of %globaltimer.
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s
+
+// Programmatic dependent launch: every kernel of the library is launched with
+// launch_pdl, lets the next kernel in the stream start its prologue at once
+// (pdl_trigger), and waits for the previous kernel's results (pdl_wait)
+// before touching global data another kernel writes or reads.  Without the
+// launch attribute both are no-ops.
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+#define ZSAA_LAUNCH(...)                          \
+  do {                                            \
+    cudaError_t le_ = ::zsaa::launch_pdl(__VA_ARGS__); \
+    if (le_ != cudaSuccess) return le_;           \
+  } while (0)
 
 __device__ __forceinline__ unsigned long long globaltimer_ns() {
   unsigned long long t;

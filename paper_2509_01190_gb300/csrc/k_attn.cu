@@ -50,6 +50,8 @@ template <int HD>
 __global__ void __launch_bounds__(128)
     attn_fwd_bf16_kernel(const bf16* __restrict__ qkv, int N, int Hq, int Hkv,
                          bf16* __restrict__ out, float* __restrict__ lse2, float scale_log2) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int ROWB = HD * 2;
   constexpr int TILE = 64 * ROWB;
   extern __shared__ __align__(128) uint8_t sm[];
@@ -220,6 +222,8 @@ __global__ void __launch_bounds__(128)
     colmass_bf16_kernel(const bf16* __restrict__ qkv, const float* __restrict__ lse2, int N,
                         int Hq, int Hkv, int B, int q_per, int weight_vnorm,
                         float* __restrict__ parts, float scale_log2) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int ROWB = HD * 2;
   constexpr int TILE = 64 * ROWB;
   extern __shared__ __align__(128) uint8_t sm[];
@@ -352,6 +356,8 @@ __global__ void __launch_bounds__(128)
 // out[b][j]    = sum_qc sum_g parts[qc][b][g][j]                 (sum_groups = 1)
 __global__ void colmass_reduce_kernel(const float* __restrict__ parts, int n_qc, int B, int G,
                                       int N, int sum_groups, float* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   const int total = sum_groups ? B * N : B * G * N;
   if (idx >= total) return;
@@ -371,6 +377,8 @@ __global__ void colmass_reduce_kernel(const float* __restrict__ parts, int n_qc,
 __global__ void attn_fwd_f32_kernel(const float* __restrict__ qkv, int N, int Hq, int Hkv, int hd,
                                     float* __restrict__ out, float* __restrict__ lse2,
                                     float scale_log2) {
+  pdl_trigger();
+  pdl_wait();
   const int i = blockIdx.x * 4 + (threadIdx.x >> 5);
   const int h = blockIdx.y, b = blockIdx.z, lane = threadIdx.x & 31;
   if (i >= N) return;
@@ -424,6 +432,8 @@ __global__ void attn_fwd_f32_kernel(const float* __restrict__ qkv, int N, int Hq
 __global__ void colmass_f32_kernel(const float* __restrict__ qkv, const float* __restrict__ lse2,
                                    int N, int Hq, int Hkv, int hd, int B, int weight_vnorm,
                                    float* __restrict__ parts, float scale_log2) {
+  pdl_trigger();
+  pdl_wait();
   const int j = blockIdx.x * 4 + (threadIdx.x >> 5);
   const int g = blockIdx.y, b = blockIdx.z, lane = threadIdx.x & 31;
   if (j >= N) return;
@@ -463,7 +473,7 @@ cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, i
   const float scale_log2 = kLog2e / sqrtf(static_cast<float>(hd));
   if (dtype == ZSAA_F32) {
     dim3 grid((N + 3) / 4, Hq, B);
-    attn_fwd_f32_kernel<<<grid, 128, 0, s>>>(static_cast<const float*>(qkv), N, Hq, Hkv, hd,
+    ZSAA_LAUNCH(attn_fwd_f32_kernel, dim3(grid), dim3(128), 0, s, static_cast<const float*>(qkv), N, Hq, Hkv, hd,
                                              static_cast<float*>(out), lse, scale_log2);
     return cudaGetLastError();
   }
@@ -472,13 +482,13 @@ cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, i
     const int smem = 5 * 64 * 128;
     static cudaError_t e = set_smem(attn_fwd_bf16_kernel<64>, smem);
     if (e != cudaSuccess) return e;
-    attn_fwd_bf16_kernel<64><<<grid, 128, smem, s>>>(static_cast<const bf16*>(qkv), N, Hq, Hkv,
+    ZSAA_LAUNCH(attn_fwd_bf16_kernel<64>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), N, Hq, Hkv,
                                                       static_cast<bf16*>(out), lse, scale_log2);
   } else if (hd == 128) {
     const int smem = 5 * 64 * 256;
     static cudaError_t e = set_smem(attn_fwd_bf16_kernel<128>, smem);
     if (e != cudaSuccess) return e;
-    attn_fwd_bf16_kernel<128><<<grid, 128, smem, s>>>(static_cast<const bf16*>(qkv), N, Hq, Hkv,
+    ZSAA_LAUNCH(attn_fwd_bf16_kernel<128>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), N, Hq, Hkv,
                                                        static_cast<bf16*>(out), lse, scale_log2);
   } else {
     return cudaErrorInvalidValue;
@@ -503,7 +513,7 @@ cudaError_t colmass_parts(int dtype, const void* qkv, const float* lse, int B, i
   if (dtype == ZSAA_F32) {
     *n_qc = 1;
     dim3 grid((N + 3) / 4, Hkv, B);
-    colmass_f32_kernel<<<grid, 128, 0, s>>>(static_cast<const float*>(qkv), lse, N, Hq, Hkv, hd, B,
+    ZSAA_LAUNCH(colmass_f32_kernel, dim3(grid), dim3(128), 0, s, static_cast<const float*>(qkv), lse, N, Hq, Hkv, hd, B,
                                             weight_vnorm, parts, scale_log2);
     return cudaGetLastError();
   }
@@ -513,14 +523,14 @@ cudaError_t colmass_parts(int dtype, const void* qkv, const float* lse, int B, i
     const int smem = 3 * 64 * 128 + 2 * 64 * 4;
     static cudaError_t e = set_smem(colmass_bf16_kernel<64>, smem);
     if (e != cudaSuccess) return e;
-    colmass_bf16_kernel<64><<<grid, 128, smem, s>>>(static_cast<const bf16*>(qkv), lse, N, Hq,
+    ZSAA_LAUNCH(colmass_bf16_kernel<64>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), lse, N, Hq,
                                                      Hkv, B, kColmassQPer, weight_vnorm, parts,
                                                      scale_log2);
   } else if (hd == 128) {
     const int smem = 3 * 64 * 256 + 2 * 64 * 4;
     static cudaError_t e = set_smem(colmass_bf16_kernel<128>, smem);
     if (e != cudaSuccess) return e;
-    colmass_bf16_kernel<128><<<grid, 128, smem, s>>>(static_cast<const bf16*>(qkv), lse, N, Hq,
+    ZSAA_LAUNCH(colmass_bf16_kernel<128>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), lse, N, Hq,
                                                       Hkv, B, kColmassQPer, weight_vnorm, parts,
                                                       scale_log2);
   } else {
@@ -536,7 +546,7 @@ cudaError_t launch_colmass(int dtype, const void* qkv, const float* lse, int B, 
   cudaError_t e = colmass_parts(dtype, qkv, lse, B, N, Hq, Hkv, hd, 0, parts, &n_qc, s);
   if (e != cudaSuccess) return e;
   const int total = B * Hkv * N;
-  colmass_reduce_kernel<<<(total + 255) / 256, 256, 0, s>>>(parts, n_qc, B, Hkv, N, 0, C);
+  ZSAA_LAUNCH(colmass_reduce_kernel, dim3((total + 255) / 256), dim3(256), 0, s, parts, n_qc, B, Hkv, N, 0, C);
   return cudaGetLastError();
 }
 
@@ -548,7 +558,7 @@ cudaError_t launch_position_scores(int dtype, const void* qkv, const float* lse,
                                 mode == ZSAA_SCORE_SOFTSCORE_VNORM ? 1 : 0, parts, &n_qc, s);
   if (e != cudaSuccess) return e;
   const int total = B * N;
-  colmass_reduce_kernel<<<(total + 255) / 256, 256, 0, s>>>(parts, n_qc, B, Hkv, N, 1, scores);
+  ZSAA_LAUNCH(colmass_reduce_kernel, dim3((total + 255) / 256), dim3(256), 0, s, parts, n_qc, B, Hkv, N, 1, scores);
   return cudaGetLastError();
 }
 

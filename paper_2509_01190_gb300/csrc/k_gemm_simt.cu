@@ -14,6 +14,8 @@ __global__ void __launch_bounds__(256)
     gemm_f32_kernel(const float* __restrict__ A, int lda, const float* __restrict__ W,
                     const float* __restrict__ W2, int M, int N, int K, int epi,
                     float* __restrict__ out, int ldo, const float* resid) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float As[TK][TB + 4];
   __shared__ float Ws[TK][TB + 4];
   __shared__ float W2s[DUAL ? TK : 1][TB + 4];
@@ -76,11 +78,11 @@ cudaError_t launch_gemm_f32(const float* A, int lda, const float* W, const float
   if (p.launches) *p.launches += 1;
   dim3 grid((p.N + TB - 1) / TB, (p.M + TB - 1) / TB);
   if (epi == kEpiSwiGLU)
-    gemm_f32_kernel<true><<<grid, 256, 0, s>>>(A, lda, W, W2, p.M, p.N, p.K, epi,
+    ZSAA_LAUNCH(gemm_f32_kernel<true>, dim3(grid), dim3(256), 0, s, A, lda, W, W2, p.M, p.N, p.K, epi,
                                                static_cast<float*>(p.out), p.ldo,
                                                static_cast<const float*>(p.resid));
   else
-    gemm_f32_kernel<false><<<grid, 256, 0, s>>>(A, lda, W, nullptr, p.M, p.N, p.K, epi,
+    ZSAA_LAUNCH(gemm_f32_kernel<false>, dim3(grid), dim3(256), 0, s, A, lda, W, nullptr, p.M, p.N, p.K, epi,
                                                 static_cast<float*>(p.out), p.ldo,
                                                 static_cast<const float*>(p.resid));
   return cudaGetLastError();

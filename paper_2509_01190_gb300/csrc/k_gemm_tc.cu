@@ -1,9 +1,16 @@
 // bf16 GEMM on the sm_103a tensor cores: out = epi(A[M,K] W[N,K]^T), fp32
 // accumulation in tensor memory.
 //
-// Persistent kernel: one CTA per SM walks a static list of 128 x BN tiles
-// (tiles sharing a weight tile are adjacent, so weights stream from HBM once
-// and are re-read from L2).  Warp-specialised roles:
+// Persistent stream-K kernel: one CTA per SM.  Tiles are 128 x BN (tiles
+// sharing a weight tile are adjacent, so weights stream from HBM once and are
+// re-read from L2).  All but the last one-to-two waves of tiles are handed out
+// whole, round robin; the k-iterations of the remaining tiles are split evenly
+// over all CTAs, so no SM idles in a ragged last wave.  A tile split across
+// CTAs is finished by the CTA holding its first k-block (its last item): the
+// other contributors (for whom it is their first item) write fp32 partials
+// and raise a per-warp flag; the finisher waits (bounded) and adds them in CTA
+// order before the epilogue -- deterministic, no extra launch, no atomics.
+// Warp-specialised roles:
 //   warp 0      TMA producer: 128B-swizzled A and W tiles (64 deep in K) into a
 //               STAGES-deep shared-memory ring ("full" mbarriers, expect-tx);
 //   warp 1      MMA issuer: one thread issues tcgen05.mma (M=128, N=BN, K=16)
@@ -12,9 +19,6 @@
 //   warps 2..5  epilogue: tcgen05.ld of the finished accumulator (one row per
 //               thread), fused epilogue, 16-byte stores; then they hand the
 //               accumulator back, so the next tile's MMAs overlap this epilogue.
-// Small problems split K: each split writes an fp32 partial tile to a
-// workspace and splitk_finish_kernel sums the splits in a fixed order and
-// applies the epilogue (deterministic, no atomics).
 // Epilogues: bf16 store; residual add (h += acc, in place); SwiGLU (the tile's
 // first BN/2 accumulator columns are gate rows of W, the last BN/2 up rows of
 // W2; out = silu(gate) * up); float32 store (logits); RoPE of the query/key
@@ -48,12 +52,87 @@ struct TcMaps {
   CUtensorMap a, b0, b1, b2;
 };
 
-// Static tile list: tile t -> (m tile, n tile, K split), m fastest.
+// Work split: tiles [0, dp_tiles) go whole to CTA t % grid; the k-iterations
+// of tiles [dp_tiles, total) (sk_iters of them, num_kb per tile) are cut into
+// grid equal contiguous ranges.  Tile t -> (m tile t % m_tiles, n tile t / m_tiles).
 struct TileSched {
-  int m_tiles, n_tiles, splits, kb_per_split, num_kb, total;
-  float* ws;  // splits > 1: partial tiles [splits][M][VN] float32
-  int vn;     // columns of the (virtual) product: N, or 2N for SwiGLU
+  int m_tiles, n_tiles, num_kb, total, dp_tiles;
+  long long sk_iters;
+  float* ws;   // fp32 partial tiles, one BM x BN slot per CTA
+  int* flags;  // per CTA and epilogue warp: 1 while its partial is ready (reset by the reader)
 };
+
+// One unit of work of a CTA: k-blocks [kb0, kb1) of a tile.
+//   kind 0: the whole tile (epilogue directly);
+//   kind 1: a later part of a split tile (write the partial, raise the flags);
+//   kind 2: the first part of a split tile (add the partials of CTAs
+//           blockIdx.x+1 .. c_hi, then the epilogue).
+struct Item {
+  int tile, kb0, kb1, kind, c_hi;
+};
+
+struct WorkIter {
+  int t_dp;
+  long long it, end;
+  __device__ __forceinline__ void init(const TileSched& ts) {
+    t_dp = blockIdx.x;
+    const long long G = gridDim.x;
+    it = static_cast<long long>(blockIdx.x) * ts.sk_iters / G;
+    end = static_cast<long long>(blockIdx.x + 1) * ts.sk_iters / G;
+  }
+  __device__ __forceinline__ bool next(const TileSched& ts, Item& w) {
+    if (t_dp < ts.dp_tiles) {
+      w.tile = t_dp;
+      w.kb0 = 0;
+      w.kb1 = ts.num_kb;
+      w.kind = 0;
+      w.c_hi = 0;
+      t_dp += gridDim.x;
+      return true;
+    }
+    if (it >= end) return false;
+    const int KB = ts.num_kb;
+    const long long u = it / KB;
+    const int a = static_cast<int>(it - u * KB);
+    const int b = static_cast<int>(min(static_cast<long long>(KB), a + (end - it)));
+    w.tile = ts.dp_tiles + static_cast<int>(u);
+    w.kb0 = a;
+    w.kb1 = b;
+    w.c_hi = 0;
+    if (a == 0 && b == KB) {
+      w.kind = 0;
+    } else if (a == 0) {
+      // the CTA holding iteration x is floor(((x + 1) * grid - 1) / sk_iters)
+      w.kind = 2;
+      const long long G = gridDim.x;
+      w.c_hi = static_cast<int>(((u + 1) * KB * G - 1) / ts.sk_iters);
+    } else {
+      w.kind = 1;
+    }
+    it += b - a;
+    return true;
+  }
+};
+
+// Bounded wait until a flag written by another CTA reads 1.
+__device__ __forceinline__ bool wait_flag(const int* f, int* status, volatile int* abort) {
+  unsigned long long t0 = 0;
+  for (int n = 0;; ++n) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(f) : "memory");
+    if (v == 1) return true;
+    if ((n & 63) == 0) {
+      if (*abort) return false;
+      const unsigned long long t = globaltimer_ns();
+      if (t0 == 0) t0 = t;
+      else if (t - t0 > kWaitLimitNs) {
+        if (status) atomicOr(status, kStatusTimeout);
+        *abort = 1;
+        return false;
+      }
+    }
+  }
+}
 
 __device__ __forceinline__ float silu_f(float g) { return g / (1.f + __expf(-g)); }
 
@@ -66,31 +145,39 @@ __device__ __forceinline__ void store_bf16x16(bf16* dst, const float (&v)[16]) {
   d[1] = make_uint4(o[4], o[5], o[6], o[7]);
 }
 
-// Epilogue of one finished accumulator tile for this thread's row.
-template <int BN, int EPI>
-__device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_ok, int n0,
-                                              const GemmParams& p, const TileSched& ts, int ks) {
-  if (ts.splits > 1) {  // fp32 partial of this split, virtual column layout
-    float* ws = ts.ws + (static_cast<size_t>(ks) * p.M + row) * ts.vn + n0;
-#pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
-      uint32_t r[32];
-      __syncwarp();
-      tmem_ld16(tbase + c, *reinterpret_cast<uint32_t(*)[16]>(r));
-      tmem_ld16(tbase + c + 16, *reinterpret_cast<uint32_t(*)[16]>(r + 16));
-      tmem_ld_wait();
+// Sum of the partial tiles of CTAs c0..c1 (inclusive; none if c0 > c1) at
+// this thread's row, tile columns [col, col + 16), added to v.  Partials are
+// stored column-major ([BN][BM] per CTA slot) so a warp's loads are coalesced;
+// up to four contributors' loads are in flight together, then added in order.
+template <int BN>
+__device__ __forceinline__ void add_partials(float (&v)[16], const float* ws, int c0, int c1,
+                                             int rit, int col) {
+  for (int c = c0; c <= c1; c += 4) {
+    float t[4][16];
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        if (row_ok && n0 + c + 16 * h < ts.vn) {
-          uint4* dst = reinterpret_cast<uint4*>(ws + c + 16 * h);
+    for (int k = 0; k < 4; ++k) {
+      if (c + k <= c1) {
+        const float* q = ws + static_cast<size_t>(c + k) * BM * BN + static_cast<size_t>(col) * BM + rit;
 #pragma unroll
-          for (int q = 0; q < 4; ++q)
-            dst[q] = make_uint4(r[16 * h + 4 * q], r[16 * h + 4 * q + 1], r[16 * h + 4 * q + 2], r[16 * h + 4 * q + 3]);
-        }
+        for (int e = 0; e < 16; ++e) t[k][e] = __ldcg(q + e * BM);
       }
     }
-    return;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      if (c + k <= c1) {
+#pragma unroll
+        for (int e = 0; e < 16; ++e) v[e] += t[k][e];
+      }
+    }
   }
+}
+
+// Epilogue of one finished accumulator tile for this thread's row; the
+// partials of CTAs c0..c1 (if any) are added to the accumulator first.
+template <int BN, int EPI>
+__device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_ok, int n0,
+                                              const GemmParams& p, const float* ws, int c0, int c1,
+                                              int rit) {
   if (EPI == kEpiSwiGLU) {
     bf16* out = static_cast<bf16*>(p.out);
     const int oc0 = n0 / 2;
@@ -102,9 +189,16 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
       tmem_ld16(tbase + BN / 2 + c, u);
       tmem_ld_wait();
       if (row_ok && oc0 + c < p.N) {
-        float v[16];
+        float gv[16], uv[16], v[16];
 #pragma unroll
-        for (int e = 0; e < 16; ++e) v[e] = silu_f(__uint_as_float(g[e])) * __uint_as_float(u[e]);
+        for (int e = 0; e < 16; ++e) {
+          gv[e] = __uint_as_float(g[e]);
+          uv[e] = __uint_as_float(u[e]);
+        }
+        add_partials<BN>(gv, ws, c0, c1, rit, c);
+        add_partials<BN>(uv, ws, c0, c1, rit, BN / 2 + c);
+#pragma unroll
+        for (int e = 0; e < 16; ++e) v[e] = silu_f(gv[e]) * uv[e];
         store_bf16x16(out + static_cast<size_t>(row) * p.ldo + oc0 + c, v);
       }
     }
@@ -120,10 +214,13 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
         if (row_ok && n0 + c + 16 * h < p.N) {
-          uint4* dst = reinterpret_cast<uint4*>(out + static_cast<size_t>(row) * p.ldo + n0 + c + 16 * h);
+          float v[16];
 #pragma unroll
-          for (int q = 0; q < 4; ++q)
-            dst[q] = make_uint4(r[16 * h + 4 * q], r[16 * h + 4 * q + 1], r[16 * h + 4 * q + 2], r[16 * h + 4 * q + 3]);
+          for (int e = 0; e < 16; ++e) v[e] = __uint_as_float(r[16 * h + e]);
+          add_partials<BN>(v, ws, c0, c1, rit, c + 16 * h);
+          float4* dst = reinterpret_cast<float4*>(out + static_cast<size_t>(row) * p.ldo + n0 + c + 16 * h);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
         }
       }
     }
@@ -152,7 +249,14 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
         tmem_ld16(tbase + hs + half + c, x2);
         tmem_ld_wait();
         if (row_ok && n0 + hs < p.N) {
-          float y1[16], y2[16];
+          float a1[16], a2[16], y1[16], y2[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            a1[e] = __uint_as_float(x1[e]);
+            a2[e] = __uint_as_float(x2[e]);
+          }
+          add_partials<BN>(a1, ws, c0, c1, rit, hs + c);
+          add_partials<BN>(a2, ws, c0, c1, rit, hs + half + c);
           if (rot) {
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -160,7 +264,7 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
               const float cv[4] = {cs.x, cs.y, cs.z, cs.w}, sv[4] = {sn.x, sn.y, sn.z, sn.w};
 #pragma unroll
               for (int e = 0; e < 4; ++e) {
-                const float a = __uint_as_float(x1[4 * q + e]), b = __uint_as_float(x2[4 * q + e]);
+                const float a = a1[4 * q + e], b = a2[4 * q + e];
                 y1[4 * q + e] = a * cv[e] - b * sv[e];
                 y2[4 * q + e] = b * cv[e] + a * sv[e];
               }
@@ -168,8 +272,8 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
           } else {
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
-              y1[e] = __uint_as_float(x1[e]);
-              y2[e] = __uint_as_float(x2[e]);
+              y1[e] = a1[e];
+              y2[e] = a2[e];
             }
           }
           bf16* rowp = out + static_cast<size_t>(row) * p.ldo + n0 + hs;
@@ -210,6 +314,7 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
           float v[16];
 #pragma unroll
           for (int e = 0; e < 16; ++e) v[e] = __uint_as_float(r[16 * h + e]);
+          add_partials<BN>(v, ws, c0, c1, rit, c + 16 * h);
           if (EPI == kEpiResid) {
             const uint32_t rr[8] = {rc[2 * h].x, rc[2 * h].y, rc[2 * h].z, rc[2 * h].w,
                                     rc[2 * h + 1].x, rc[2 * h + 1].y, rc[2 * h + 1].z, rc[2 * h + 1].w};
@@ -225,6 +330,22 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
 #pragma unroll
       for (int q = 0; q < 4; ++q) rc[q] = rn[q];
     }
+  }
+}
+
+// Write this thread's row of the accumulator tile into the CTA's partial slot
+// (column-major: element (row, col) at slot[col * BM + row]).
+template <int BN>
+__device__ __forceinline__ void write_partial(uint32_t tbase, float* slot, int rit) {
+#pragma unroll 1
+  for (int c = 0; c < BN; c += 32) {
+    uint32_t r[32];
+    __syncwarp();
+    tmem_ld16(tbase + c, *reinterpret_cast<uint32_t(*)[16]>(r));
+    tmem_ld16(tbase + c + 16, *reinterpret_cast<uint32_t(*)[16]>(r + 16));
+    tmem_ld_wait();
+#pragma unroll
+    for (int e = 0; e < 32; ++e) __stcg(slot + static_cast<size_t>(c + e) * BM + rit, __uint_as_float(r[e]));
   }
 }
 
@@ -246,6 +367,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  pdl_trigger();
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
@@ -275,12 +397,36 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       uint32_t it = 0, issued_last = 0;
       bool ok = true;
-      for (int t = blockIdx.x; t < ts.total && ok; t += gridDim.x) {
-        const int mt = t % ts.m_tiles, r = t / ts.m_tiles;
-        const int nt = r % ts.n_tiles, ks = r / ts.n_tiles;
+      WorkIter wi;
+      wi.init(ts);
+      // The weights are never written by another kernel: start streaming the
+      // first stages' weight tiles before waiting for the previous kernel.
+      int npre = 0;
+      {
+        WorkIter peek = wi;
+        Item w0;
+        if (peek.next(ts, w0)) {
+          const int n0 = (w0.tile / ts.m_tiles) * BN;
+          npre = min(C::STAGES, w0.kb1 - w0.kb0);
+          for (int j = 0; j < npre; ++j) {
+            const int kb = w0.kb0 + j;
+            mbar_arrive_expect_tx(&full[j], C::STAGE_BYTES);
+            if (EPI == kEpiSwiGLU) {
+              tma_load_2d(sB + j * C::B_BYTES, &maps.b0, kb * BK, n0 / 2, &full[j]);
+              tma_load_2d(sB + j * C::B_BYTES + (BN / 2) * 128, &maps.b1, kb * BK, n0 / 2, &full[j]);
+            } else {
+              const CUtensorMap* mb = n0 >= n2 ? &maps.b2 : (n0 >= n1 ? &maps.b1 : &maps.b0);
+              const int nb = n0 >= n2 ? n0 - n2 : (n0 >= n1 ? n0 - n1 : n0);
+              tma_load_2d(sB + j * C::B_BYTES, mb, kb * BK, nb, &full[j]);
+            }
+          }
+        }
+      }
+      pdl_wait();
+      Item w;
+      while (ok && wi.next(ts, w)) {
+        const int mt = w.tile % ts.m_tiles, nt = w.tile / ts.m_tiles;
         const int m0 = mt * BM, n0 = nt * BN;
-        const int kb0 = ks * ts.kb_per_split;
-        const int kb1 = min(ts.num_kb, kb0 + ts.kb_per_split);
         const CUtensorMap* mb = &maps.b0;
         int nb = n0;
         if (EPI != kEpiSwiGLU) {
@@ -292,21 +438,23 @@ __global__ void __launch_bounds__(kThreads, 1)
             nb = n0 - n1;
           }
         }
-        for (int kb = kb0; kb < kb1; ++kb, ++it) {
+        for (int kb = w.kb0; kb < w.kb1; ++kb, ++it) {
           const int s = it % C::STAGES;
           const uint32_t ph = (it / C::STAGES) & 1;
-          if (!mbar_wait_ab(&empty[s], ph ^ 1, p.status, abort_flag)) {
-            ok = false;
-            break;
+          if (static_cast<int>(it) >= npre) {  // the first npre stages' weights are in flight already
+            if (!mbar_wait_ab(&empty[s], ph ^ 1, p.status, abort_flag)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
+            if (EPI == kEpiSwiGLU) {
+              tma_load_2d(sB + s * C::B_BYTES, &maps.b0, kb * BK, n0 / 2, &full[s]);
+              tma_load_2d(sB + s * C::B_BYTES + (BN / 2) * 128, &maps.b1, kb * BK, n0 / 2, &full[s]);
+            } else {
+              tma_load_2d(sB + s * C::B_BYTES, mb, kb * BK, nb, &full[s]);
+            }
           }
-          mbar_arrive_expect_tx(&full[s], C::STAGE_BYTES);
           tma_load_2d(sA + s * C::A_BYTES, &maps.a, kb * BK, m0, &full[s]);
-          if (EPI == kEpiSwiGLU) {
-            tma_load_2d(sB + s * C::B_BYTES, &maps.b0, kb * BK, n0 / 2, &full[s]);
-            tma_load_2d(sB + s * C::B_BYTES + (BN / 2) * 128, &maps.b1, kb * BK, n0 / 2, &full[s]);
-          } else {
-            tma_load_2d(sB + s * C::B_BYTES, mb, kb * BK, nb, &full[s]);
-          }
           issued_last = it + 1;
         }
       }
@@ -325,17 +473,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t it = 0;
       bool ok = true;
       int i = 0;
-      for (int t = blockIdx.x; t < ts.total && ok; t += gridDim.x, ++i) {
-        const int r = t / ts.m_tiles;
-        const int ks = r / ts.n_tiles;
-        const int kb0 = ks * ts.kb_per_split;
-        const int kb1 = min(ts.num_kb, kb0 + ts.kb_per_split);
+      WorkIter wi;
+      wi.init(ts);
+      Item w;
+      while (ok && wi.next(ts, w)) {
         const int ab = i & 1;
         const uint32_t use = static_cast<uint32_t>(i >> 1);
+        ++i;
         if (!mbar_wait_ab(&acc_empty[ab], (use & 1) ^ 1, p.status, abort_flag)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem + static_cast<uint32_t>(ab * BN);
-        for (int kb = kb0; kb < kb1; ++kb, ++it) {
+        for (int kb = w.kb0; kb < w.kb1; ++kb, ++it) {
           const int s = it % C::STAGES;
           const uint32_t ph = (it / C::STAGES) & 1;
           if (!mbar_wait_ab(&full[s], ph, p.status, abort_flag)) {
@@ -348,7 +496,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
             tc_mma_bf16(d_tmem, sdesc_sw128(a_base + k * 32), sdesc_sw128(b_base + k * 32), idesc,
-                        (kb > kb0 || k > 0) ? 1u : 0u);
+                        (kb > w.kb0 || k > 0) ? 1u : 0u);
           tc_commit(&empty[s]);
         }
         tc_commit(&acc_full[ab]);
@@ -357,19 +505,49 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else {
     // Epilogue: warp w reads TMEM lanes 32*(w%4) .. +32, i.e. tile rows.
+    pdl_wait();
     const int quad = warp & 3;
+    const int rit = quad * 32 + lane;  // row within the tile
     int i = 0;
-    for (int t = blockIdx.x; t < ts.total; t += gridDim.x, ++i) {
-      const int mt = t % ts.m_tiles, r = t / ts.m_tiles;
-      const int nt = r % ts.n_tiles, ks = r / ts.n_tiles;
-      const int row = mt * BM + quad * 32 + lane;
+    WorkIter wi;
+    wi.init(ts);
+    Item w;
+    while (wi.next(ts, w)) {
+      const int mt = w.tile % ts.m_tiles, nt = w.tile / ts.m_tiles;
+      const int row = mt * BM + rit;
       const int ab = i & 1;
       const uint32_t use = static_cast<uint32_t>(i >> 1);
+      ++i;
       const bool ok = __all_sync(0xffffffffu, mbar_wait_ab(&acc_full[ab], use & 1, p.status, abort_flag));
       if (!ok) break;
       tc_fence_after();
       const uint32_t tbase = tmem + static_cast<uint32_t>(ab * BN) + (static_cast<uint32_t>(quad * 32) << 16);
-      tile_epilogue<BN, EPI>(tbase, row, row < p.M, nt * BN, p, ts, ks);
+      if (w.kind == 1) {
+        // a later part of a split tile: hand the partial to the tile's first CTA
+        write_partial<BN>(tbase, ts.ws + static_cast<size_t>(blockIdx.x) * BM * BN, rit);
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) {
+          int* f = ts.flags + blockIdx.x * 4 + quad;
+          asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(f), "r"(1) : "memory");
+        }
+      } else {
+        int c0 = 1, c1 = 0;  // no partials
+        if (w.kind == 2) {
+          c0 = blockIdx.x + 1;
+          c1 = w.c_hi;
+          bool got = true;
+          for (int c = c0; c <= c1; ++c)
+            got = got && wait_flag(ts.flags + c * 4 + quad, p.status, abort_flag);
+          if (!__all_sync(0xffffffffu, got)) c1 = c0 - 1;  // gave up: status already set
+        }
+        tile_epilogue<BN, EPI>(tbase, row, row < p.M, nt * BN, p, ts.ws, c0, c1, rit);
+        if (w.kind == 2) {
+          __syncwarp();
+          if (lane == 0)
+            for (int c = c0; c <= c1; ++c) ts.flags[c * 4 + quad] = 0;
+        }
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&acc_empty[ab])) : "memory");
@@ -380,90 +558,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);
-  }
-}
-
-// Sum the K splits in order and apply the epilogue.  One thread per 8 output
-// columns of one row (RoPE: per 8 rotation pairs of one head).
-template <int EPI>
-__global__ void splitk_finish_kernel(const float* __restrict__ ws, int splits, int BN,
-                                     const GemmParams p, int vn) {
-  const int row = blockIdx.y;
-  const int ncols = EPI == kEpiRope ? p.rope_cols / 2 + (p.N - p.rope_cols) : p.N;
-  const int chunk = blockIdx.x * blockDim.x + threadIdx.x;
-  if (row >= p.M || chunk * 8 >= ncols) return;
-  const size_t plane = static_cast<size_t>(p.M) * vn;
-  const float* base = ws + static_cast<size_t>(row) * vn;
-  auto sum8 = [&](int col, float (&v)[8]) {
-#pragma unroll
-    for (int e = 0; e < 8; ++e) v[e] = 0.f;
-    for (int s = 0; s < splits; ++s) {
-      const float4* q = reinterpret_cast<const float4*>(base + s * plane + col);
-      const float4 a = q[0], b = q[1];
-      v[0] += a.x; v[1] += a.y; v[2] += a.z; v[3] += a.w;
-      v[4] += b.x; v[5] += b.y; v[6] += b.z; v[7] += b.w;
-    }
-  };
-  auto put_bf16 = [&](bf16* dst, const float (&v)[8]) {
-    *reinterpret_cast<uint4*>(dst) = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
-                                                pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
-  };
-  if (EPI == kEpiSwiGLU) {
-    const int c = chunk * 8, half = BN / 2;
-    const int vcol = (c / half) * BN + c % half;
-    float g[8], u[8], v[8];
-    sum8(vcol, g);
-    sum8(vcol + half, u);
-#pragma unroll
-    for (int e = 0; e < 8; ++e) v[e] = silu_f(g[e]) * u[e];
-    put_bf16(static_cast<bf16*>(p.out) + static_cast<size_t>(row) * p.ldo + c, v);
-  } else if (EPI == kEpiRope) {
-    const int pairs = p.rope_cols / 2;
-    const int half = p.hd / 2;
-    bf16* out = static_cast<bf16*>(p.out) + static_cast<size_t>(row) * p.ldo;
-    if (chunk * 8 < pairs) {
-      const int pr = chunk * 8, head = pr / half, c = pr % half;
-      const int col1 = head * p.hd + c, col2 = col1 + half;
-      float x1[8], x2[8], y1[8], y2[8];
-      sum8(col1, x1);
-      sum8(col2, x2);
-      const int ps = p.pos[row];
-#pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        const float cs = p.cos_t[static_cast<size_t>(ps) * half + c + e];
-        const float sn = p.sin_t[static_cast<size_t>(ps) * half + c + e];
-        y1[e] = x1[e] * cs - x2[e] * sn;
-        y2[e] = x2[e] * cs + x1[e] * sn;
-      }
-      put_bf16(out + col1, y1);
-      put_bf16(out + col2, y2);
-    } else {
-      const int col = p.rope_cols + (chunk * 8 - pairs);
-      float v[8];
-      sum8(col, v);
-      put_bf16(out + col, v);
-    }
-  } else {
-    const int c = chunk * 8;
-    float v[8];
-    sum8(c, v);
-    const size_t off = static_cast<size_t>(row) * p.ldo + c;
-    if (EPI == kEpiStoreF32) {
-      float4* d = reinterpret_cast<float4*>(static_cast<float*>(p.out) + off);
-      d[0] = make_float4(v[0], v[1], v[2], v[3]);
-      d[1] = make_float4(v[4], v[5], v[6], v[7]);
-    } else {
-      if (EPI == kEpiResid) {
-        const uint4 r = *reinterpret_cast<const uint4*>(static_cast<const bf16*>(p.resid) + off);
-        const uint32_t rr[4] = {r.x, r.y, r.z, r.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          v[2 * e] += bf16lo(rr[e]);
-          v[2 * e + 1] += bf16hi(rr[e]);
-        }
-      }
-      put_bf16(static_cast<bf16*>(p.out) + off, v);
-    }
   }
 }
 
@@ -495,7 +589,7 @@ int num_sms() {
 
 template <int BN, int EPI>
 cudaError_t run_tc(const TcMaps& maps, int n1, int n2, const GemmParams& p, const TileSched& ts,
-                   cudaStream_t s) {
+                   int grid, cudaStream_t s) {
   using C = TcCfg<BN>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
@@ -505,28 +599,20 @@ cudaError_t run_tc(const TcMaps& maps, int n1, int n2, const GemmParams& p, cons
                                     static_cast<int>(C::SMEM));
   });
   if (attr_err != cudaSuccess) return attr_err;
-  const int grid = ts.total < num_sms() ? ts.total : num_sms();
-  gemm_tc_kernel<BN, EPI><<<grid, kThreads, C::SMEM, s>>>(maps, n1, n2, p, ts);
-  cudaError_t e = cudaGetLastError();
+  ZSAA_LAUNCH(gemm_tc_kernel<BN, EPI>, dim3(grid), dim3(kThreads), C::SMEM, s, maps, n1, n2, p, ts);
   if (p.launches) *p.launches += 1;
-  if (e != cudaSuccess || ts.splits == 1) return e;
-  if (p.launches) *p.launches += 1;
-  const int ncols = EPI == kEpiRope ? p.rope_cols / 2 + (p.N - p.rope_cols) : p.N;
-  const int chunks = (ncols + 7) / 8;
-  dim3 fgrid((chunks + 127) / 128, p.M);
-  splitk_finish_kernel<EPI><<<fgrid, 128, 0, s>>>(ts.ws, ts.splits, BN, p, ts.vn);
   return cudaGetLastError();
 }
 
 template <int BN>
 cudaError_t dispatch_epi(int epi, const TcMaps& maps, int n1, int n2, const GemmParams& p,
-                         const TileSched& ts, cudaStream_t s) {
+                         const TileSched& ts, int grid, cudaStream_t s) {
   switch (epi) {
-    case kEpiStore: return run_tc<BN, kEpiStore>(maps, n1, n2, p, ts, s);
-    case kEpiResid: return run_tc<BN, kEpiResid>(maps, n1, n2, p, ts, s);
-    case kEpiSwiGLU: return run_tc<BN, kEpiSwiGLU>(maps, n1, n2, p, ts, s);
-    case kEpiStoreF32: return run_tc<BN, kEpiStoreF32>(maps, n1, n2, p, ts, s);
-    case kEpiRope: return run_tc<BN, kEpiRope>(maps, n1, n2, p, ts, s);
+    case kEpiStore: return run_tc<BN, kEpiStore>(maps, n1, n2, p, ts, grid, s);
+    case kEpiResid: return run_tc<BN, kEpiResid>(maps, n1, n2, p, ts, grid, s);
+    case kEpiSwiGLU: return run_tc<BN, kEpiSwiGLU>(maps, n1, n2, p, ts, grid, s);
+    case kEpiStoreF32: return run_tc<BN, kEpiStoreF32>(maps, n1, n2, p, ts, grid, s);
+    case kEpiRope: return run_tc<BN, kEpiRope>(maps, n1, n2, p, ts, grid, s);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -547,32 +633,49 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
   const int sms = num_sms();
   const int vn = epi == kEpiSwiGLU ? 2 * p.N : p.N;
   const int m_tiles = (p.M + BM - 1) / BM;
-  // Widest tile that still gives a full wave; otherwise the narrowest legal one.
+  // Tile width by problem size, from sweeps of the pruned-prefill shapes on
+  // GB300 (graph-timed): narrow tiles only while M is small enough that wide
+  // ones leave most SMs idle; the SwiGLU GEMM (2x the columns) always wide.
+  // (also wide whenever there are two waves of wide tiles: the LM head's
+  // 128256 columns would otherwise re-read the activation thousands of times)
+  const long wide_tiles = static_cast<long>(m_tiles) * ((vn + 255) / 256);
+  const int want = (epi == kEpiSwiGLU || wide_tiles >= 2L * sms)
+                       ? 256
+                       : (p.M <= 256 ? 64 : (p.M <= 768 ? 128 : 256));
   int BN = 0;
-  for (int cand : {256, 128, 64}) {
-    if (!bn_ok(cand, epi, W, p)) continue;
-    BN = cand;
-    if (static_cast<long>(m_tiles) * ((vn + cand - 1) / cand) >= sms) break;
-  }
+  for (int cand : {64, 128, 256})
+    if (bn_ok(cand, epi, W, p) && (BN == 0 || cand <= want)) BN = cand;
   if (BN == 0) return cudaErrorInvalidValue;
   TileSched ts{};
   ts.m_tiles = m_tiles;
   ts.n_tiles = (vn + BN - 1) / BN;
   ts.num_kb = p.K / BK;
-  ts.vn = vn;
-  ts.splits = 1;
-  const long tiles = static_cast<long>(ts.m_tiles) * ts.n_tiles;
-  // Split K while the tiles fill less than one wave and each split keeps >= 4 k-blocks.
-  if (p.splitk_ws != nullptr) {
-    while (tiles * ts.splits < sms && ts.num_kb / (2 * ts.splits) >= 4 &&
-           static_cast<size_t>(2 * ts.splits) * p.M * vn <= p.splitk_ws_elems)
-      ts.splits *= 2;
-  }
-  ts.kb_per_split = (ts.num_kb + ts.splits - 1) / ts.splits;
-  ts.splits = (ts.num_kb + ts.kb_per_split - 1) / ts.kb_per_split;
-  ts.total = static_cast<int>(tiles * ts.splits);
+  ts.total = ts.m_tiles * ts.n_tiles;
   ts.ws = p.splitk_ws;
-
+  ts.flags = p.splitk_flags;
+  int grid;
+  // Whole tiles unless K is deep (>= 64 k-blocks, the MLP down projection) and
+  // the last wave of whole tiles would leave over a quarter of the SM-time
+  // idle; then stream-K over the last one-to-two waves (or over everything,
+  // for problems smaller than a wave).  Measured: stream-K loses to whole tiles
+  // at K = 2048 (the partial hand-off costs more than the tail it removes).
+  const int waves = (ts.total + sms - 1) / sms;
+  const double idle = 1.0 - static_cast<double>(ts.total) / (static_cast<double>(waves) * sms);
+  const bool can_split = p.splitk_ws != nullptr && p.splitk_flags != nullptr && sms <= kMaxGemmCtas &&
+                         static_cast<size_t>(sms) * BM * BN <= p.splitk_ws_elems;
+  if (!can_split || idle <= 0.25 || ts.num_kb < 64) {
+    ts.dp_tiles = ts.total;
+    ts.sk_iters = 0;
+    grid = ts.total < sms ? ts.total : sms;
+  } else {
+    ts.dp_tiles = ts.total >= 2 * sms ? (ts.total / sms - 1) * sms : 0;
+    ts.sk_iters = static_cast<long long>(ts.total - ts.dp_tiles) * ts.num_kb;
+    grid = sms;
+    if (ts.dp_tiles == 0) {  // small problem: keep at least 8 k-blocks per CTA
+      const long long g = ts.sk_iters / 8;
+      grid = static_cast<int>(g < 1 ? 1 : (g < sms ? g : sms));
+    }
+  }
   TcMaps maps;
   memset(&maps, 0, sizeof(maps));
   const uint32_t brows = epi == kEpiSwiGLU ? BN / 2 : BN;
@@ -596,9 +699,9 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
     }
   }
   switch (BN) {
-    case 256: return dispatch_epi<256>(epi, maps, n1, n2, p, ts, s);
-    case 128: return dispatch_epi<128>(epi, maps, n1, n2, p, ts, s);
-    default: return dispatch_epi<64>(epi, maps, n1, n2, p, ts, s);
+    case 256: return dispatch_epi<256>(epi, maps, n1, n2, p, ts, grid, s);
+    case 128: return dispatch_epi<128>(epi, maps, n1, n2, p, ts, grid, s);
+    default: return dispatch_epi<64>(epi, maps, n1, n2, p, ts, grid, s);
   }
 }
 

@@ -20,6 +20,8 @@ inline int row_blocks(int rows) { return (rows + kWarpsPerBlock - 1) / kWarpsPer
 __global__ void embed_kernel(const uint4* __restrict__ E, const int32_t* __restrict__ tok, int rows,
                              int L, int vocab, int vec_per_row, uint4* __restrict__ h,
                              int32_t* __restrict__ pos, int* status) {
+  pdl_trigger();
+  pdl_wait();
   const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= rows) return;
@@ -39,6 +41,8 @@ __global__ void embed_kernel(const uint4* __restrict__ E, const int32_t* __restr
 template <typename T>
 __global__ void rmsnorm_kernel(const T* __restrict__ h, const T* __restrict__ w, int rows, int d,
                                float eps, T* __restrict__ x) {
+  pdl_trigger();
+  pdl_wait();
   const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= rows) return;
@@ -58,6 +62,8 @@ __global__ void rmsnorm_kernel(const T* __restrict__ h, const T* __restrict__ w,
 __global__ void rmsnorm_bf16_vec_kernel(const uint4* __restrict__ h, const uint4* __restrict__ w,
                                         int rows, int vec_per_row, float eps,
                                         uint4* __restrict__ x) {
+  pdl_trigger();
+  pdl_wait();
   const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= rows) return;
@@ -93,6 +99,8 @@ __global__ void rmsnorm_bf16_vec_kernel(const uint4* __restrict__ h, const uint4
 template <int UNROLL>
 __global__ void row_norm_bf16_kernel(const uint4* __restrict__ h, int rows, int vec_per_row,
                                      float* __restrict__ s) {
+  pdl_trigger();
+  pdl_wait();
   const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= rows) return;
@@ -130,6 +138,8 @@ __global__ void row_norm_bf16_kernel(const uint4* __restrict__ h, int rows, int 
 
 __global__ void row_norm_f32_kernel(const float* __restrict__ h, int rows, int d,
                                     float* __restrict__ s) {
+  pdl_trigger();
+  pdl_wait();
   const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= rows) return;
@@ -161,6 +171,8 @@ constexpr int kSelThreads = 1024;
 __global__ void __launch_bounds__(kSelThreads)
     select_topk_kernel(const float* __restrict__ scores, int N, int k, int force_last,
                        int32_t* __restrict__ idx_out) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int nwarps = kSelThreads / 32;
@@ -269,6 +281,8 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ src, int N, int k, 
                                    const int32_t* __restrict__ idx, uint4* __restrict__ dst,
                                    const int32_t* __restrict__ pos_in, int32_t* __restrict__ pos_out,
                                    int total, int* status) {
+  pdl_trigger();
+  pdl_wait();
   const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= total) return;
@@ -299,6 +313,8 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ src, int N, int k, 
 __global__ void rope_f32_kernel(float* __restrict__ qkv, int rows, int ld, int rope_cols, int hd,
                                 const int32_t* __restrict__ pos, const float* __restrict__ cos_t,
                                 const float* __restrict__ sin_t) {
+  pdl_trigger();
+  pdl_wait();
   const int r = blockIdx.y;
   const int half = hd / 2;
   const int pairs = rope_cols / 2;
@@ -321,6 +337,8 @@ template <typename T>
 __global__ void cls_head_kernel(const T* __restrict__ h, int N, int d,
                                 const T* __restrict__ norm_w, float eps, const T* __restrict__ W,
                                 int n_classes, float* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
   extern __shared__ float xs[];  // d floats
   __shared__ float red[32];
   const int b = blockIdx.x;
@@ -359,7 +377,7 @@ cudaError_t launch_embed(int dtype, const void* E, const int32_t* tok, int rows,
                          int d, void* h, int32_t* pos, int* status, cudaStream_t s) {
   const int esz = dtype == ZSAA_BF16 ? 2 : 4;
   const int vec = d * esz / 16;
-  embed_kernel<<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
+  ZSAA_LAUNCH(embed_kernel, dim3(row_blocks(rows)), dim3(32 * kWarpsPerBlock), 0, s, 
       static_cast<const uint4*>(E), tok, rows, L, vocab, vec, static_cast<uint4*>(h), pos, status);
   return cudaGetLastError();
 }
@@ -367,15 +385,15 @@ cudaError_t launch_embed(int dtype, const void* E, const int32_t* tok, int rows,
 cudaError_t launch_rmsnorm(int dtype, const void* h, const void* w, int rows, int d, float eps,
                            void* x, cudaStream_t s) {
   if (dtype == ZSAA_BF16 && d % 8 == 0) {
-    rmsnorm_bf16_vec_kernel<<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
+    ZSAA_LAUNCH(rmsnorm_bf16_vec_kernel, dim3(row_blocks(rows)), dim3(32 * kWarpsPerBlock), 0, s, 
         static_cast<const uint4*>(h), static_cast<const uint4*>(w), rows, d / 8, eps,
         static_cast<uint4*>(x));
   } else if (dtype == ZSAA_BF16) {
-    rmsnorm_kernel<bf16><<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
+    ZSAA_LAUNCH(rmsnorm_kernel<bf16>, dim3(row_blocks(rows)), dim3(32 * kWarpsPerBlock), 0, s, 
         static_cast<const bf16*>(h), static_cast<const bf16*>(w), rows, d, eps,
         static_cast<bf16*>(x));
   } else {
-    rmsnorm_kernel<float><<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
+    ZSAA_LAUNCH(rmsnorm_kernel<float>, dim3(row_blocks(rows)), dim3(32 * kWarpsPerBlock), 0, s, 
         static_cast<const float*>(h), static_cast<const float*>(w), rows, d, eps,
         static_cast<float*>(x));
   }
@@ -385,10 +403,10 @@ cudaError_t launch_rmsnorm(int dtype, const void* h, const void* w, int rows, in
 cudaError_t launch_row_norm(int dtype, const void* h, int rows, int d, float* scores,
                             cudaStream_t s) {
   if (dtype == ZSAA_BF16) {
-    row_norm_bf16_kernel<8><<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
+    ZSAA_LAUNCH(row_norm_bf16_kernel<8>, dim3(row_blocks(rows)), dim3(32 * kWarpsPerBlock), 0, s, 
         static_cast<const uint4*>(h), rows, d / 8, scores);
   } else {
-    row_norm_f32_kernel<<<row_blocks(rows), 32 * kWarpsPerBlock, 0, s>>>(
+    ZSAA_LAUNCH(row_norm_f32_kernel, dim3(row_blocks(rows)), dim3(32 * kWarpsPerBlock), 0, s, 
         static_cast<const float*>(h), rows, d, scores);
   }
   return cudaGetLastError();
@@ -396,7 +414,7 @@ cudaError_t launch_row_norm(int dtype, const void* h, int rows, int d, float* sc
 
 cudaError_t launch_select(const float* scores, int B, int N, int k, int force_last, int32_t* idx,
                           cudaStream_t s) {
-  select_topk_kernel<<<B, kSelThreads, 0, s>>>(scores, N, k, force_last, idx);
+  ZSAA_LAUNCH(select_topk_kernel, dim3(B), dim3(kSelThreads), 0, s, scores, N, k, force_last, idx);
   return cudaGetLastError();
 }
 
@@ -404,7 +422,7 @@ cudaError_t launch_gather(const void* src, int B, int N, int k, int row_bytes, c
                           void* dst, const int32_t* pos_in, int32_t* pos_out, int* status,
                           cudaStream_t s) {
   const int total = B * k;
-  gather_rows_kernel<4><<<row_blocks(total), 32 * kWarpsPerBlock, 0, s>>>(
+  ZSAA_LAUNCH(gather_rows_kernel<4>, dim3(row_blocks(total)), dim3(32 * kWarpsPerBlock), 0, s, 
       static_cast<const uint4*>(src), N, k, row_bytes / 16, idx, static_cast<uint4*>(dst),
       pos_in, pos_out, total, status);
   return cudaGetLastError();
@@ -415,7 +433,7 @@ cudaError_t launch_rope_f32(float* qkv, int rows, int ld, int rope_cols, int hd,
                             cudaStream_t s) {
   const int pairs = rope_cols / 2;
   dim3 grid((pairs + 127) / 128, rows);
-  rope_f32_kernel<<<grid, 128, 0, s>>>(qkv, rows, ld, rope_cols, hd, pos, cos_t, sin_t);
+  ZSAA_LAUNCH(rope_f32_kernel, dim3(grid), dim3(128), 0, s, qkv, rows, ld, rope_cols, hd, pos, cos_t, sin_t);
   return cudaGetLastError();
 }
 
@@ -423,11 +441,11 @@ cudaError_t launch_cls_head(int dtype, const void* h, int B, int N, int d, const
                             float eps, const void* W, int n_classes, float* out, cudaStream_t s) {
   const size_t smem = static_cast<size_t>(d) * sizeof(float);
   if (dtype == ZSAA_BF16)
-    cls_head_kernel<bf16><<<B, 256, smem, s>>>(static_cast<const bf16*>(h), N, d,
+    ZSAA_LAUNCH(cls_head_kernel<bf16>, dim3(B), dim3(256), smem, s, static_cast<const bf16*>(h), N, d,
                                                static_cast<const bf16*>(norm_w), eps,
                                                static_cast<const bf16*>(W), n_classes, out);
   else
-    cls_head_kernel<float><<<B, 256, smem, s>>>(static_cast<const float*>(h), N, d,
+    ZSAA_LAUNCH(cls_head_kernel<float>, dim3(B), dim3(256), smem, s, static_cast<const float*>(h), N, d,
                                                 static_cast<const float*>(norm_w), eps,
                                                 static_cast<const float*>(W), n_classes, out);
   return cudaGetLastError();

@@ -39,13 +39,17 @@ struct GemmParams {
   int rope_cols;        // kEpiRope: columns [0, rope_cols) are rotated
   int hd;               // kEpiRope: head size
   int* status;          // device status word
-  float* splitk_ws;     // optional fp32 workspace for split-K partial tiles (NULL: no split)
+  float* splitk_ws;     // optional fp32 workspace for split tiles (NULL: whole tiles only)
   size_t splitk_ws_elems;
+  int* splitk_flags;    // kMaxGemmCtas * 4 ints, zero before the first launch
   int* launches;        // optional host counter: kernels launched are added to it
 };
 
-// Split-K workspace a caller should provide: two waves of 128 x 256 fp32 tiles.
-constexpr size_t kSplitKWorkspaceElems = static_cast<size_t>(2) * 160 * 128 * 256;
+// Stream-K workspace a caller should provide: one 128 x 256 fp32 tile per CTA
+// (at most kMaxGemmCtas CTAs), and 4 flags per CTA.
+constexpr int kMaxGemmCtas = 256;
+constexpr size_t kSplitKWorkspaceElems = static_cast<size_t>(kMaxGemmCtas) * 128 * 256;
+constexpr size_t kSplitKFlags = static_cast<size_t>(kMaxGemmCtas) * 4;
 
 // bf16 tensor-core GEMM: out = epi(A[M,K] * W^T).  W is given as up to three
 // row blocks (w0: rows [0, n1), w1: rows [n1, n2), w2: rows [n2, N)) so the

@@ -163,18 +163,24 @@ int* shared_status() {
 
 // Split-K workspace of zsaa_op_linear, one per device, allocated on first use.
 std::mutex g_ws_mu;
-std::unordered_map<int, float*> g_op_ws;
+std::unordered_map<int, std::pair<float*, int*>> g_op_ws;
 
-float* op_splitk_ws() {
+bool op_splitk_ws(float** ws, int** flags) {
   int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
   std::lock_guard<std::mutex> lk(g_ws_mu);
   auto it = g_op_ws.find(dev);
-  if (it != g_op_ws.end()) return it->second;
-  float* p = nullptr;
-  if (cudaMalloc(&p, kSplitKWorkspaceElems * sizeof(float)) != cudaSuccess) return nullptr;
-  g_op_ws[dev] = p;
-  return p;
+  if (it == g_op_ws.end()) {
+    float* p = nullptr;
+    int* f = nullptr;
+    if (cudaMalloc(&p, kSplitKWorkspaceElems * sizeof(float)) != cudaSuccess) return false;
+    if (cudaMalloc(&f, kSplitKFlags * sizeof(int)) != cudaSuccess) return false;
+    if (cudaMemset(f, 0, kSplitKFlags * sizeof(int)) != cudaSuccess) return false;
+    it = g_op_ws.emplace(dev, std::make_pair(p, f)).first;
+  }
+  *ws = it->second.first;
+  *flags = it->second.second;
+  return true;
 }
 
 // RoPE tables of zsaa_op_linear, cached per (device, theta, head size):
@@ -261,6 +267,7 @@ struct zsaa_model {
   float* rope_cos = nullptr;
   float* rope_sin = nullptr;
   float* splitk_ws = nullptr;
+  int* splitk_flags = nullptr;
   int* status = nullptr;
   // host-buffer staging (zsaa_forward_host)
   int32_t* stage_tok = nullptr;
@@ -346,7 +353,8 @@ void free_model(zsaa_model* m) {
   if (m->capture_stream) cudaStreamDestroy(m->capture_stream);
   void* ptrs[] = {m->h[0], m->h[1], m->x, m->qkv, m->attn, m->act, m->lse, m->colmass,
                   m->scores, m->idx, m->pos[0], m->pos[1], m->rope_cos, m->rope_sin,
-                  m->splitk_ws, m->status, m->stage_tok, m->stage_logits, m->stage_pos};
+                  m->splitk_ws, m->splitk_flags, m->status, m->stage_tok, m->stage_logits,
+                  m->stage_pos};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   delete m;
@@ -358,6 +366,7 @@ zsaa_status linear(zsaa_model* m, const void* A, int lda, const TcWeights& W, in
   p.status = m->status;
   p.splitk_ws = m->splitk_ws;
   p.splitk_ws_elems = m->splitk_ws ? kSplitKWorkspaceElems : 0;
+  p.splitk_flags = m->splitk_flags;
   p.launches = kernels;
   if (m->cfg.dtype == ZSAA_BF16) {
     ZCK(launch_gemm_tc(A, lda, W, epi, p, s));
@@ -778,8 +787,10 @@ zsaa_status zsaa_model_create(const zsaa_config* cfg, const zsaa_weights* w, int
   alloc(reinterpret_cast<void**>(&m->rope_cos), static_cast<size_t>(max_L) * half * sizeof(float));
   alloc(reinterpret_cast<void**>(&m->rope_sin), static_cast<size_t>(max_L) * half * sizeof(float));
   alloc(reinterpret_cast<void**>(&m->status), sizeof(int));
-  if (cfg->dtype == ZSAA_BF16)
+  if (cfg->dtype == ZSAA_BF16) {
     alloc(reinterpret_cast<void**>(&m->splitk_ws), kSplitKWorkspaceElems * sizeof(float));
+    alloc(reinterpret_cast<void**>(&m->splitk_flags), kSplitKFlags * sizeof(int));
+  }
   if (!ok) {
     cudaGetLastError();
     free_model(m);
@@ -798,6 +809,7 @@ zsaa_status zsaa_model_create(const zsaa_config* cfg, const zsaa_weights* w, int
   cudaError_t e = cudaMemcpy(m->rope_cos, cs.data(), cs.size() * sizeof(float), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(m->rope_sin, sn.data(), sn.size() * sizeof(float), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemset(m->status, 0, sizeof(int));
+  if (e == cudaSuccess && m->splitk_flags) e = cudaMemset(m->splitk_flags, 0, kSplitKFlags * sizeof(int));
   if (e != cudaSuccess) {
     free_model(m);
     return fail(ZSAA_ERR_CUDA, "workspace initialisation failed: %s", cudaGetErrorString(e));
@@ -924,7 +936,7 @@ zsaa_status zsaa_op_linear(const void* A, const void* W, const void* W2, const v
       p.hd = rope_hd;
     }
     TcWeights Wt{W, W2, nullptr, N, N};
-    p.splitk_ws = op_splitk_ws();
+    if (!op_splitk_ws(&p.splitk_ws, &p.splitk_flags)) p.splitk_ws = nullptr, p.splitk_flags = nullptr;
     p.splitk_ws_elems = p.splitk_ws ? kSplitKWorkspaceElems : 0;
     ZCK(launch_gemm_tc(A, K, Wt, epilogue, p, s));
   } else if (dtype == ZSAA_F32) {
