@@ -310,6 +310,40 @@ def main():
         line["ms_per_step_eager"] = timed(args.accel, args.steps, 3)
         zsaa.zsaa_model_set_graphs(model, True)
 
+        # ---- isolated score + select + compaction on [32, 4096, 4096] bf16 (1 GiB,
+        # larger than L2): algorithmic bytes = read every row once + write the
+        # kept rows = 2*B*L*d + 2*B*k*d
+        mb = I.WORKLOADS["microbench"]
+        mB, mL, md = mb["B"], mb["L"], mb["d"]
+        hidden = I.make_hidden(mB, mL, md, device=dev)
+        peaks_mb, src_mb = load_peaks()
+        hbm = peaks_mb.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+        micro = {}
+        for a in mb["accels"]:
+            k = int(mL // a)
+            idx = torch.empty(mB, k, device=dev, dtype=torch.int32)
+            rows = torch.empty(mB, k, md, device=dev, dtype=torch.bfloat16)
+            for _ in range(3):
+                zsaa.zsaa_score_select(hidden, mB, mL, md, k, idx, rows, stream=stream)
+            torch.cuda.synchronize()
+            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(10)]
+            for e0, e1 in evs:
+                flush.zero_()
+                e0.record(stream)
+                zsaa.zsaa_score_select(hidden, mB, mL, md, k, idx, rows, stream=stream)
+                e1.record(stream)
+            torch.cuda.synchronize()
+            us = 1e3 * sum(e0.elapsed_time(e1) for e0, e1 in evs) / len(evs)
+            nbytes = 2.0 * mB * mL * md + 2.0 * mB * k * md
+            micro[f"{a:g}"] = {"k": k, "us": us, "algorithmic_bytes": nbytes,
+                               "gbs": nbytes / (us * 1e3), "frac_of_hbm": nbytes / (us * 1e3) / hbm}
+            del idx, rows
+        del hidden
+        line["microbench_score_select"] = {
+            "workload": f"hidden [{mB}, {mL}, {md}] bf16, N(0,1) x per-row log-normal scale; "
+                        "zsaa_score_select (row-norm score, top-k, gather)",
+            "peak_gbs": hbm, "peak_source": f"{src_mb} hbm_gbs", "by_accel": micro}
+
         # ---- per-kernel trace of the headline forward (separate traced steps)
         zsaa.zsaa_trace_begin(model)
         n_tr = 3

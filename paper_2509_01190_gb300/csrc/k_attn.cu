@@ -501,14 +501,20 @@ int colmass_chunks(int N) {
   return (n_qb + kColmassQPer - 1) / kColmassQPer;
 }
 
-size_t colmass_parts_elems(int B, int N, int Hkv) {
-  return static_cast<size_t>(colmass_chunks(N)) * B * Hkv * N;
+size_t colmass_parts_elems(int B, int N, int Hq, int Hkv) {
+  const int tc_chunks = 2 * (Hq / Hkv);  // the tensor-core kernel: (head, column half)
+  const int c = colmass_chunks(N) > tc_chunks ? colmass_chunks(N) : tc_chunks;
+  return static_cast<size_t>(c) * B * Hkv * N;
 }
 
 namespace {
-cudaError_t colmass_parts(int dtype, const void* qkv, const float* lse, int B, int N, int Hq,
-                          int Hkv, int hd, int weight_vnorm, float* parts, int* n_qc,
-                          cudaStream_t s) {
+cudaError_t colmass_parts(int dtype, const void* qkv, const float* lse, const float* vnorm, int B,
+                          int N, int Hq, int Hkv, int hd, int weight_vnorm, float* parts, int* n_qc,
+                          int* status, cudaStream_t s) {
+  // tensor-core path (with precomputed norms when they are needed)
+  if (dtype == ZSAA_BF16 && status != nullptr && (!weight_vnorm || vnorm != nullptr))
+    return launch_colmass_tc(qkv, lse, weight_vnorm ? vnorm : nullptr, B, N, Hq, Hkv, hd, parts,
+                             status, n_qc, s);
   const float scale_log2 = kLog2e / sqrtf(static_cast<float>(hd));
   if (dtype == ZSAA_F32) {
     *n_qc = 1;
@@ -541,21 +547,28 @@ cudaError_t colmass_parts(int dtype, const void* qkv, const float* lse, int B, i
 }  // namespace
 
 cudaError_t launch_colmass(int dtype, const void* qkv, const float* lse, int B, int N, int Hq,
-                           int Hkv, int hd, float* parts, float* C, cudaStream_t s) {
+                           int Hkv, int hd, float* parts, float* C, int* status, cudaStream_t s) {
   int n_qc = 1;
-  cudaError_t e = colmass_parts(dtype, qkv, lse, B, N, Hq, Hkv, hd, 0, parts, &n_qc, s);
+  cudaError_t e = colmass_parts(dtype, qkv, lse, nullptr, B, N, Hq, Hkv, hd, 0, parts, &n_qc, status, s);
   if (e != cudaSuccess) return e;
   const int total = B * Hkv * N;
   ZSAA_LAUNCH(colmass_reduce_kernel, dim3((total + 255) / 256), dim3(256), 0, s, parts, n_qc, B, Hkv, N, 0, C);
   return cudaGetLastError();
 }
 
-cudaError_t launch_position_scores(int dtype, const void* qkv, const float* lse, int B, int N,
-                                   int Hq, int Hkv, int hd, int mode, float* parts,
-                                   float* scores, cudaStream_t s) {
+cudaError_t launch_position_parts(int dtype, const void* qkv, const float* lse, const float* vnorm,
+                                  int B, int N, int Hq, int Hkv, int hd, int mode, float* parts,
+                                  int* n_qc, int* status, cudaStream_t s) {
+  return colmass_parts(dtype, qkv, lse, vnorm, B, N, Hq, Hkv, hd,
+                       mode == ZSAA_SCORE_SOFTSCORE_VNORM ? 1 : 0, parts, n_qc, status, s);
+}
+
+cudaError_t launch_position_scores(int dtype, const void* qkv, const float* lse, const float* vnorm,
+                                   int B, int N, int Hq, int Hkv, int hd, int mode, float* parts,
+                                   float* scores, int* status, cudaStream_t s) {
   int n_qc = 1;
-  cudaError_t e = colmass_parts(dtype, qkv, lse, B, N, Hq, Hkv, hd,
-                                mode == ZSAA_SCORE_SOFTSCORE_VNORM ? 1 : 0, parts, &n_qc, s);
+  cudaError_t e = colmass_parts(dtype, qkv, lse, vnorm, B, N, Hq, Hkv, hd,
+                                mode == ZSAA_SCORE_SOFTSCORE_VNORM ? 1 : 0, parts, &n_qc, status, s);
   if (e != cudaSuccess) return e;
   const int total = B * N;
   ZSAA_LAUNCH(colmass_reduce_kernel, dim3((total + 255) / 256), dim3(256), 0, s, parts, n_qc, B, Hkv, N, 1, scores);

@@ -231,6 +231,7 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
 #pragma unroll 1
     for (int hs = 0; hs < BN; hs += hd) {
       const bool rot = n0 + hs < p.rope_cols;
+      float vss = 0.f;  // value heads: sum of squares of the stored (bf16) values
 #pragma unroll 1
       for (int c = 0; c < half; c += 16) {
         uint32_t x1[16], x2[16];
@@ -279,7 +280,19 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
           bf16* rowp = out + static_cast<size_t>(row) * p.ldo + n0 + hs;
           store_bf16x16(rowp + c, y1);
           store_bf16x16(rowp + half + c, y2);
+          if (!rot && p.vnorm_out != nullptr) {
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+              const float r1 = __bfloat162float(__float2bfloat16_rn(y1[e]));
+              const float r2 = __bfloat162float(__float2bfloat16_rn(y2[e]));
+              vss += r1 * r1 + r2 * r2;
+            }
+          }
         }
+      }
+      if (!rot && p.vnorm_out != nullptr && row_ok && n0 + hs < p.N) {
+        const int groups = (p.N - p.rope_cols) / hd;
+        p.vnorm_out[static_cast<size_t>(row) * groups + (n0 + hs - p.rope_cols) / hd] = sqrtf(vss);
       }
     }
   } else {  // kEpiStore / kEpiResid, bf16 out

@@ -168,15 +168,33 @@ constexpr int kSelThreads = 1024;
 // then an index-ordered ballot/prefix scan writes the kept indices ascending.
 // Ties (equal keys) keep lower indices first.  With force_last the last index
 // is kept and the other k-1 come from indices [0, N-1).
+// FROM_PARTS: the scores are first summed from column-mass partials
+// parts[qc][b][g][j] (n_qc chunks, G groups) into shared memory (and copied to
+// scores_out when it is not null); otherwise they are read from `scores`.
+template <bool FROM_PARTS>
 __global__ void __launch_bounds__(kSelThreads)
     select_topk_kernel(const float* __restrict__ scores, int N, int k, int force_last,
-                       int32_t* __restrict__ idx_out) {
+                       int32_t* __restrict__ idx_out, const float* __restrict__ parts, int n_qc,
+                       int B, int G, float* __restrict__ scores_out) {
   pdl_trigger();
   pdl_wait();
   const int b = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int nwarps = kSelThreads / 32;
+  extern __shared__ float sscore[];
   const float* s = scores + static_cast<size_t>(b) * N;
+  if (FROM_PARTS) {
+    const size_t plane = static_cast<size_t>(B) * G * N;
+    for (int j = tid; j < N; j += kSelThreads) {
+      float acc = 0.f;
+      for (int qc = 0; qc < n_qc; ++qc)
+        for (int g = 0; g < G; ++g) acc += parts[qc * plane + (static_cast<size_t>(b) * G + g) * N + j];
+      sscore[j] = acc;
+      if (scores_out != nullptr) scores_out[static_cast<size_t>(b) * N + j] = acc;
+    }
+    __syncthreads();
+    s = sscore;
+  }
   int32_t* out = idx_out + static_cast<size_t>(b) * k;
   const int n_cand = force_last ? N - 1 : N;
   const int need = force_last ? k - 1 : k;
@@ -307,6 +325,86 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ src, int N, int k, 
   if (pos_out != nullptr && lane == 0) pos_out[r] = pos_in[srow];
 }
 
+// ---------------------------------------------------------------- row copy + RMSNorm
+
+// Copies source rows into the residual buffer and writes their RMSNorm, for
+// bf16 rows of d = 8 * vec elements (vec <= 32 * kMaxVecPerLane):
+//   embedding (idx == nullptr): source row tok[r] of E, pos_out[r] = r mod L;
+//   compaction: source row b*N + idx[r] of h (b = r / k), pos_out[r] =
+//     pos_in[that row] -- the kept rows of the previous layer, already normed
+//     for the next layer's attention.
+// An index outside its range sets kStatusBadIndex and copies row 0.
+constexpr int kMaxVecPerLane = 16;
+
+__global__ void rows_norm_bf16_kernel(const uint4* __restrict__ src, const int32_t* __restrict__ tok,
+                                      int vocab, int L, const int32_t* __restrict__ idx, int N,
+                                      int k, const int32_t* __restrict__ pos_in, int rows, int vec,
+                                      const uint4* __restrict__ w, float eps,
+                                      uint4* __restrict__ h_out, uint4* __restrict__ x_out,
+                                      int32_t* __restrict__ pos_out, int* status) {
+  pdl_trigger();
+  pdl_wait();
+  const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= rows) return;
+  size_t srow;
+  int p;
+  if (idx == nullptr) {
+    int t = tok[r];
+    if (t < 0 || t >= vocab) {
+      if (lane == 0 && status != nullptr) atomicOr(status, kStatusBadIndex);
+      t = 0;
+    }
+    srow = static_cast<size_t>(t);
+    p = r % L;
+  } else {
+    const int b = r / k;
+    int j = idx[r];
+    if (j < 0 || j >= N) {
+      if (lane == 0 && status != nullptr) atomicOr(status, kStatusBadIndex);
+      j = 0;
+    }
+    srow = static_cast<size_t>(b) * N + j;
+    p = pos_in[srow];
+  }
+  const uint4* sr = src + srow * vec;
+  uint4* hr = h_out + static_cast<size_t>(r) * vec;
+  uint4* xr = x_out + static_cast<size_t>(r) * vec;
+  uint4 u[kMaxVecPerLane];
+  float ss = 0.f;
+#pragma unroll
+  for (int q = 0; q < kMaxVecPerLane; ++q) {
+    const int v = lane + 32 * q;
+    if (v < vec) {
+      u[q] = sr[v];
+      hr[v] = u[q];
+      const uint32_t e4[4] = {u[q].x, u[q].y, u[q].z, u[q].w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float a = bf16lo(e4[e]), c = bf16hi(e4[e]);
+        ss += a * a + c * c;
+      }
+    }
+  }
+  ss = warp_sum(ss);
+  const float inv = rsqrtf(ss / static_cast<float>(vec * 8) + eps);
+#pragma unroll
+  for (int q = 0; q < kMaxVecPerLane; ++q) {
+    const int v = lane + 32 * q;
+    if (v < vec) {
+      const uint4 wv = __ldg(w + v);
+      const uint32_t e4[4] = {u[q].x, u[q].y, u[q].z, u[q].w};
+      const uint32_t w4[4] = {wv.x, wv.y, wv.z, wv.w};
+      uint32_t o[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        o[e] = pack_bf16x2(bf16lo(e4[e]) * inv * bf16lo(w4[e]), bf16hi(e4[e]) * inv * bf16hi(w4[e]));
+      xr[v] = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+  }
+  if (lane == 0) pos_out[r] = p;
+}
+
 // ---------------------------------------------------------------- RoPE (fp32 path)
 
 // Rotate pairs (c, c + hd/2) of every head in columns [0, rope_cols) of each row.
@@ -414,7 +512,31 @@ cudaError_t launch_row_norm(int dtype, const void* h, int rows, int d, float* sc
 
 cudaError_t launch_select(const float* scores, int B, int N, int k, int force_last, int32_t* idx,
                           cudaStream_t s) {
-  ZSAA_LAUNCH(select_topk_kernel, dim3(B), dim3(kSelThreads), 0, s, scores, N, k, force_last, idx);
+  ZSAA_LAUNCH(select_topk_kernel<false>, dim3(B), dim3(kSelThreads), 0, s, scores, N, k, force_last,
+              idx, static_cast<const float*>(nullptr), 0, B, 0, static_cast<float*>(nullptr));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_select_parts(const float* parts, int n_qc, int B, int G, int N, int k,
+                                int force_last, int32_t* idx, float* scores_out, cudaStream_t s) {
+  const size_t smem = static_cast<size_t>(N) * sizeof(float);
+  static cudaError_t attr = cudaFuncSetAttribute(select_topk_kernel<true>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 static_cast<int>(kSelectPartsMaxN * sizeof(float)));
+  if (attr != cudaSuccess) return attr;
+  ZSAA_LAUNCH(select_topk_kernel<true>, dim3(B), dim3(kSelThreads), smem, s,
+              static_cast<const float*>(nullptr), N, k, force_last, idx, parts, n_qc, B, G, scores_out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rows_norm(const void* src, const int32_t* tok, int vocab, int L,
+                             const int32_t* idx, int N, int k, const int32_t* pos_in, int rows,
+                             int d, const void* w, float eps, void* h_out, void* x_out,
+                             int32_t* pos_out, int* status, cudaStream_t s) {
+  ZSAA_LAUNCH(rows_norm_bf16_kernel, dim3(row_blocks(rows)), dim3(32 * kWarpsPerBlock), 0, s,
+              static_cast<const uint4*>(src), tok, vocab, L, idx, N, k, pos_in, rows, d / 8,
+              static_cast<const uint4*>(w), eps, static_cast<uint4*>(h_out),
+              static_cast<uint4*>(x_out), pos_out, status);
   return cudaGetLastError();
 }
 

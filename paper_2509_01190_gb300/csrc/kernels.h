@@ -16,6 +16,20 @@ cudaError_t launch_row_norm(int dtype, const void* h, int rows, int d, float* sc
                             cudaStream_t s);
 cudaError_t launch_select(const float* scores, int B, int N, int k, int force_last, int32_t* idx,
                           cudaStream_t s);
+// Top-k from column-mass partials parts[n_qc][B][G][N] (scores summed in shared
+// memory, copied to scores_out when not null); N <= kSelectPartsMaxN.
+constexpr int kSelectPartsMaxN = 12288;
+cudaError_t launch_select_parts(const float* parts, int n_qc, int B, int G, int N, int k,
+                                int force_last, int32_t* idx, float* scores_out, cudaStream_t s);
+// bf16 rows: h_out[r] = source row, x_out[r] = RMSNorm(h_out[r]) * w, pos_out[r].
+// Embedding when idx == nullptr (rows = B*L, source row tok[r] of E);
+// otherwise compaction (rows = B*k, source row b*N + idx[r] of h).
+// d % 8 == 0 and d <= kRowsNormMaxD.
+constexpr int kRowsNormMaxD = 8 * 32 * 16;
+cudaError_t launch_rows_norm(const void* src, const int32_t* tok, int vocab, int L,
+                             const int32_t* idx, int N, int k, const int32_t* pos_in, int rows,
+                             int d, const void* w, float eps, void* h_out, void* x_out,
+                             int32_t* pos_out, int* status, cudaStream_t s);
 cudaError_t launch_gather(const void* src, int B, int N, int k, int row_bytes, const int32_t* idx,
                           void* dst, const int32_t* pos_in, int32_t* pos_out, int* status,
                           cudaStream_t s);
@@ -43,6 +57,7 @@ struct GemmParams {
   size_t splitk_ws_elems;
   int* splitk_flags;    // kMaxGemmCtas * 4 ints, zero before the first launch
   int* launches;        // optional host counter: kernels launched are added to it
+  float* vnorm_out;     // kEpiRope: if set, ||v|| of each row's value heads, [M, (N - rope_cols) / hd]
 };
 
 // Stream-K workspace a caller should provide: one 128 x 256 fp32 tile per CTA
@@ -71,18 +86,32 @@ cudaError_t launch_gemm_f32(const float* A, int lda, const float* W, const float
 // ---- attention (k_attn.cu)
 cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, int Hkv, int hd,
                              void* out, float* lse, cudaStream_t s);
-// Column mass C[B, Hkv, N] (via query-chunk partials in `parts`, which must
-// hold colmass_parts_elems(B, N, Hkv) floats).
-constexpr int kColmassQPer = 2;  // query blocks of 64 per column-mass CTA
+// Column mass C[B, Hkv, N] (via partial sums in `parts`, which must hold
+// colmass_parts_elems(B, N, Hq, Hkv) floats).  bf16 with a status word runs
+// the tensor-core kernel (k_colmass_tc.cu); otherwise the mma.sync / fp32 ones.
+constexpr int kColmassQPer = 2;  // query blocks of 64 per mma.sync column-mass CTA
 int colmass_chunks(int N);
-size_t colmass_parts_elems(int B, int N, int Hkv);
+size_t colmass_parts_elems(int B, int N, int Hq, int Hkv);
 cudaError_t launch_colmass(int dtype, const void* qkv, const float* lse, int B, int N, int Hq,
-                           int Hkv, int hd, float* parts, float* C, cudaStream_t s);
+                           int Hkv, int hd, float* parts, float* C, int* status, cudaStream_t s);
+// The score paths below take vnorm = ||v|| per row and group ([B*N, Hkv], from
+// the QKV epilogue) for the bf16 tensor-core kernel; NULL makes the kernels
+// compute the norms from qkv themselves.
 // Position scores s[B, N] of R1 (mode ZSAA_SCORE_*): column mass weighted by
 // ||v|| per group, summed over groups; same workspace as launch_colmass.
-cudaError_t launch_position_scores(int dtype, const void* qkv, const float* lse, int B, int N,
-                                   int Hq, int Hkv, int hd, int mode, float* parts,
-                                   float* scores, cudaStream_t s);
+cudaError_t launch_position_scores(int dtype, const void* qkv, const float* lse, const float* vnorm,
+                                   int B, int N, int Hq, int Hkv, int hd, int mode, float* parts,
+                                   float* scores, int* status, cudaStream_t s);
+// Only the partials of the position scores (for launch_select_parts); *n_qc
+// receives the number of partial chunks.
+cudaError_t launch_position_parts(int dtype, const void* qkv, const float* lse, const float* vnorm,
+                                  int B, int N, int Hq, int Hkv, int hd, int mode, float* parts,
+                                  int* n_qc, int* status, cudaStream_t s);
+// Tensor-core column-mass partials: parts[Hq/Hkv][B][Hkv][N] (per head of the
+// group), times vnorm when it is not NULL; hd 64 or 128.
+cudaError_t launch_colmass_tc(const void* qkv, const float* lse, const float* vnorm, int B, int N,
+                              int Hq, int Hkv, int hd, float* parts, int* status, int* n_chunks,
+                              cudaStream_t s);
 
 // ---- thread-local message returned by zsaa_last_error (zsaa_api.cu)
 void set_last_error(const char* msg);

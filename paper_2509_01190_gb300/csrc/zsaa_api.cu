@@ -261,6 +261,7 @@ struct zsaa_model {
   void* act = nullptr;
   float* lse = nullptr;
   float* colmass = nullptr;  // query-chunk partials of the column mass / scores
+  float* vnorm = nullptr;    // ||v|| per row and KV group, from the QKV epilogue (bf16)
   float* scores = nullptr;
   int32_t* idx = nullptr;
   int32_t* pos[2] = {nullptr, nullptr};
@@ -351,7 +352,7 @@ void free_model(zsaa_model* m) {
   for (auto& g : m->graphs)
     if (g.exec) cudaGraphExecDestroy(g.exec);
   if (m->capture_stream) cudaStreamDestroy(m->capture_stream);
-  void* ptrs[] = {m->h[0], m->h[1], m->x, m->qkv, m->attn, m->act, m->lse, m->colmass,
+  void* ptrs[] = {m->h[0], m->h[1], m->x, m->qkv, m->attn, m->act, m->lse, m->colmass, m->vnorm,
                   m->scores, m->idx, m->pos[0], m->pos[1], m->rope_cos, m->rope_sin,
                   m->splitk_ws, m->splitk_flags, m->status, m->stage_tok, m->stage_logits,
                   m->stage_pos};
@@ -426,9 +427,22 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
                           cudaMemcpyHostToDevice, s));
       ZCK(cudaStreamSynchronize(s));
     }
-  } else {
-    TRACE("embed", 0.0, static_cast<double>(B) * L * (d * es + 8.0));
-    ZCK(launch_embed(dt, m->embed, tok, B * L, L, c.vocab, d, m->h[cur], m->pos[cur], m->status, s));
+  }
+  // bf16 rows of moderate width: embedding and compaction also write the next
+  // layer's normed input (x_ready), saving that layer's RMSNorm launch.
+  const bool fuse_norm = dt == ZSAA_BF16 && d % 8 == 0 && d <= kRowsNormMaxD;
+  bool x_ready = false;
+  if (!from_hidden) {
+    if (fuse_norm && first <= n_run) {
+      TRACE("embed_norm", 0.0, static_cast<double>(B) * L * (3.0 * d * es + 8.0));
+      ZCK(launch_rows_norm(m->embed, tok, c.vocab, L, nullptr, 0, 0, nullptr, B * L, d,
+                           LW(m, first - 1, kAttnNorm), c.rms_eps, m->h[cur], m->x, m->pos[cur],
+                           m->status, s));
+      x_ready = true;
+    } else {
+      TRACE("embed", 0.0, static_cast<double>(B) * L * (d * es + 8.0));
+      ZCK(launch_embed(dt, m->embed, tok, B * L, L, c.vocab, d, m->h[cur], m->pos[cur], m->status, s));
+    }
   }
   size_t off_forced = 0, off_scores = 0, off_idx = 0;
   int N = L;
@@ -438,10 +452,11 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
     void* h = m->h[cur];
     const double Md = static_cast<double>(M);
     // attention branch
-    {
+    if (!x_ready) {
       TRACE("rmsnorm", 0.0, 2.0 * Md * d * es);
       ZCK(launch_rmsnorm(dt, h, LW(m, li, kAttnNorm), M, d, c.rms_eps, m->x, s));
     }
+    x_ready = false;
     GemmParams p{};
     p.M = M;
     p.K = d;
@@ -454,6 +469,7 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
       p.sin_t = m->rope_sin;
       p.rope_cols = m->dq + m->dkv;
       p.hd = hd;
+      p.vnorm_out = m->vnorm;
       TcWeights W{LW(m, li, kWq), LW(m, li, kWk), LW(m, li, kWv), m->dq, m->dq + m->dkv};
       TRACE("gemm_qkv_rope", 2.0 * Md * m->ld_qkv * d, (Md * d + static_cast<double>(m->ld_qkv) * d + Md * m->ld_qkv) * es);
       trace_scope_.kernels = 0;
@@ -538,28 +554,50 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
       const bool want_idx = opts && opts->idx_out;
       if (k < N || want_scores || want_idx) {
         float* sc = want_scores ? opts->scores_out + off_scores : m->scores;
-        {
-          const double pairs = static_cast<double>(B) * Hq * (static_cast<double>(N) * (N + 1) / 2.0);
-          TRACE("colmass_score", 2.0 * pairs * hd,
-                Md * (m->dq + 2 * m->dkv) * es + static_cast<double>(B) * Hq * N * 4.0 + Md * 4.0);
-          trace_scope_.kernels = 2;
-          ZCK(launch_position_scores(dt, m->qkv, m->lse, B, N, Hq, Hkv, hd, c.score_mode, m->colmass,
-                                     sc, s));
-        }
+        const double pairs = static_cast<double>(B) * Hq * (static_cast<double>(N) * (N + 1) / 2.0);
         const int32_t* idx = m->idx;
-        if (forced) {
-          idx = opts->forced_idx + off_forced;
-        } else {  // with k == N (only when idx_out is requested) this yields 0..N-1
-          TRACE("select", 0.0, Md * 4.0 + static_cast<double>(B) * k * 4.0);
-          ZCK(launch_select(sc, B, N, k, c.force_keep_last, m->idx, s));
+        if (dt == ZSAA_BF16 && !forced && k < N && N <= kSelectPartsMaxN) {
+          // column-mass partials, then top-k with the score reduction fused in
+          int n_qc = 1;
+          {
+            TRACE("colmass", 2.0 * pairs * hd,
+                  Md * (m->dq + 2 * m->dkv) * es + static_cast<double>(B) * Hq * N * 4.0);
+            ZCK(launch_position_parts(dt, m->qkv, m->lse, dt == ZSAA_BF16 ? m->vnorm : nullptr, B, N,
+                                      Hq, Hkv, hd, c.score_mode, m->colmass, &n_qc, m->status, s));
+          }
+          TRACE("select", 0.0, static_cast<double>(n_qc) * B * Hkv * N * 4.0 + static_cast<double>(B) * k * 4.0);
+          ZCK(launch_select_parts(m->colmass, n_qc, B, Hkv, N, k, c.force_keep_last, m->idx,
+                                  want_scores ? sc : nullptr, s));
+        } else {
+          {
+            TRACE("colmass", 2.0 * pairs * hd,
+                  Md * (m->dq + 2 * m->dkv) * es + static_cast<double>(B) * Hq * N * 4.0 + Md * 4.0);
+            trace_scope_.kernels = 2;
+            ZCK(launch_position_scores(dt, m->qkv, m->lse, dt == ZSAA_BF16 ? m->vnorm : nullptr, B, N,
+                                       Hq, Hkv, hd, c.score_mode, m->colmass, sc, m->status, s));
+          }
+          if (forced) {
+            idx = opts->forced_idx + off_forced;
+          } else {  // with k == N (only when idx_out is requested) this yields 0..N-1
+            TRACE("select", 0.0, Md * 4.0 + static_cast<double>(B) * k * 4.0);
+            ZCK(launch_select(sc, B, N, k, c.force_keep_last, m->idx, s));
+          }
         }
         if (want_idx)
           ZCK(cudaMemcpyAsync(opts->idx_out + off_idx, idx, sizeof(int32_t) * B * k,
                               cudaMemcpyDeviceToDevice, s));
         if (k < N) {
-          TRACE("gather", 0.0, static_cast<double>(B) * k * (2.0 * d * es + 12.0));
-          ZCK(launch_gather(h, B, N, k, static_cast<int>(d * m->esz), idx, m->h[cur ^ 1],
-                            m->pos[cur], m->pos[cur ^ 1], m->status, s));
+          if (fuse_norm && l < n_run) {
+            TRACE("gather_norm", 0.0, static_cast<double>(B) * k * (3.0 * d * es + 12.0));
+            ZCK(launch_rows_norm(h, nullptr, 0, 0, idx, N, k, m->pos[cur], B * k, d,
+                                 LW(m, l, kAttnNorm), c.rms_eps, m->h[cur ^ 1], m->x,
+                                 m->pos[cur ^ 1], m->status, s));
+            x_ready = true;
+          } else {
+            TRACE("gather", 0.0, static_cast<double>(B) * k * (2.0 * d * es + 12.0));
+            ZCK(launch_gather(h, B, N, k, static_cast<int>(d * m->esz), idx, m->h[cur ^ 1],
+                              m->pos[cur], m->pos[cur ^ 1], m->status, s));
+          }
           cur ^= 1;
         }
       }
@@ -778,7 +816,8 @@ zsaa_status zsaa_model_create(const zsaa_config* cfg, const zsaa_weights* w, int
   alloc(&m->act, rows * F * esz);
   alloc(reinterpret_cast<void**>(&m->lse), rows * cfg->n_heads * sizeof(float));
   alloc(reinterpret_cast<void**>(&m->colmass),
-        colmass_parts_elems(max_B, max_L, cfg->n_kv_heads) * sizeof(float));
+        colmass_parts_elems(max_B, max_L, cfg->n_heads, cfg->n_kv_heads) * sizeof(float));
+  alloc(reinterpret_cast<void**>(&m->vnorm), rows * cfg->n_kv_heads * sizeof(float));
   alloc(reinterpret_cast<void**>(&m->scores), rows * sizeof(float));
   alloc(reinterpret_cast<void**>(&m->idx), rows * sizeof(int32_t));
   alloc(reinterpret_cast<void**>(&m->pos[0]), rows * sizeof(int32_t));
@@ -966,9 +1005,11 @@ zsaa_status zsaa_op_colmass(const void* qkv, const float* lse, int B, int N, int
   if (dtype == ZSAA_BF16 && hd != 64 && hd != 128) return fail(ZSAA_ERR_UNSUPPORTED, "bf16 column mass needs hd 64 or 128");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   float* parts = nullptr;
+  int* status = shared_status();
+  if (status == nullptr) return fail(ZSAA_ERR_CUDA, "status word allocation failed");
   ZCK(cudaMallocAsync(reinterpret_cast<void**>(&parts),
-                      colmass_parts_elems(B, N, Hkv) * sizeof(float), s));
-  cudaError_t e = launch_colmass(dtype, qkv, lse, B, N, Hq, Hkv, hd, parts, colmass, s);
+                      colmass_parts_elems(B, N, Hq, Hkv) * sizeof(float), s));
+  cudaError_t e = launch_colmass(dtype, qkv, lse, B, N, Hq, Hkv, hd, parts, colmass, status, s);
   cudaError_t e2 = cudaFreeAsync(parts, s);
   ZCK(e);
   ZCK(e2);
