@@ -20,6 +20,9 @@ Every function follows one passage of the paper:
   with the Sec. 3.3 elimination applied after each pruning layer.
 * ``forward_masked`` -- Appendix B: the "marked as pruned but not removed"
   formulation, an independent second route to the same kept-row outputs.
+* ``decode_step`` / ``generate`` -- Sec. 3.3 carried into generation: a row
+  eliminated before layer l is absent from layer l, so a generated token
+  attends, in layer l, to the keys and values of the rows that layer kept.
 
 Readings of points the paper leaves open (each is listed in the design notes):
 
@@ -296,10 +299,12 @@ def _as64(a) -> np.ndarray:
 
 
 def attention_block(cfg: OracleConfig, lw: Dict[str, np.ndarray], h: np.ndarray, pos: np.ndarray,
-                    store: _Store, key_mask: Optional[np.ndarray] = None):
+                    store: _Store, key_mask: Optional[np.ndarray] = None,
+                    kv_out: Optional[list] = None):
     """Pre-norm attention branch of one layer on rows h [n, d].
 
-    Returns (new residual h, P [H, n, n], v [n, Hkv, hd]).
+    Returns (new residual h, P [H, n, n], v [n, Hkv, hd]).  If ``kv_out`` is a
+    list, the layer's stored keys (after RoPE) and values are appended to it.
     """
     n = h.shape[0]
     H, G, hd = cfg.n_heads, cfg.n_kv_heads, cfg.head_dim
@@ -308,6 +313,8 @@ def attention_block(cfg: OracleConfig, lw: Dict[str, np.ndarray], h: np.ndarray,
     q = store(apply_rope((x @ _as64(lw["wq"]).T).reshape(n, H, hd), cos, sin))
     k = store(apply_rope((x @ _as64(lw["wk"]).T).reshape(n, G, hd), cos, sin))
     v = store((x @ _as64(lw["wv"]).T).reshape(n, G, hd))
+    if kv_out is not None:
+        kv_out.append((k, v))
     per = H // G
     P = np.empty((H, n, n))
     o = np.empty((n, H, hd))
@@ -339,7 +346,7 @@ def head(cfg: OracleConfig, weights, h: np.ndarray, store: _Store) -> np.ndarray
 
 def forward(cfg: OracleConfig, weights, tokens: np.ndarray, accel: Optional[float] = None,
             alpha: Optional[float] = None, forced_idx: Optional[Dict[int, np.ndarray]] = None,
-            collect: bool = False):
+            collect: bool = False, collect_cache: bool = False):
     """Pruned prefill of a batch of token sequences [B, L].
 
     The preservation schedule comes from ``accel`` (via ``plan``) or from
@@ -352,6 +359,8 @@ def forward(cfg: OracleConfig, weights, tokens: np.ndarray, accel: Optional[floa
     ``idx`` [B, k] and ``scores`` [B, N_{l-1}].  With ``collect`` it also has
     ``layer_inputs`` {l: (h [B, N_{l-1}, d], pos [B, N_{l-1}])} and
     ``final_hidden`` [B, N_n, d] (the residual rows entering the head).
+    With ``collect_cache`` it also has ``cache`` (see ``decode_step``): per
+    layer the stored keys and values of the rows that layer ran on.
     """
     tokens = np.asarray(tokens)
     B, L = tokens.shape
@@ -367,6 +376,7 @@ def forward(cfg: OracleConfig, weights, tokens: np.ndarray, accel: Optional[floa
     idx_all: Dict[int, list] = {}
     scores_all: Dict[int, list] = {}
     inputs_all: Dict[int, list] = {}
+    cache_all: Dict[int, list] = {}
     finals = []
     for b in range(B):
         h = store(emb[tokens[b]])
@@ -375,7 +385,10 @@ def forward(cfg: OracleConfig, weights, tokens: np.ndarray, accel: Optional[floa
             lw = weights["layers"][layer - 1]
             if collect:
                 inputs_all.setdefault(layer, []).append((h, pos))
-            h, P, v = attention_block(cfg, lw, h, pos, store)
+            kv: list = []
+            h, P, v = attention_block(cfg, lw, h, pos, store, kv_out=kv)
+            if collect_cache:
+                cache_all.setdefault(layer, []).append((kv[0][0], kv[0][1], pos))
             h = mlp_block(cfg, lw, h, store)
             k_keep = sched[layer]
             if layer in set(cfg.prune_layers):
@@ -406,6 +419,11 @@ def forward(cfg: OracleConfig, weights, tokens: np.ndarray, accel: Optional[floa
         out["layer_inputs"] = {k: (np.stack([a for a, _ in v]), np.stack([p for _, p in v]))
                                for k, v in inputs_all.items()}
         out["final_hidden"] = np.stack(finals)
+    if collect_cache:
+        out["cache"] = {"L": L, "layers": {
+            layer: {"k": np.stack([a for a, _, _ in v]), "v": np.stack([b for _, b, _ in v]),
+                    "pos": np.stack([p for _, _, p in v])}
+            for layer, v in cache_all.items()}}
     return out
 
 
@@ -450,6 +468,96 @@ def forward_masked(cfg: OracleConfig, weights, tokens: np.ndarray, sched: Sequen
         "kept_pos": np.stack(kept_pos),
         "kept_by_layer": {k: np.stack(v) for k, v in kept_by_layer.items()},
     }
+
+
+# --------------------------------------------------------------------------
+# generation over the pruned KV cache
+# --------------------------------------------------------------------------
+
+
+def attention_probs_one(q: np.ndarray, k: np.ndarray) -> np.ndarray:
+    """Eq. 1 for one query that comes after every key: softmax(q k^T / sqrt(d_k)).
+
+    q: [hd], k: [n, hd].  The causal mask hides nothing here (every cached key
+    is at an earlier position, or is the query's own).  Returns p [n]."""
+    logits = (k @ q) / math.sqrt(q.shape[0])
+    e = np.exp(logits - np.max(logits))
+    return e / np.sum(e)
+
+
+def decode_step(cfg: OracleConfig, weights, cache, tokens: np.ndarray):
+    """One generated token per sequence after a pruned prefill.
+
+    Sec. 3.3 removes a pruned row from every later layer, so in layer l the
+    new token attends to the rows layer l ran on during the prefill (their
+    stored keys and values, RoPE at their original positions) plus the tokens
+    generated so far and itself; generated tokens are never pruned.
+
+    cache: ``{"L": L, "layers": {l: {"k": [B, n_l, Hkv, hd], "v": ..., "pos": [B, n_l]}}}``
+    as returned by ``forward(..., collect_cache=True)`` or a previous call.
+    tokens: [B] ids of the new tokens, at position L + (tokens generated so far).
+    Returns (logits [B, V] of the new tokens, the cache with their keys and values appended).
+    """
+    if cfg.n_classes > 0:
+        raise ValueError("generation needs the language-model head")
+    tokens = np.asarray(tokens)
+    B = tokens.shape[0]
+    H, G, hd = cfg.n_heads, cfg.n_kv_heads, cfg.head_dim
+    per = H // G
+    store = _Store(cfg.dtype)
+    emb = _as64(weights["embed"])
+    layers = cache["layers"]
+    position = cache["L"] + cache.get("generated", 0)
+    new_layers = {}
+    logits = []
+    for layer in range(1, cfg.n_layers + 1):
+        new_layers[layer] = {"k": [], "v": [], "pos": []}
+    for b in range(B):
+        h = store(emb[tokens[b]])[None, :]
+        for layer in range(1, cfg.n_layers + 1):
+            lw = weights["layers"][layer - 1]
+            c = layers[layer]
+            x = store(rmsnorm(h, lw["attn_norm"], cfg.rms_eps))
+            cos, sin = rope_angles(np.array([position]), hd, cfg.rope_theta)
+            q = store(apply_rope((x @ _as64(lw["wq"]).T).reshape(1, H, hd), cos, sin))[0]
+            k = store(apply_rope((x @ _as64(lw["wk"]).T).reshape(1, G, hd), cos, sin))
+            v = store((x @ _as64(lw["wv"]).T).reshape(1, G, hd))
+            K = np.concatenate([c["k"][b], k], axis=0)
+            V = np.concatenate([c["v"][b], v], axis=0)
+            o = np.empty((H, hd))
+            for hh in range(H):
+                g = hh // per
+                o[hh] = attention_probs_one(q[hh], K[:, g, :]) @ V[:, g, :]
+            o = store(o.reshape(1, H * hd))
+            h = store(h + o @ _as64(lw["wo"]).T)
+            h = mlp_block(cfg, lw, h, store)
+            new_layers[layer]["k"].append(K)
+            new_layers[layer]["v"].append(V)
+            new_layers[layer]["pos"].append(np.append(c["pos"][b], position))
+        logits.append(head(cfg, weights, h, store)[0])
+    out_cache = {"L": cache["L"], "generated": cache.get("generated", 0) + 1,
+                 "layers": {layer: {kk: np.stack(vv) for kk, vv in d.items()}
+                            for layer, d in new_layers.items()}}
+    return np.stack(logits), out_cache
+
+
+def generate(cfg: OracleConfig, weights, tokens: np.ndarray, new_tokens: np.ndarray,
+             accel: Optional[float] = None, alpha: Optional[float] = None,
+             forced_idx: Optional[Dict[int, np.ndarray]] = None):
+    """Pruned prefill of tokens [B, L], then one ``decode_step`` per column of
+    new_tokens [B, T] (teacher-forced ids).  Returns a dict with the prefill's
+    output (``prefill``), ``logits`` [B, T, V] of the generated tokens and the
+    final ``cache``."""
+    pre = forward(cfg, weights, tokens, accel=accel, alpha=alpha, forced_idx=forced_idx,
+                  collect_cache=True)
+    cache = pre["cache"]
+    out = []
+    for t in range(np.asarray(new_tokens).shape[1]):
+        lg, cache = decode_step(cfg, weights, cache, np.asarray(new_tokens)[:, t])
+        out.append(lg)
+    T = np.asarray(new_tokens).shape[1]
+    logits = np.stack(out, axis=1) if T else np.zeros((tokens.shape[0], 0, cfg.vocab))
+    return {"prefill": pre, "logits": logits, "cache": cache}
 
 
 # --------------------------------------------------------------------------

@@ -287,8 +287,11 @@ def _tiny_weights(cfg, seed=0, scale=0.3):
     return dict(embed=nrm(cfg.vocab, d), layers=layers, final_norm=1 + 0.1 * nrm(d), head=nrm(heads, d))
 
 
-def _torch_forward_unpruned(cfg, w, tokens):
-    """Unpruned decoder composed from torch library routines (float64)."""
+def _torch_forward_unpruned(cfg, w, tokens, key_alive=None, all_rows=False):
+    """Unpruned decoder composed from torch library routines (float64).
+
+    ``key_alive[l]`` (bool [B, n], 0-based layer l) hides keys from layer l on
+    top of the causal mask; ``all_rows`` returns logits of every row."""
     T = lambda a: torch.from_numpy(np.asarray(a, np.float64))  # noqa: E731
     H, G, hd, d = cfg.n_heads, cfg.n_kv_heads, cfg.head_dim, cfg.d_model
     out = []
@@ -296,21 +299,27 @@ def _torch_forward_unpruned(cfg, w, tokens):
         n = tokens.shape[1]
         h = T(w["embed"])[torch.from_numpy(tokens[b].astype(np.int64))]
         pos = np.arange(n)
-        for lw in w["layers"]:
+        for li, lw in enumerate(w["layers"]):
             x = F.rms_norm(h, (d,), weight=T(lw["attn_norm"]), eps=cfg.rms_eps)
             q = F.linear(x, T(lw["wq"])).view(n, H, hd).numpy()
             k = F.linear(x, T(lw["wk"])).view(n, G, hd).numpy()
             v = F.linear(x, T(lw["wv"])).view(n, G, hd)
             q = T(_rope_complex(q, pos, cfg.rope_theta)).transpose(0, 1)[None]
             k = T(_rope_complex(k, pos, cfg.rope_theta)).transpose(0, 1)[None]
-            o = F.scaled_dot_product_attention(q, k, v.transpose(0, 1)[None], is_causal=True,
-                                               enable_gqa=True)
+            if key_alive is None:
+                o = F.scaled_dot_product_attention(q, k, v.transpose(0, 1)[None], is_causal=True,
+                                                   enable_gqa=True)
+            else:
+                allowed = torch.tril(torch.ones(n, n, dtype=torch.bool))
+                allowed &= torch.from_numpy(np.asarray(key_alive[li][b], bool))[None, :]
+                o = F.scaled_dot_product_attention(q, k, v.transpose(0, 1)[None], attn_mask=allowed,
+                                                   enable_gqa=True)
             h = h + F.linear(o[0].transpose(0, 1).reshape(n, H * hd), T(lw["wo"]))
             x = F.rms_norm(h, (d,), weight=T(lw["mlp_norm"]), eps=cfg.rms_eps)
             h = h + F.linear(F.silu(F.linear(x, T(lw["wg"]))) * F.linear(x, T(lw["wu"])), T(lw["wd"]))
         x = F.rms_norm(h, (d,), weight=T(w["final_norm"]), eps=cfg.rms_eps)
         logits = F.linear(x, T(w["head"]))
-        out.append(logits[-1] if cfg.n_classes else logits)
+        out.append(logits[-1] if cfg.n_classes and not all_rows else logits)
     return torch.stack(out).numpy()
 
 
@@ -389,3 +398,88 @@ def test_score_select_norms_and_gather():
         assert np.array_equal(g[b], hid[b][idx[b]])
         order = np.argsort(-s[b], kind="stable")[:7]
         assert sorted(order.tolist()) == idx[b].tolist()
+
+
+# ---------------------------------------------------------------- generation
+
+def test_attention_one_query_is_last_row_of_causal_attention():
+    rng = np.random.default_rng(21)
+    q, k = rng.standard_normal((9, 16)), rng.standard_normal((9, 16))
+    P = O.attention_probs(q, k)
+    np.testing.assert_allclose(O.attention_probs_one(q[-1], k), P[-1], rtol=1e-13, atol=1e-15)
+
+
+def test_decode_unpruned_equals_full_forward_of_longer_sequence():
+    # accel = 1: prefill L tokens, then generate T; every generated token's
+    # logits equal the plain causal decoder's on the L + T sequence.
+    cfg = _cfg(prune_layers=[])
+    w = _tiny_weights(cfg, seed=5)
+    rng = np.random.default_rng(14)
+    L, T = 13, 4
+    seq = rng.integers(0, cfg.vocab, (2, L + T))
+    out = O.generate(cfg, w, seq[:, :L], seq[:, L:], accel=1.0)
+    ref = _torch_forward_unpruned(cfg, w, seq, all_rows=True)
+    np.testing.assert_allclose(out["prefill"]["logits"][:, -1], ref[:, L - 1], rtol=1e-9, atol=1e-9)
+    np.testing.assert_allclose(out["logits"], ref[:, L:], rtol=1e-9, atol=1e-9)
+    assert out["cache"]["layers"][1]["k"].shape == (2, L + T, cfg.n_kv_heads, cfg.head_dim)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_decode_over_pruned_cache_equals_masked_longer_sequence(dtype):
+    # Sec. 3.3 / Appendix B: a row pruned before layer l is a hidden key in
+    # layer l and later.  Generating after a pruned prefill must equal one
+    # causal pass over the L + T tokens with exactly those keys hidden (the
+    # generated tokens are never hidden).
+    cfg = _cfg(dtype=dtype)
+    w = _tiny_weights(cfg, seed=6)
+    rng = np.random.default_rng(15)
+    L, T = 29, 3
+    seq = rng.integers(0, cfg.vocab, (2, L + T))
+    out = O.generate(cfg, w, seq[:, :L], seq[:, L:], alpha=0.55)
+    pre = out["prefill"]
+    assert pre["schedule"][-1] < L // 2
+    alive = []
+    kept = np.tile(np.arange(L), (2, 1))
+    for layer in range(1, cfg.n_layers + 1):
+        a = np.zeros((2, L + T), bool)
+        a[:, L:] = True
+        for b in range(2):
+            a[b, kept[b]] = True
+        alive.append(a)
+        np.testing.assert_array_equal(out["cache"]["layers"][layer]["pos"][:, :-T], kept)
+        if layer in pre["idx"]:
+            kept = np.stack([kept[b][pre["idx"][layer][b]] for b in range(2)])
+    if dtype == "f32":
+        ref = _torch_forward_unpruned(cfg, w, seq, key_alive=alive, all_rows=True)
+        np.testing.assert_allclose(out["logits"], ref[:, L:], rtol=1e-9, atol=1e-9)
+    else:
+        # the torch composition has no bf16 storage points; compare with the
+        # compacted prefill of the L + T tokens in which every layer keeps the
+        # prefix rows the prefill kept plus all generated rows
+        forced, n_in = {}, L
+        for layer in sorted(pre["idx"]):
+            idx = pre["idx"][layer]
+            forced[layer] = np.concatenate([idx, np.tile(np.arange(n_in, n_in + T), (2, 1))], axis=1)
+            n_in = idx.shape[1]
+        full = O.forward(cfg, w, seq, alpha=1.0, forced_idx=forced)
+        np.testing.assert_array_equal(full["kept_pos"][:, -T:], np.tile(np.arange(L, L + T), (2, 1)))
+        assert np.max(np.abs(out["logits"] - full["logits"][:, -T:])) < 2e-2
+    # the cache holds, per layer, exactly the rows that layer ran on, then the generated ones
+    for layer in range(1, cfg.n_layers + 1):
+        pos = out["cache"]["layers"][layer]["pos"]
+        assert pos.shape[1] == pre["schedule"][layer - 1] + T
+        np.testing.assert_array_equal(pos[:, -T:], np.tile(np.arange(L, L + T), (2, 1)))
+        assert np.all(np.diff(pos, axis=1) > 0)
+
+
+def test_decode_cache_keys_are_the_prefill_keys_of_the_kept_rows():
+    # Layer 1 runs on every row; its cached keys must equal layer 1's keys of
+    # an unpruned run on the same prefix (pruning only acts after layer 1).
+    cfg = _cfg()
+    w = _tiny_weights(cfg, seed=7)
+    toks = np.random.default_rng(16).integers(0, cfg.vocab, (2, 21))
+    a = O.forward(cfg, w, toks, alpha=0.5, collect_cache=True)["cache"]["layers"]
+    b = O.forward(_cfg(prune_layers=[]), w, toks, accel=1.0, collect_cache=True)["cache"]["layers"]
+    np.testing.assert_array_equal(a[1]["k"], b[1]["k"])
+    np.testing.assert_array_equal(a[1]["v"], b[1]["v"])
+    assert a[4]["k"].shape[1] < b[4]["k"].shape[1]
