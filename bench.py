@@ -153,6 +153,63 @@ def time_oracle(shape, weights_np, tokens, accel, budget_s, max_seqs):
     return n, time.perf_counter() - t0
 
 
+def decode_leg(zsaa, model, weights, shape, B, L, accel, tok_dev, stream, barrier, max_over_ranks,
+               world, steps=48, warmup=8):
+    """Decode steps after a pruned prefill (CUDA-graph replay, events on the
+    launch stream), the same with an unpruned cache, and the weight-streaming
+    roofline of a step: every weight is read once per step (2.5 GB > L2, no
+    flush needed) plus the cached keys/values the step attends to."""
+    import torch
+    peaks, src = load_peaks()
+    hbm = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+    seen, wbytes = set(), 0
+    for t in [weights["embed"], weights["final_norm"], weights["head"]] + \
+            [v for lw in weights["layers"] for v in lw.values()]:
+        if t.data_ptr() not in seen:
+            seen.add(t.data_ptr())
+            wbytes += t.numel() * t.element_size()
+    wbytes -= weights["embed"].numel() * weights["embed"].element_size() \
+        if weights["embed"].data_ptr() != weights["head"].data_ptr() else 0  # only B embedding rows are read
+    g = torch.Generator(device=tok_dev.device).manual_seed(5)
+    new_tok = torch.randint(0, shape.vocab, (steps + warmup, B), generator=g, device=tok_dev.device,
+                            dtype=torch.int32)
+    out = {}
+    for name, a in (("pruned", accel), ("unpruned", 1.0)):
+        cache = zsaa.Cache(model, B, L, a, steps + warmup)
+        sched, _ = zsaa.zsaa_plan(model, L, a)
+        logits = torch.empty(B, shape.vocab, device=tok_dev.device, dtype=torch.float32)
+        step_tok = torch.empty(B, device=tok_dev.device, dtype=torch.int32)
+        zsaa.zsaa_prefill(model, cache, tok_dev, logits)
+        for t in range(warmup):
+            step_tok.copy_(new_tok[t])
+            zsaa.zsaa_decode_step(model, cache, step_tok, logits, stream=stream)
+        barrier()
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+        for t, (e0, e1) in enumerate(evs):
+            step_tok.copy_(new_tok[warmup + t])
+            e0.record(stream)
+            zsaa.zsaa_decode_step(model, cache, step_tok, logits, stream=stream)
+            e1.record(stream)
+        torch.cuda.synchronize()
+        zsaa.zsaa_sync(model)
+        ms = max_over_ranks(sum(e0.elapsed_time(e1) for e0, e1 in evs) / steps)
+        kv_rows = sum(sched[:-1]) + shape.n_layers * (warmup + steps / 2.0)  # mean rows attended
+        kv_read = 2.0 * B * shape.n_kv_heads * shape.head_dim * 2 * kv_rows
+        nbytes = wbytes + kv_read
+        pruned_b, full_b = zsaa.zsaa_cache_bytes(cache)
+        out[name] = {"accel": a, "ms_per_step": ms, "tokens_per_s": world * B / (ms / 1e3),
+                     "algorithmic_bytes_per_step": nbytes, "gbs": nbytes / (ms * 1e6),
+                     "frac_of_hbm": nbytes / (ms * 1e6) / hbm, "kv_cache_bytes": pruned_b,
+                     "kv_cache_bytes_unpruned": full_b}
+        cache.close()
+    out["workload"] = (f"{steps} timed decode steps (after {warmup}) of B={B} sequences after a "
+                       f"prefill of L={L}; teacher-forced random token ids")
+    out["peak_gbs"] = hbm
+    out["peak_source"] = f"{src} hbm_gbs"
+    out["speedup_vs_unpruned_cache"] = out["unpruned"]["ms_per_step"] / out["pruned"]["ms_per_step"]
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -402,6 +459,11 @@ def main():
                        "d2h_bytes_per_step": n_logit * 4, "ms_per_step": e2e_s * 1e3,
                        "note": "zsaa_forward_host: pinned host tokens in, host float32 logits out; "
                                "the 256 MiB L2 flush runs inside this span"}
+
+        # ---- generation over the pruned KV cache (LM head only): B tokens per step
+        if not shape.n_classes:
+            line["decode"] = decode_leg(zsaa, model, weights, shape, B, L, args.accel, tok_dev, stream,
+                                        barrier, max_over_ranks, world)
 
         # ---- CPU oracle on the host cores (rank 0, N=1 only)
         if rank == 0 and world == 1:

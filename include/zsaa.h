@@ -181,6 +181,60 @@ zsaa_status zsaa_forward_host(zsaa_model* m, const int32_t* token_ids, int B, in
                               double accel, float* logits_out, int32_t* kept_pos_out,
                               zsaa_stream stream);
 
+/* ---- Generation over the pruned KV cache.
+ *
+ * Sec. 3.3 removes an eliminated row from every later layer, so after a pruned
+ * prefill layer l holds the keys and values of only the N_{l-1} rows it ran
+ * on.  A generated token attends, in layer l, to those rows, the tokens
+ * generated before it and itself; generated tokens are never pruned.  The
+ * cache therefore shrinks with depth like the prefill's rows do.
+ *
+ * zsaa_cache_create: a cache for B sequences of L prompt tokens pruned at
+ * acceleration accel (the schedule of zsaa_plan), with room for max_new
+ * generated tokens.  Layer l keeps cap_l = N_{l-1} + max_new rows per sequence
+ * and KV group: K and V bf16 [B, Hkv, cap_l, hd] (keys after RoPE), positions
+ * int32 [B, cap_l].  The cache belongs to the model's device and must not
+ * outlive the model.  bf16 models with the language-model head and
+ * force_keep_last set only (the last prompt position gives the first
+ * generated token), else ZSAA_ERR_UNSUPPORTED.  B <= max_B, L <= max_L of the
+ * model, max_new >= 1. */
+typedef struct zsaa_cache zsaa_cache;
+zsaa_status zsaa_cache_create(zsaa_model* m, int B, int L, double accel, int max_new,
+                              zsaa_cache** out);
+void zsaa_cache_destroy(zsaa_cache* c);
+
+/* zsaa_prefill: the pruned prefill of zsaa_forward on token_ids (device int32
+ * [B, L], the sizes the cache was made for) that also fills the cache, and
+ * resets its generated count to 0.  logits_out: device float32 [B, V], the
+ * logits of the last prompt position of each sequence (the next token).
+ * opts may be NULL; its forced_idx / scores_out / idx_out hooks work as in
+ * zsaa_forward_ex (the other fields must be zero). */
+zsaa_status zsaa_prefill(zsaa_model* m, zsaa_cache* c, const int32_t* token_ids,
+                         float* logits_out, const zsaa_forward_opts* opts, zsaa_stream stream);
+
+/* zsaa_decode_step: one generated token per sequence.  token_ids: device int32
+ * [B], the tokens at position L + t, where t = tokens generated since the
+ * prefill (t < max_new, else ZSAA_ERR_INVALID_ARG; so is a call before the
+ * first zsaa_prefill on the cache); logits_out: device float32
+ * [B, V] for the next position.  Appends each layer's key and value to the
+ * cache.  The position lives in device memory, so the step is recorded as a
+ * CUDA graph on its second call with the same pointers and replayed after
+ * that (zsaa_model_set_graphs controls this too). */
+zsaa_status zsaa_decode_step(zsaa_model* m, zsaa_cache* c, const int32_t* token_ids,
+                             float* logits_out, zsaa_stream stream);
+
+/* zsaa_cache_layer: device pointers and sizes of layer l (1-based): k, v (bf16
+ * [B, Hkv, cap, hd]), pos (int32 [B, cap]); *base = rows from the prefill
+ * (N_{l-1}); *len = rows written so far (base + generated, counting steps
+ * already enqueued).  Any out pointer may be NULL.  The pointers stay valid
+ * for the cache's lifetime. */
+zsaa_status zsaa_cache_layer(const zsaa_cache* c, int layer, void** k, void** v, int32_t** pos,
+                             int* base, int* len, int* cap);
+
+/* zsaa_cache_bytes: device bytes the cache holds for keys and values, and
+ * what an unpruned cache (every layer L + max_new rows) would hold. */
+zsaa_status zsaa_cache_bytes(const zsaa_cache* c, size_t* pruned, size_t* unpruned);
+
 /* Isolated score + select + compaction (Sec. 3.3 with unit column mass and one
  * group, so the score of a row is its L2 norm):
  *   hidden      : device bf16 [B, L, d]
@@ -221,7 +275,10 @@ zsaa_status zsaa_score_select_noalloc(const void* hidden, int B, int L, int d, i
 /* Single steps of the path, for per-kernel checks and timing.  All pointers
  * device; shapes as stated.
  * zsaa_op_linear: out[M,N] = epilogue(A[M,K] W[N,K]^T); dtype ZSAA_BF16 uses
- * the tensor-core GEMM, ZSAA_F32 the fp32 CUDA-core GEMM.  epilogue:
+ * the tcgen05 GEMM (M <= 16 without RoPE: the weight-streaming GEMM), ZSAA_F32
+ * the fp32 CUDA-core GEMM.  The bf16 kernels start reading W before the
+ * previous library kernel on the stream has finished: W and W2 must not be
+ * written by that kernel.  epilogue:
  *   0 store (out has dtype; bf16 rounds once),
  *   1 residual: out = resid + acc (resid may alias out),
  *   2 SwiGLU: out[M,N] = silu(A W^T) * (A W2^T), W and W2 both [N,K],

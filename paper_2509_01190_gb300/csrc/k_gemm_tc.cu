@@ -643,6 +643,9 @@ bool bn_ok(int BN, int epi, const TcWeights& W, const GemmParams& p) {
 cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
                            const GemmParams& p, cudaStream_t s) {
   if (p.K % BK != 0 || p.N % 16 != 0 || lda % 8 != 0) return cudaErrorInvalidValue;
+  // a handful of rows: 128-row tiles would idle most of the tensor core and
+  // most SMs; stream the weights instead
+  if (skinny_supported(A, lda, W, epi, p)) return launch_gemm_skinny(A, lda, W, epi, p, s);
   const int sms = num_sms();
   const int vn = epi == kEpiSwiGLU ? 2 * p.N : p.N;
   const int m_tiles = (p.M + BM - 1) / BM;

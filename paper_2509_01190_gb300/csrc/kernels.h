@@ -79,6 +79,14 @@ struct TcWeights {
 cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
                            const GemmParams& p, cudaStream_t s);
 
+// Weight-streaming bf16 GEMM for M <= kSkinnyMaxM rows (k_skinny.cu): every
+// epilogue but RoPE; N % 16 == 0, K % 32 == 0, lda % 8 == 0, 16-byte aligned
+// A and W.  launch_gemm_tc routes such calls here.
+constexpr int kSkinnyMaxM = 16;
+bool skinny_supported(const void* A, int lda, const TcWeights& W, int epi, const GemmParams& p);
+cudaError_t launch_gemm_skinny(const void* A, int lda, const TcWeights& W, int epi,
+                               const GemmParams& p, cudaStream_t s);
+
 // fp32 CUDA-core GEMM, same epilogues (kEpiRope is applied by launch_rope_f32).
 cudaError_t launch_gemm_f32(const float* A, int lda, const float* W, const float* W2, int epi,
                             const GemmParams& p, cudaStream_t s);
@@ -112,6 +120,29 @@ cudaError_t launch_position_parts(int dtype, const void* qkv, const float* lse, 
 cudaError_t launch_colmass_tc(const void* qkv, const float* lse, const float* vnorm, int B, int N,
                               int Hq, int Hkv, int hd, float* parts, int* status, int* n_chunks,
                               cudaStream_t s);
+
+// ---- generation over the pruned KV cache (k_decode.cu)
+// Cache of one layer: K and V bf16 [B, Hkv, cap, hd], positions int32 [B, cap].
+struct KvLayer {
+  void* k;  // bf16
+  void* v;  // bf16
+  int32_t* pos;
+  int cap;   // rows per (sequence, group)
+  int base;  // rows written by the prefill (N_{l-1})
+};
+// Prefill: copy the keys/values of the N rows per sequence in qkv (bf16,
+// [B*N, ld], RoPE applied) and their positions into rows [0, N) of the cache.
+cudaError_t launch_kv_write(const void* qkv, int ld, const int32_t* pos, int B, int N, int Hq,
+                            int Hkv, int hd, const KvLayer& c, cudaStream_t s);
+// One generated token per sequence: qkv32 [B, ld] float32 projections of the
+// new rows; RoPE at position L0 + *step, bf16 rounding of q/k/v, k/v appended
+// at cache row base + *step, then attention of the Hq queries over rows
+// [0, base + *step]; out [B, Hq*hd] bf16.
+cudaError_t launch_decode_attention(const float* qkv32, int ld, int B, int Hq, int Hkv, int hd,
+                                    const KvLayer& c, const int* step, int L0, const float* cos_t,
+                                    const float* sin_t, void* out, cudaStream_t s);
+// *step += 1 (after every kernel of the decode step).
+cudaError_t launch_decode_advance(int* step, cudaStream_t s);
 
 // ---- thread-local message returned by zsaa_last_error (zsaa_api.cu)
 void set_last_error(const char* msg);

@@ -292,10 +292,34 @@ struct zsaa_model {
     std::string key;
     int seen = 0;                 // eager runs so far with this key
     cudaGraphExec_t exec = nullptr;
+    const void* cache = nullptr;  // zsaa_cache whose buffers the graph uses, if any
   };
   bool use_graphs = true;
   std::list<GraphEntry> graphs;
   cudaStream_t capture_stream = nullptr;  // graphs are recorded here, launched on the caller's
+};
+
+// Pruned KV cache for generation (zsaa_cache_create).
+struct zsaa_cache {
+  zsaa_model* m = nullptr;
+  int B = 0, L = 0, max_new = 0;
+  double accel = 1.0, alpha = 1.0;
+  std::vector<int> sched;                // N_0 .. N_n
+  std::vector<zsaa::KvLayer> layers;     // per layer (0-based)
+  void* kv = nullptr;                    // every layer's K then V
+  int32_t* pos = nullptr;                // every layer's positions
+  size_t kv_bytes = 0, kv_bytes_unpruned = 0;
+  float* rope_cos = nullptr;             // [L + max_new, hd/2]
+  float* rope_sin = nullptr;
+  float* qkv32 = nullptr;                // [B, ld_qkv] float32 projections of the new rows
+  int32_t* last_idx = nullptr;           // [B]: N_n - 1, the last kept row
+  int* step = nullptr;                   // device: tokens generated since the prefill
+  int generated = 0;                     // host: decode steps enqueued since the prefill
+  bool prefilled = false;                // a prefill has been enqueued
+  // CUDA graph of the decode step, keyed by its pointers
+  std::string graph_key;
+  int graph_seen = 0;
+  cudaGraphExec_t graph = nullptr;
 };
 
 namespace {
@@ -379,9 +403,11 @@ zsaa_status linear(zsaa_model* m, const void* A, int lda, const TcWeights& W, in
   return ZSAA_OK;
 }
 
+// With a cache (zsaa_prefill) every layer's keys/values are copied into it and
+// only the last kept row of each sequence goes through the head.
 zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double accel,
                         float* logits, int32_t* kept_pos, const zsaa_forward_opts* opts,
-                        cudaStream_t s) {
+                        cudaStream_t s, zsaa_cache* kc = nullptr) {
   const zsaa_config& c = m->cfg;
   const bool from_hidden = opts && opts->hidden_in;
   if ((!from_hidden && tok == nullptr) || logits == nullptr)
@@ -492,6 +518,10 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
       }
       ZCK(launch_rope_f32(static_cast<float*>(m->qkv), M, m->ld_qkv, m->dq + m->dkv, hd,
                           m->pos[cur], m->rope_cos, m->rope_sin, s));
+    }
+    if (kc != nullptr) {
+      TRACE("kv_write", 0.0, 4.0 * Md * m->dkv * es);
+      ZCK(launch_kv_write(m->qkv, m->ld_qkv, m->pos[cur], B, N, Hq, Hkv, hd, kc->layers[li], s));
     }
     {
       const double pairs = static_cast<double>(B) * Hq * (static_cast<double>(N) * (N + 1) / 2.0);
@@ -611,7 +641,34 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
   const int M = B * N;
   if (opts && opts->hidden_out)
     ZCK(cudaMemcpyAsync(opts->hidden_out, m->h[cur], M * d * m->esz, cudaMemcpyDeviceToDevice, s));
-  if (c.n_classes > 0) {
+  if (kc != nullptr) {  // next-token logits: final norm and LM head of the last kept row
+    if (fuse_norm) {
+      TRACE("gather_norm", 0.0, static_cast<double>(B) * (3.0 * d * es + 12.0));
+      ZCK(launch_rows_norm(m->h[cur], nullptr, 0, 0, kc->last_idx, N, 1, m->pos[cur], B, d,
+                           m->final_norm, c.rms_eps, m->h[cur ^ 1], m->x, m->pos[cur ^ 1],
+                           m->status, s));
+    } else {
+      {
+        TRACE("gather", 0.0, static_cast<double>(B) * (2.0 * d * es + 12.0));
+        ZCK(launch_gather(m->h[cur], B, N, 1, static_cast<int>(d * m->esz), kc->last_idx,
+                          m->h[cur ^ 1], m->pos[cur], m->pos[cur ^ 1], m->status, s));
+      }
+      TRACE("rmsnorm", 0.0, 2.0 * static_cast<double>(B) * d * es);
+      ZCK(launch_rmsnorm(dt, m->h[cur ^ 1], m->final_norm, B, d, c.rms_eps, m->x, s));
+    }
+    GemmParams q{};
+    q.M = B;
+    q.N = c.vocab;
+    q.K = d;
+    q.out = logits;
+    q.ldo = c.vocab;
+    TcWeights W{m->head, nullptr, nullptr, c.vocab, c.vocab};
+    const double V = c.vocab, Mh = B;
+    TRACE("gemm_lm_head", 2.0 * Mh * V * d, (Mh * d + V * d) * es + Mh * V * 4.0);
+    trace_scope_.kernels = 0;
+    st = linear(m, m->x, d, W, kEpiStoreF32, q, s, &trace_scope_.kernels);
+    if (st != ZSAA_OK) return st;
+  } else if (c.n_classes > 0) {
     TRACE("cls_head", 2.0 * B * d * c.n_classes, (static_cast<double>(B) * d + static_cast<double>(c.n_classes) * d) * es);
     ZCK(launch_cls_head(dt, m->h[cur], B, N, d, m->final_norm, c.rms_eps, m->head, c.n_classes,
                         logits, s));
@@ -646,17 +703,18 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
 constexpr size_t kMaxGraphs = 16;
 
 zsaa_status forward_cached(zsaa_model* m, const int32_t* tok, int B, int L, double accel,
-                           float* logits, int32_t* kept_pos, cudaStream_t s) {
+                           float* logits, int32_t* kept_pos, cudaStream_t s,
+                           zsaa_cache* kc = nullptr) {
   if (!m->use_graphs || m->tracing)
-    return run_forward(m, tok, B, L, accel, logits, kept_pos, nullptr, s);
-  char key[160];
-  snprintf(key, sizeof(key), "%p/%d/%d/%.17g/%p/%p", static_cast<const void*>(tok), B, L, accel,
-           static_cast<void*>(logits), static_cast<void*>(kept_pos));
+    return run_forward(m, tok, B, L, accel, logits, kept_pos, nullptr, s, kc);
+  char key[200];
+  snprintf(key, sizeof(key), "%p/%d/%d/%.17g/%p/%p/%p", static_cast<const void*>(tok), B, L, accel,
+           static_cast<void*>(logits), static_cast<void*>(kept_pos), static_cast<void*>(kc));
   auto it = m->graphs.begin();
   for (; it != m->graphs.end(); ++it)
     if (it->key == key) break;
   if (it == m->graphs.end()) {
-    m->graphs.push_front(zsaa_model::GraphEntry{key, 0, nullptr});
+    m->graphs.push_front(zsaa_model::GraphEntry{key, 0, nullptr, kc});
     if (m->graphs.size() > kMaxGraphs) {
       if (m->graphs.back().exec) cudaGraphExecDestroy(m->graphs.back().exec);
       m->graphs.pop_back();
@@ -671,7 +729,7 @@ zsaa_status forward_cached(zsaa_model* m, const int32_t* tok, int B, int L, doub
     return ZSAA_OK;
   }
   if (it->seen == 0) {  // first sight: eager (also sets up kernel attributes)
-    zsaa_status st = run_forward(m, tok, B, L, accel, logits, kept_pos, nullptr, s);
+    zsaa_status st = run_forward(m, tok, B, L, accel, logits, kept_pos, nullptr, s, kc);
     if (st == ZSAA_OK) it->seen = 1;
     return st;
   }
@@ -681,7 +739,7 @@ zsaa_status forward_cached(zsaa_model* m, const int32_t* tok, int B, int L, doub
     ZCK(cudaStreamCreateWithFlags(&m->capture_stream, cudaStreamNonBlocking));
   cudaGraph_t graph = nullptr;
   ZCK(cudaStreamBeginCapture(m->capture_stream, cudaStreamCaptureModeThreadLocal));
-  zsaa_status st = run_forward(m, tok, B, L, accel, logits, kept_pos, nullptr, m->capture_stream);
+  zsaa_status st = run_forward(m, tok, B, L, accel, logits, kept_pos, nullptr, m->capture_stream, kc);
   cudaError_t e = cudaStreamEndCapture(m->capture_stream, &graph);
   if (st != ZSAA_OK) {
     if (graph) cudaGraphDestroy(graph);
@@ -749,6 +807,185 @@ zsaa_status read_status(int* word, cudaStream_t s, bool whole_device) {
       return fail(ZSAA_ERR_TIMEOUT, "a kernel gave up a bounded wait (status 0x%x)", v);
     return fail(ZSAA_ERR_INVALID_ARG, "a token id or forced index was out of range (status 0x%x)", v);
   }
+  return ZSAA_OK;
+}
+
+// cos/sin of RoPE for positions [0, n_pos): angle(p, i) = p * theta^(-2i/hd), in double.
+void rope_host_table(double theta, int hd, int n_pos, std::vector<float>* cs, std::vector<float>* sn) {
+  const int half = hd / 2;
+  cs->assign(static_cast<size_t>(n_pos) * half, 0.f);
+  sn->assign(cs->size(), 0.f);
+  for (int p = 0; p < n_pos; ++p)
+    for (int i = 0; i < half; ++i) {
+      const double a = static_cast<double>(p) *
+                       std::pow(theta, -2.0 * static_cast<double>(i) / static_cast<double>(hd));
+      (*cs)[static_cast<size_t>(p) * half + i] = static_cast<float>(std::cos(a));
+      (*sn)[static_cast<size_t>(p) * half + i] = static_cast<float>(std::sin(a));
+    }
+}
+
+void free_cache(zsaa_cache* c) {
+  if (c == nullptr) return;
+  if (c->graph) cudaGraphExecDestroy(c->graph);
+  void* ptrs[] = {c->kv, c->pos, c->rope_cos, c->rope_sin, c->qkv32, c->last_idx, c->step};
+  for (void* p : ptrs)
+    if (p) cudaFree(p);
+  delete c;
+}
+
+// One generated token per sequence (B rows through every layer, attention over
+// the pruned cache), then the next-token logits; the step counter advances last.
+zsaa_status run_decode(zsaa_model* m, zsaa_cache* kc, const int32_t* tok, float* logits,
+                       cudaStream_t s) {
+  const zsaa_config& c = m->cfg;
+  const int B = kc->B, d = c.d_model, hd = c.head_dim, Hq = c.n_heads, Hkv = c.n_kv_heads;
+  const double es = static_cast<double>(m->esz), Bd = B;
+  void* h = m->h[0];
+  zsaa_status st = ZSAA_OK;
+#define TRACE(name, fl, by) TraceScope trace_scope_(m, name, fl, by, s)
+  {
+    TRACE("embed_norm", 0.0, Bd * (3.0 * d * es + 8.0));
+    ZCK(launch_rows_norm(m->embed, tok, c.vocab, 1, nullptr, 0, 0, nullptr, B, d,
+                         LW(m, 0, kAttnNorm), c.rms_eps, h, m->x, m->pos[0], m->status, s));
+  }
+  for (int li = 0; li < c.n_layers; ++li) {
+    if (li > 0) {
+      TRACE("rmsnorm", 0.0, 2.0 * Bd * d * es);
+      ZCK(launch_rmsnorm(c.dtype, h, LW(m, li, kAttnNorm), B, d, c.rms_eps, m->x, s));
+    }
+    {
+      GemmParams p{};
+      p.M = B;
+      p.N = m->ld_qkv;
+      p.K = d;
+      p.out = kc->qkv32;
+      p.ldo = m->ld_qkv;
+      TcWeights W{LW(m, li, kWq), LW(m, li, kWk), LW(m, li, kWv), m->dq, m->dq + m->dkv};
+      TRACE("gemm_qkv", 2.0 * Bd * m->ld_qkv * d, (Bd * d + static_cast<double>(m->ld_qkv) * d) * es + Bd * m->ld_qkv * 4.0);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->x, d, W, kEpiStoreF32, p, s, &trace_scope_.kernels);
+      if (st != ZSAA_OK) return st;
+    }
+    {
+      const zsaa::KvLayer& L = kc->layers[li];
+      const double keys = static_cast<double>(L.base) + kc->generated + 1;
+      TRACE("decode_attention", 4.0 * Bd * Hq * hd * keys, 2.0 * Bd * Hkv * hd * keys * es + Bd * m->ld_qkv * 4.0);
+      ZCK(launch_decode_attention(kc->qkv32, m->ld_qkv, B, Hq, Hkv, hd, L, kc->step, kc->L,
+                                  kc->rope_cos, kc->rope_sin, m->attn, s));
+    }
+    {
+      GemmParams q{};
+      q.M = B;
+      q.N = d;
+      q.K = m->dq;
+      q.out = h;
+      q.ldo = d;
+      q.resid = h;
+      TcWeights W{LW(m, li, kWo), nullptr, nullptr, d, d};
+      TRACE("gemm_o_resid", 2.0 * Bd * d * m->dq, (Bd * m->dq + static_cast<double>(d) * m->dq + 2.0 * Bd * d) * es);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->attn, m->dq, W, kEpiResid, q, s, &trace_scope_.kernels);
+      if (st != ZSAA_OK) return st;
+    }
+    {
+      TRACE("rmsnorm", 0.0, 2.0 * Bd * d * es);
+      ZCK(launch_rmsnorm(c.dtype, h, LW(m, li, kMlpNorm), B, d, c.rms_eps, m->x, s));
+    }
+    const double F = c.ffn_dim;
+    {
+      GemmParams q{};
+      q.M = B;
+      q.N = c.ffn_dim;
+      q.K = d;
+      q.out = m->act;
+      q.ldo = c.ffn_dim;
+      TcWeights W{LW(m, li, kWg), LW(m, li, kWu), nullptr, c.ffn_dim, c.ffn_dim};
+      TRACE("gemm_gate_up_swiglu", 4.0 * Bd * F * d, (Bd * d + 2.0 * F * d + Bd * F) * es);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->x, d, W, kEpiSwiGLU, q, s, &trace_scope_.kernels);
+      if (st != ZSAA_OK) return st;
+    }
+    {
+      GemmParams q{};
+      q.M = B;
+      q.N = d;
+      q.K = c.ffn_dim;
+      q.out = h;
+      q.ldo = d;
+      q.resid = h;
+      TcWeights W{LW(m, li, kWd), nullptr, nullptr, d, d};
+      TRACE("gemm_down_resid", 2.0 * Bd * d * F, (Bd * F + F * d + 2.0 * Bd * d) * es);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->act, c.ffn_dim, W, kEpiResid, q, s, &trace_scope_.kernels);
+      if (st != ZSAA_OK) return st;
+    }
+  }
+  {
+    TRACE("rmsnorm", 0.0, 2.0 * Bd * d * es);
+    ZCK(launch_rmsnorm(c.dtype, h, m->final_norm, B, d, c.rms_eps, m->x, s));
+  }
+  {
+    GemmParams q{};
+    q.M = B;
+    q.N = c.vocab;
+    q.K = d;
+    q.out = logits;
+    q.ldo = c.vocab;
+    TcWeights W{m->head, nullptr, nullptr, c.vocab, c.vocab};
+    const double V = c.vocab;
+    TRACE("gemm_lm_head", 2.0 * Bd * V * d, (Bd * d + V * d) * es + Bd * V * 4.0);
+    trace_scope_.kernels = 0;
+    st = linear(m, m->x, d, W, kEpiStoreF32, q, s, &trace_scope_.kernels);
+    if (st != ZSAA_OK) return st;
+  }
+  {
+    TRACE("advance", 0.0, 8.0);
+    ZCK(launch_decode_advance(kc->step, s));
+  }
+#undef TRACE
+  return ZSAA_OK;
+}
+
+// The decode step reads its position from device memory, so one graph serves
+// every step: the first call with given pointers runs eagerly, the second is
+// recorded, later ones launch the recording.
+zsaa_status decode_cached(zsaa_model* m, zsaa_cache* kc, const int32_t* tok, float* logits,
+                          cudaStream_t s) {
+  if (!m->use_graphs || m->tracing) return run_decode(m, kc, tok, logits, s);
+  char key[96];
+  snprintf(key, sizeof(key), "%p/%p", static_cast<const void*>(tok), static_cast<void*>(logits));
+  if (kc->graph_key != key) {
+    if (kc->graph) cudaGraphExecDestroy(kc->graph);
+    kc->graph = nullptr;
+    kc->graph_key = key;
+    kc->graph_seen = 0;
+  }
+  if (kc->graph) {
+    ZCK(cudaGraphLaunch(kc->graph, s));
+    return ZSAA_OK;
+  }
+  if (kc->graph_seen == 0) {
+    zsaa_status st = run_decode(m, kc, tok, logits, s);
+    if (st == ZSAA_OK) kc->graph_seen = 1;
+    return st;
+  }
+  if (m->capture_stream == nullptr)
+    ZCK(cudaStreamCreateWithFlags(&m->capture_stream, cudaStreamNonBlocking));
+  cudaGraph_t graph = nullptr;
+  ZCK(cudaStreamBeginCapture(m->capture_stream, cudaStreamCaptureModeThreadLocal));
+  zsaa_status st = run_decode(m, kc, tok, logits, m->capture_stream);
+  cudaError_t e = cudaStreamEndCapture(m->capture_stream, &graph);
+  if (st != ZSAA_OK) {
+    if (graph) cudaGraphDestroy(graph);
+    return st;
+  }
+  ZCK(e);
+  cudaGraphExec_t exec = nullptr;
+  e = cudaGraphInstantiate(&exec, graph, 0);
+  cudaGraphDestroy(graph);
+  ZCK(e);
+  kc->graph = exec;
+  ZCK(cudaGraphLaunch(exec, s));
   return ZSAA_OK;
 }
 
@@ -1048,6 +1285,160 @@ zsaa_status zsaa_trace_end(zsaa_model* m, zsaa_trace_row* rows, int max_rows, in
   for (int i = 0; i < n && i < max_rows && rows != nullptr; ++i) rows[i] = agg[i];
   m->trace.clear();
   m->ev_used = 0;
+  return ZSAA_OK;
+}
+
+zsaa_status zsaa_cache_create(zsaa_model* m, int B, int L, double accel, int max_new,
+                              zsaa_cache** out) {
+  if (out == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null out");
+  *out = nullptr;
+  if (m == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null model");
+  const zsaa_config& c = m->cfg;
+  if (c.dtype != ZSAA_BF16 || c.n_classes != 0 || !c.force_keep_last)
+    return fail(ZSAA_ERR_UNSUPPORTED, "generation needs a bf16 model with the LM head and force_keep_last");
+  if (B < 1 || B > m->max_B || L < 1 || L > m->max_L)
+    return fail(ZSAA_ERR_INVALID_ARG, "B=%d L=%d outside [1,%d] x [1,%d]", B, L, m->max_B, m->max_L);
+  if (max_new < 1 || max_new > (1 << 20))
+    return fail(ZSAA_ERR_INVALID_ARG, "max_new=%d outside [1, 2^20]", max_new);
+  if (c.n_heads % c.n_kv_heads != 0 || (c.n_heads / c.n_kv_heads) > 8 ||
+      ((c.n_heads / c.n_kv_heads) & (c.n_heads / c.n_kv_heads - 1)) != 0 ||
+      (c.head_dim != 64 && c.head_dim != 128))
+    return fail(ZSAA_ERR_UNSUPPORTED, "generation supports head_dim 64/128 and 1/2/4/8 query heads per KV head");
+  std::vector<int> sched(c.n_layers + 1);
+  double alpha = 1.0;
+  zsaa_status st = plan_impl(c, L, accel, sched.data(), &alpha);
+  if (st != ZSAA_OK) return st;
+  zsaa_cache* kc = new zsaa_cache();
+  kc->m = m;
+  kc->B = B;
+  kc->L = L;
+  kc->max_new = max_new;
+  kc->accel = accel;
+  kc->alpha = alpha;
+  kc->sched = sched;
+  const int Hkv = c.n_kv_heads, hd = c.head_dim;
+  size_t kv_elems = 0, pos_elems = 0;
+  for (int l = 1; l <= c.n_layers; ++l) {
+    const size_t cap = static_cast<size_t>(sched[l - 1]) + max_new;
+    kv_elems += 2 * static_cast<size_t>(B) * Hkv * cap * hd;
+    pos_elems += static_cast<size_t>(B) * cap;
+  }
+  kc->kv_bytes = kv_elems * 2;
+  kc->kv_bytes_unpruned = static_cast<size_t>(c.n_layers) * 2 * B * Hkv * (static_cast<size_t>(L) + max_new) * hd * 2;
+  bool ok = true;
+  auto alloc = [&](void** p, size_t bytes) {
+    if (ok && cudaMalloc(p, bytes + 16) != cudaSuccess) ok = false;
+  };
+  const int n_pos = L + max_new;
+  alloc(&kc->kv, kv_elems * 2);
+  alloc(reinterpret_cast<void**>(&kc->pos), pos_elems * sizeof(int32_t));
+  alloc(reinterpret_cast<void**>(&kc->rope_cos), static_cast<size_t>(n_pos) * (hd / 2) * sizeof(float));
+  alloc(reinterpret_cast<void**>(&kc->rope_sin), static_cast<size_t>(n_pos) * (hd / 2) * sizeof(float));
+  alloc(reinterpret_cast<void**>(&kc->qkv32), static_cast<size_t>(B) * m->ld_qkv * sizeof(float));
+  alloc(reinterpret_cast<void**>(&kc->last_idx), static_cast<size_t>(B) * sizeof(int32_t));
+  alloc(reinterpret_cast<void**>(&kc->step), sizeof(int));
+  if (!ok) {
+    cudaGetLastError();
+    const size_t want = kc->kv_bytes;
+    free_cache(kc);
+    return fail(ZSAA_ERR_OOM, "cache allocation failed (%zu bytes of keys/values)", want);
+  }
+  size_t off_kv = 0, off_pos = 0;
+  for (int l = 1; l <= c.n_layers; ++l) {
+    const int cap = sched[l - 1] + max_new;
+    const size_t plane = static_cast<size_t>(B) * Hkv * cap * hd;
+    zsaa::KvLayer kl;
+    kl.k = static_cast<uint16_t*>(kc->kv) + off_kv;
+    kl.v = static_cast<uint16_t*>(kc->kv) + off_kv + plane;
+    kl.pos = kc->pos + off_pos;
+    kl.cap = cap;
+    kl.base = sched[l - 1];
+    kc->layers.push_back(kl);
+    off_kv += 2 * plane;
+    off_pos += static_cast<size_t>(B) * cap;
+  }
+  std::vector<float> cs, sn;
+  rope_host_table(c.rope_theta, hd, n_pos, &cs, &sn);
+  std::vector<int32_t> last(B, sched[c.n_layers] - 1);
+  cudaError_t e = cudaMemcpy(kc->rope_cos, cs.data(), cs.size() * sizeof(float), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemcpy(kc->rope_sin, sn.data(), sn.size() * sizeof(float), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemcpy(kc->last_idx, last.data(), last.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemset(kc->step, 0, sizeof(int));
+  if (e != cudaSuccess) {
+    free_cache(kc);
+    return fail(ZSAA_ERR_CUDA, "cache initialisation failed: %s", cudaGetErrorString(e));
+  }
+  *out = kc;
+  return ZSAA_OK;
+}
+
+void zsaa_cache_destroy(zsaa_cache* c) {
+  if (c == nullptr) return;
+  cudaDeviceSynchronize();
+  zsaa_model* m = c->m;
+  for (auto it = m->graphs.begin(); it != m->graphs.end();) {  // graphs that use this cache
+    if (it->cache == c) {
+      if (it->exec) cudaGraphExecDestroy(it->exec);
+      it = m->graphs.erase(it);
+    } else {
+      ++it;
+    }
+  }
+  free_cache(c);
+}
+
+zsaa_status zsaa_prefill(zsaa_model* m, zsaa_cache* c, const int32_t* token_ids,
+                         float* logits_out, const zsaa_forward_opts* opts, zsaa_stream stream) {
+  if (m == nullptr || c == nullptr || c->m != m) return fail(ZSAA_ERR_INVALID_ARG, "null model/cache or cache of another model");
+  if (token_ids == nullptr || logits_out == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null token or logits pointer");
+  if (opts && (opts->hidden_out || opts->n_layers_run || opts->hidden_in || opts->pos_in ||
+               opts->first_layer || opts->plan_L))
+    return fail(ZSAA_ERR_INVALID_ARG, "zsaa_prefill takes only the forced_idx/scores_out/idx_out hooks");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  ZCK(cudaMemsetAsync(c->step, 0, sizeof(int), s));
+  zsaa_status st;
+  if (opts && (opts->forced_idx || opts->scores_out || opts->idx_out))
+    st = run_forward(m, token_ids, c->B, c->L, c->accel, logits_out, nullptr, opts, s, c);
+  else
+    st = forward_cached(m, token_ids, c->B, c->L, c->accel, logits_out, nullptr, s, c);
+  if (st == ZSAA_OK) {
+    c->generated = 0;
+    c->prefilled = true;
+  }
+  return st;
+}
+
+zsaa_status zsaa_decode_step(zsaa_model* m, zsaa_cache* c, const int32_t* token_ids,
+                             float* logits_out, zsaa_stream stream) {
+  if (m == nullptr || c == nullptr || c->m != m) return fail(ZSAA_ERR_INVALID_ARG, "null model/cache or cache of another model");
+  if (token_ids == nullptr || logits_out == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null token or logits pointer");
+  if (!c->prefilled) return fail(ZSAA_ERR_INVALID_ARG, "zsaa_decode_step before zsaa_prefill");
+  if (c->generated >= c->max_new)
+    return fail(ZSAA_ERR_INVALID_ARG, "cache full: %d tokens generated, max_new %d", c->generated, c->max_new);
+  zsaa_status st = decode_cached(m, c, token_ids, logits_out, reinterpret_cast<cudaStream_t>(stream));
+  if (st == ZSAA_OK) c->generated += 1;
+  return st;
+}
+
+zsaa_status zsaa_cache_layer(const zsaa_cache* c, int layer, void** k, void** v, int32_t** pos,
+                             int* base, int* len, int* cap) {
+  if (c == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null cache");
+  if (layer < 1 || layer > static_cast<int>(c->layers.size()))
+    return fail(ZSAA_ERR_INVALID_ARG, "layer %d outside [1, %zu]", layer, c->layers.size());
+  const zsaa::KvLayer& l = c->layers[layer - 1];
+  if (k) *k = l.k;
+  if (v) *v = l.v;
+  if (pos) *pos = l.pos;
+  if (base) *base = l.base;
+  if (len) *len = l.base + c->generated;
+  if (cap) *cap = l.cap;
+  return ZSAA_OK;
+}
+
+zsaa_status zsaa_cache_bytes(const zsaa_cache* c, size_t* pruned, size_t* unpruned) {
+  if (c == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null cache");
+  if (pruned) *pruned = c->kv_bytes;
+  if (unpruned) *unpruned = c->kv_bytes_unpruned;
   return ZSAA_OK;
 }
 

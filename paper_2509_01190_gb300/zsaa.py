@@ -27,7 +27,8 @@ EXPORTED = [
     "zsaa_forward_ex", "zsaa_forward_host", "zsaa_score_select", "zsaa_score_select_ex",
     "zsaa_op_linear", "zsaa_op_attention", "zsaa_op_colmass", "zsaa_sync", "zsaa_device_status",
     "zsaa_last_error", "zsaa_version", "zsaa_trace_begin", "zsaa_trace_end",
-    "zsaa_score_select_noalloc", "zsaa_model_set_graphs",
+    "zsaa_score_select_noalloc", "zsaa_model_set_graphs", "zsaa_cache_create", "zsaa_cache_destroy",
+    "zsaa_prefill", "zsaa_decode_step", "zsaa_cache_layer", "zsaa_cache_bytes",
 ]
 
 
@@ -98,6 +99,13 @@ def lib():
             "zsaa_version": ([], C.c_char_p),
             "zsaa_trace_begin": ([_P], _I),
             "zsaa_trace_end": ([_P, C.POINTER(zsaa_trace_row), _I, C.POINTER(_I)], _I),
+            "zsaa_cache_create": ([_P, _I, _I, _D, _I, C.POINTER(_P)], _I),
+            "zsaa_cache_destroy": ([_P], None),
+            "zsaa_prefill": ([_P, _P, _P, _P, C.POINTER(zsaa_forward_opts), _P], _I),
+            "zsaa_decode_step": ([_P, _P, _P, _P, _P], _I),
+            "zsaa_cache_layer": ([_P, _I, C.POINTER(_P), C.POINTER(_P), C.POINTER(_P), C.POINTER(_I),
+                                  C.POINTER(_I), C.POINTER(_I)], _I),
+            "zsaa_cache_bytes": ([_P, C.POINTER(C.c_size_t), C.POINTER(C.c_size_t)], _I),
         }
         for name, (args, res) in sig.items():
             f = getattr(L, name)
@@ -251,6 +259,68 @@ def zsaa_forward_host(model: Model, token_ids, B: int, L: int, accel: float, log
 
     _check(lib().zsaa_forward_host(model.handle, hp(token_ids), B, L, float(accel), hp(logits_out),
                                    hp(kept_pos_out), _stream(stream)))
+
+
+# ------------------------------------------------------------------ generation
+
+class Cache:
+    """Owns a zsaa_cache handle (pruned KV cache of one prompt batch)."""
+
+    def __init__(self, model: Model, B: int, L: int, accel: float, max_new: int):
+        h = C.c_void_p()
+        _check(lib().zsaa_cache_create(model.handle, B, L, float(accel), max_new, C.byref(h)))
+        self.handle = h
+        self.model = model  # the cache must not outlive its model
+        self.B, self.L, self.accel, self.max_new = B, L, accel, max_new
+
+    def close(self):
+        if getattr(self, "handle", None) is not None and self.handle.value:
+            lib().zsaa_cache_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def zsaa_cache_create(model: Model, B: int, L: int, accel: float, max_new: int) -> Cache:
+    return Cache(model, B, L, accel, max_new)
+
+
+def zsaa_cache_destroy(cache: Cache):
+    cache.close()
+
+
+def zsaa_prefill(model: Model, cache: Cache, token_ids, logits_out, forced_idx=None,
+                 scores_out=None, idx_out=None, stream=None):
+    opts = None
+    if forced_idx is not None or scores_out is not None or idx_out is not None:
+        opts = C.byref(zsaa_forward_opts(_ptr(forced_idx), _ptr(scores_out), _ptr(idx_out), None,
+                                         0, None, None, 0, 0))
+    _check(lib().zsaa_prefill(model.handle, cache.handle, _ptr(token_ids), _ptr(logits_out), opts,
+                              _stream(stream)))
+
+
+def zsaa_decode_step(model: Model, cache: Cache, token_ids, logits_out, stream=None):
+    _check(lib().zsaa_decode_step(model.handle, cache.handle, _ptr(token_ids), _ptr(logits_out),
+                                  _stream(stream)))
+
+
+def zsaa_cache_layer(cache: Cache, layer: int) -> Dict:
+    """Device pointers (ints) k, v, pos and the sizes base, len, cap of one layer (1-based)."""
+    k, v, pos = C.c_void_p(), C.c_void_p(), C.c_void_p()
+    base, ln, cap = C.c_int(), C.c_int(), C.c_int()
+    _check(lib().zsaa_cache_layer(cache.handle, layer, C.byref(k), C.byref(v), C.byref(pos),
+                                  C.byref(base), C.byref(ln), C.byref(cap)))
+    return dict(k=k.value, v=v.value, pos=pos.value, base=base.value, len=ln.value, cap=cap.value)
+
+
+def zsaa_cache_bytes(cache: Cache) -> Tuple[int, int]:
+    a, b = C.c_size_t(), C.c_size_t()
+    _check(lib().zsaa_cache_bytes(cache.handle, C.byref(a), C.byref(b)))
+    return a.value, b.value
 
 
 def zsaa_trace_begin(model: Model):

@@ -104,3 +104,17 @@ def test_bad_arguments_rejected_without_device_work(zlib):
     assert e.value.status == zlib.ZSAA_ERR_INVALID_ARG
     with pytest.raises(zlib.ZsaaError):
         zlib.zsaa_op_linear(None, fake, None, None, fake, 4, 16, 64, zlib.ZSAA_BF16, 0, stream=0)
+
+
+def test_generation_entry_points_reject_null_handles(zlib):
+    import ctypes as C
+    L = zlib.lib()
+    h = C.c_void_p()
+    assert L.zsaa_cache_create(None, 1, 16, 2.0, 4, C.byref(h)) == zlib.ZSAA_ERR_INVALID_ARG
+    assert h.value is None
+    assert L.zsaa_cache_create(None, 1, 16, 2.0, 4, None) == zlib.ZSAA_ERR_INVALID_ARG
+    assert L.zsaa_prefill(None, None, None, None, None, None) == zlib.ZSAA_ERR_INVALID_ARG
+    assert L.zsaa_decode_step(None, None, None, None, None) == zlib.ZSAA_ERR_INVALID_ARG
+    assert L.zsaa_cache_layer(None, 1, None, None, None, None, None, None) == zlib.ZSAA_ERR_INVALID_ARG
+    assert L.zsaa_cache_bytes(None, None, None) == zlib.ZSAA_ERR_INVALID_ARG
+    L.zsaa_cache_destroy(None)  # no-op
