@@ -31,7 +31,9 @@ Readings of points the paper leaves open (each is listed in the design notes):
   ("softscore_vnorm"); ``"softscore"`` drops the norm factor.
 * R2 unnormalised column sums (no division by the number of queries).
 * R3 pruning happens after the whole layer: layer l scores its own rows and its
-  output rows are compacted; layer l+1 runs on the kept rows.
+  output rows are compacted; layer l+1 runs on the kept rows.  With
+  ``prune_point="attention"`` the compaction happens between attention and
+  MLP instead; the kept rows are the same (the MLP acts on each row alone).
 * R5 acceleration -> alpha: bisection on the modelled per-sequence FLOPs.
 * R6 ``N_l = min(N_{l-1}, max(floor(alpha N_{l-1}), min(tau, N_{l-1})))``.
 * R7 ties by lower index; NaN scores rank lowest.
@@ -73,6 +75,9 @@ class OracleConfig:
     force_keep_last: bool = True
     score_mode: str = "softscore_vnorm"  # or "softscore"
     plan_mode: str = "cost"  # "cost" (R5 bisection) or "rate" (alpha = 1/accel)
+    # where a pruning layer compacts its rows: "layer" (after the MLP, R3) or
+    # "attention" (between attention and MLP; the MLP then runs on kept rows only)
+    prune_point: str = "layer"
 
 
 # --------------------------------------------------------------------------
@@ -389,7 +394,10 @@ def forward(cfg: OracleConfig, weights, tokens: np.ndarray, accel: Optional[floa
             h, P, v = attention_block(cfg, lw, h, pos, store, kv_out=kv)
             if collect_cache:
                 cache_all.setdefault(layer, []).append((kv[0][0], kv[0][1], pos))
-            h = mlp_block(cfg, lw, h, store)
+            if cfg.prune_point not in ("layer", "attention"):
+                raise ValueError(cfg.prune_point)
+            if cfg.prune_point == "layer":
+                h = mlp_block(cfg, lw, h, store)
             k_keep = sched[layer]
             if layer in set(cfg.prune_layers):
                 C = column_mass(P, cfg.n_kv_heads)
@@ -404,6 +412,8 @@ def forward(cfg: OracleConfig, weights, tokens: np.ndarray, accel: Optional[floa
                 scores_all.setdefault(layer, []).append(s)
                 h = h[idx]
                 pos = pos[idx]
+            if cfg.prune_point == "attention":
+                h = mlp_block(cfg, lw, h, store)
         logits.append(head(cfg, weights, h, store))
         kept_pos.append(pos)
         finals.append(h)

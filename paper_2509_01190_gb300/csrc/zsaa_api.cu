@@ -3,9 +3,11 @@
 //
 // Forward pass of one call (Sec. 3.3): embed -> for each layer l on N_{l-1}
 // rows: RMSNorm, QKV GEMM with RoPE at original positions, causal GQA
-// attention, O GEMM + residual, RMSNorm, gate/up GEMM with SwiGLU, down GEMM
-// + residual; if layer l prunes and N_l < N_{l-1}: column mass, scores, top-k,
-// gather of the residual rows and their positions -> final RMSNorm + head.
+// attention, O GEMM + residual; if layer l prunes and N_l < N_{l-1}: column
+// mass, scores, top-k, gather of the residual rows and their positions; then
+// RMSNorm, gate/up GEMM with SwiGLU, down GEMM + residual on the N_l kept rows
+// (the MLP is row-wise, so compacting before it changes no kept row) -> final
+// RMSNorm + head.
 // The schedule is computed on the host before any launch; there is no
 // host/device synchronisation inside a forward.
 #include <cmath>
@@ -542,41 +544,11 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
       st = linear(m, m->attn, m->dq, W, kEpiResid, q, s, &trace_scope_.kernels);
       if (st != ZSAA_OK) return st;
     }
-    // MLP branch
-    {
-      TRACE("rmsnorm", 0.0, 2.0 * Md * d * es);
-      ZCK(launch_rmsnorm(dt, h, LW(m, li, kMlpNorm), M, d, c.rms_eps, m->x, s));
-    }
-    {
-      GemmParams q{};
-      q.M = M;
-      q.N = c.ffn_dim;
-      q.K = d;
-      q.out = m->act;
-      q.ldo = c.ffn_dim;
-      TcWeights W{LW(m, li, kWg), LW(m, li, kWu), nullptr, c.ffn_dim, c.ffn_dim};
-      const double F = c.ffn_dim;
-      TRACE("gemm_gate_up_swiglu", 4.0 * Md * F * d, (Md * d + 2.0 * F * d + Md * F) * es);
-      trace_scope_.kernels = 0;
-      st = linear(m, m->x, d, W, kEpiSwiGLU, q, s, &trace_scope_.kernels);
-      if (st != ZSAA_OK) return st;
-    }
-    {
-      GemmParams q{};
-      q.M = M;
-      q.N = d;
-      q.K = c.ffn_dim;
-      q.out = h;
-      q.ldo = d;
-      q.resid = h;
-      TcWeights W{LW(m, li, kWd), nullptr, nullptr, d, d};
-      const double F = c.ffn_dim;
-      TRACE("gemm_down_resid", 2.0 * Md * d * F, (Md * F + F * d + 2.0 * Md * d) * es);
-      trace_scope_.kernels = 0;
-      st = linear(m, m->act, c.ffn_dim, W, kEpiResid, q, s, &trace_scope_.kernels);
-      if (st != ZSAA_OK) return st;
-    }
-    // elimination after the layer (Sec. 3.3)
+    // Elimination (Sec. 3.3), between attention and MLP: the scores come from
+    // this layer's attention and the MLP acts on each row alone, so the kept
+    // rows come out exactly as if the whole layer ran first -- but the MLP
+    // only runs on the kept rows.
+    bool mlp_x_ready = false;
     if (prunes(c, l)) {
       const int k = sched[l];
       const bool want_scores = opts && opts->scores_out;
@@ -617,12 +589,12 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
           ZCK(cudaMemcpyAsync(opts->idx_out + off_idx, idx, sizeof(int32_t) * B * k,
                               cudaMemcpyDeviceToDevice, s));
         if (k < N) {
-          if (fuse_norm && l < n_run) {
+          if (fuse_norm) {  // the kept rows and their pre-MLP RMSNorm in one pass
             TRACE("gather_norm", 0.0, static_cast<double>(B) * k * (3.0 * d * es + 12.0));
             ZCK(launch_rows_norm(h, nullptr, 0, 0, idx, N, k, m->pos[cur], B * k, d,
-                                 LW(m, l, kAttnNorm), c.rms_eps, m->h[cur ^ 1], m->x,
+                                 LW(m, li, kMlpNorm), c.rms_eps, m->h[cur ^ 1], m->x,
                                  m->pos[cur ^ 1], m->status, s));
-            x_ready = true;
+            mlp_x_ready = true;
           } else {
             TRACE("gather", 0.0, static_cast<double>(B) * k * (2.0 * d * es + 12.0));
             ZCK(launch_gather(h, B, N, k, static_cast<int>(d * m->esz), idx, m->h[cur ^ 1],
@@ -636,6 +608,44 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
       off_scores += static_cast<size_t>(B) * N;
       N = k;
     }
+    // MLP branch on the rows left after the elimination
+    const int Mm = B * N;
+    const double Mmd = static_cast<double>(Mm);
+    void* hm = m->h[cur];
+    if (!mlp_x_ready) {
+      TRACE("rmsnorm", 0.0, 2.0 * Mmd * d * es);
+      ZCK(launch_rmsnorm(dt, hm, LW(m, li, kMlpNorm), Mm, d, c.rms_eps, m->x, s));
+    }
+    {
+      GemmParams q{};
+      q.M = Mm;
+      q.N = c.ffn_dim;
+      q.K = d;
+      q.out = m->act;
+      q.ldo = c.ffn_dim;
+      TcWeights W{LW(m, li, kWg), LW(m, li, kWu), nullptr, c.ffn_dim, c.ffn_dim};
+      const double F = c.ffn_dim;
+      TRACE("gemm_gate_up_swiglu", 4.0 * Mmd * F * d, (Mmd * d + 2.0 * F * d + Mmd * F) * es);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->x, d, W, kEpiSwiGLU, q, s, &trace_scope_.kernels);
+      if (st != ZSAA_OK) return st;
+    }
+    {
+      GemmParams q{};
+      q.M = Mm;
+      q.N = d;
+      q.K = c.ffn_dim;
+      q.out = hm;
+      q.ldo = d;
+      q.resid = hm;
+      TcWeights W{LW(m, li, kWd), nullptr, nullptr, d, d};
+      const double F = c.ffn_dim;
+      TRACE("gemm_down_resid", 2.0 * Mmd * d * F, (Mmd * F + F * d + 2.0 * Mmd * d) * es);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->act, c.ffn_dim, W, kEpiResid, q, s, &trace_scope_.kernels);
+      if (st != ZSAA_OK) return st;
+    }
+    x_ready = false;  // the next layer normalises its own input
   }
   // head
   const int M = B * N;

@@ -483,3 +483,26 @@ def test_decode_cache_keys_are_the_prefill_keys_of_the_kept_rows():
     np.testing.assert_array_equal(a[1]["k"], b[1]["k"])
     np.testing.assert_array_equal(a[1]["v"], b[1]["v"])
     assert a[4]["k"].shape[1] < b[4]["k"].shape[1]
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_pruning_between_attention_and_mlp_gives_the_same_rows(dtype):
+    # The scores come from the layer's attention, and the MLP acts on each row
+    # alone, so compacting before the MLP (which then runs on kept rows only)
+    # must leave every kept row, index and logit unchanged.
+    cfg = _cfg(dtype=dtype)
+    w = _tiny_weights(cfg, seed=8)
+    tokens = np.random.default_rng(17).integers(0, cfg.vocab, (2, 33))
+    a = O.forward(cfg, w, tokens, alpha=0.6)
+    cfg2 = _cfg(dtype=dtype, prune_point="attention")
+    b = O.forward(cfg2, w, tokens, alpha=0.6)
+    # (float64 products over a different number of rows may round differently
+    # in the last bit, and in bf16 such a bit can flip a rounding)
+    tol = 1e-12 if dtype == "f32" else 2e-2
+    for layer in a["idx"]:
+        np.testing.assert_array_equal(a["idx"][layer], b["idx"][layer])
+        np.testing.assert_allclose(a["scores"][layer], b["scores"][layer], rtol=tol)
+    np.testing.assert_array_equal(a["kept_pos"], b["kept_pos"])
+    np.testing.assert_allclose(a["logits"], b["logits"], rtol=tol, atol=tol)
+    with pytest.raises(ValueError):
+        O.forward(_cfg(prune_point="mlp"), w, tokens, alpha=0.6)
