@@ -8,7 +8,8 @@ it.  It shares no code with the CUDA path and imports nothing from it.
 Every function follows one passage of the paper:
 
 * ``attention_probs`` / ``attention_output`` -- Eq. 1 (Sec. 3.2): the soft-score
-  ``softmax(QK^T/sqrt(d_k) + M)`` with a causal mask M, then multiplied by V.
+  ``softmax(QK^T/sqrt(d_k) + M)`` with a causal mask M (or none, for the
+  bidirectional-encoder variant), then multiplied by V.
 * ``column_mass`` / ``position_scores`` -- Sec. 3.2 and Sec. 3.3: the soft-score
   times V gives each V row's contribution to the layer output; rows with the
   lowest contribution are eliminated from the following layers.
@@ -78,6 +79,8 @@ class OracleConfig:
     # where a pruning layer compacts its rows: "layer" (after the MLP, R3) or
     # "attention" (between attention and MLP; the MLP then runs on kept rows only)
     prune_point: str = "layer"
+    # Eq. 1's mask M: causal (decoder) or none (bidirectional encoder)
+    causal: bool = True
 
 
 # --------------------------------------------------------------------------
@@ -146,16 +149,18 @@ def silu(x: np.ndarray) -> np.ndarray:
     return x / (1.0 + np.exp(-x))
 
 
-def attention_probs(q: np.ndarray, k: np.ndarray, key_mask: Optional[np.ndarray] = None) -> np.ndarray:
+def attention_probs(q: np.ndarray, k: np.ndarray, key_mask: Optional[np.ndarray] = None,
+                    causal: bool = True) -> np.ndarray:
     """Soft-score of Eq. 1 for one head: softmax(q k^T / sqrt(d_k) + M).
 
-    q: [n, hd], k: [n, hd].  M is causal (-inf above the diagonal); if
-    ``key_mask`` (bool [n]) is given, keys where it is False are also -inf.
+    q: [n, hd], k: [n, hd].  M is causal (-inf above the diagonal), or zero
+    for a bidirectional encoder (``causal=False``); if ``key_mask`` (bool [n])
+    is given, keys where it is False are also -inf.
     Returns P [n, n] with rows summing to one.
     """
     n, hd = q.shape
     logits = (q @ k.T) / math.sqrt(hd)
-    allowed = np.tril(np.ones((n, n), dtype=bool))
+    allowed = np.tril(np.ones((n, n), dtype=bool)) if causal else np.ones((n, n), dtype=bool)
     if key_mask is not None:
         allowed = allowed & key_mask[None, :]
     logits = np.where(allowed, logits, -np.inf)
@@ -325,7 +330,7 @@ def attention_block(cfg: OracleConfig, lw: Dict[str, np.ndarray], h: np.ndarray,
     o = np.empty((n, H, hd))
     for hh in range(H):
         g = hh // per
-        P[hh] = attention_probs(q[:, hh, :], k[:, g, :], key_mask)
+        P[hh] = attention_probs(q[:, hh, :], k[:, g, :], key_mask, cfg.causal)
         o[:, hh, :] = P[hh] @ v[:, g, :]
     o = store(o.reshape(n, H * hd))
     h = store(h + o @ _as64(lw["wo"]).T)
@@ -510,6 +515,8 @@ def decode_step(cfg: OracleConfig, weights, cache, tokens: np.ndarray):
     """
     if cfg.n_classes > 0:
         raise ValueError("generation needs the language-model head")
+    if not cfg.causal:
+        raise ValueError("generation needs causal attention")
     tokens = np.asarray(tokens)
     B = tokens.shape[0]
     H, G, hd = cfg.n_heads, cfg.n_kv_heads, cfg.head_dim

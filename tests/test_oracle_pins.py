@@ -287,7 +287,7 @@ def _tiny_weights(cfg, seed=0, scale=0.3):
     return dict(embed=nrm(cfg.vocab, d), layers=layers, final_norm=1 + 0.1 * nrm(d), head=nrm(heads, d))
 
 
-def _torch_forward_unpruned(cfg, w, tokens, key_alive=None, all_rows=False):
+def _torch_forward_unpruned(cfg, w, tokens, key_alive=None, all_rows=False):  # noqa: C901
     """Unpruned decoder composed from torch library routines (float64).
 
     ``key_alive[l]`` (bool [B, n], 0-based layer l) hides keys from layer l on
@@ -307,7 +307,7 @@ def _torch_forward_unpruned(cfg, w, tokens, key_alive=None, all_rows=False):
             q = T(_rope_complex(q, pos, cfg.rope_theta)).transpose(0, 1)[None]
             k = T(_rope_complex(k, pos, cfg.rope_theta)).transpose(0, 1)[None]
             if key_alive is None:
-                o = F.scaled_dot_product_attention(q, k, v.transpose(0, 1)[None], is_causal=True,
+                o = F.scaled_dot_product_attention(q, k, v.transpose(0, 1)[None], is_causal=cfg.causal,
                                                    enable_gqa=True)
             else:
                 allowed = torch.tril(torch.ones(n, n, dtype=torch.bool))
@@ -506,3 +506,52 @@ def test_pruning_between_attention_and_mlp_gives_the_same_rows(dtype):
     np.testing.assert_allclose(a["logits"], b["logits"], rtol=tol, atol=tol)
     with pytest.raises(ValueError):
         O.forward(_cfg(prune_point="mlp"), w, tokens, alpha=0.6)
+
+
+# ---------------------------------------------------------------- bidirectional encoder variant
+
+@pytest.mark.parametrize("n,hd", [(1, 8), (9, 16)])
+def test_attention_without_mask_matches_sdpa(n, hd):
+    rng = np.random.default_rng(30 + n)
+    q, k = rng.standard_normal((n, hd)), rng.standard_normal((n, hd))
+    P = O.attention_probs(q, k, causal=False)
+    tq, tk = torch.from_numpy(q)[None, None], torch.from_numpy(k)[None, None]
+    eye = torch.eye(n, dtype=torch.float64)[None, None]
+    ref = F.scaled_dot_product_attention(tq, tk, eye, is_causal=False)[0, 0].numpy()
+    np.testing.assert_allclose(P, ref, rtol=1e-12, atol=1e-14)
+    assert np.all(P > 0)
+
+
+def test_column_mass_closed_form_uniform_bidirectional():
+    # q = 0: every query spreads 1/n over all n keys, so each key collects
+    # exactly one unit per query head of its group.
+    n, H, G = 10, 4, 2
+    P = np.stack([O.attention_probs(np.zeros((n, 8)), np.ones((n, 8)), causal=False) for _ in range(H)])
+    np.testing.assert_allclose(O.column_mass(P, G), np.full((G, n), H // G), rtol=1e-13)
+
+
+def test_bidirectional_forward_matches_torch_composition():
+    cfg = _cfg(prune_layers=[], causal=False)
+    w = _tiny_weights(cfg, seed=9)
+    tokens = np.random.default_rng(18).integers(0, cfg.vocab, (2, 15))
+    got = O.forward(cfg, w, tokens, accel=1.0)
+    ref = _torch_forward_unpruned(cfg, w, tokens)
+    np.testing.assert_allclose(got["logits"], ref, rtol=1e-9, atol=1e-9)
+    causal = O.forward(_cfg(prune_layers=[]), w, tokens, accel=1.0)
+    # in one layer only the last row would see the same keys under both
+    # masks; the first row sees all keys here and one key under the causal mask
+    assert np.abs(got["logits"][:, 0] - causal["logits"][:, 0]).max() > 1e-6
+
+
+def test_bidirectional_compacted_equals_masked_formulation():
+    cfg = _cfg(causal=False)
+    w = _tiny_weights(cfg, seed=10)
+    tokens = np.random.default_rng(19).integers(0, cfg.vocab, (2, 31))
+    sched = O.schedule(31, 0.6, cfg.n_layers, cfg.prune_layers, cfg.tau)
+    a = O.forward(cfg, w, tokens, alpha=0.6)
+    m = O.forward_masked(cfg, w, tokens, sched)
+    np.testing.assert_array_equal(a["kept_pos"], m["kept_pos"])
+    np.testing.assert_allclose(a["logits"], m["logits"], rtol=1e-9, atol=1e-9)
+    with pytest.raises(ValueError):
+        O.decode_step(cfg, w, O.forward(cfg, w, tokens, alpha=0.6, collect_cache=True)["cache"],
+                      tokens[:, 0])
