@@ -85,6 +85,7 @@ typedef struct {
   int force_keep_last;  /* 1: the last position is always kept (counts toward N_l) */
   int score_mode;       /* ZSAA_SCORE_* */
   int plan_mode;        /* ZSAA_PLAN_* */
+  int bidirectional;    /* 0: causal decoder (Eq. 1 with the causal mask M); 1: encoder, M = 0 */
 } zsaa_config;
 
 /* Borrowed device weights; they must outlive the model.  layers points to a
@@ -304,6 +305,14 @@ zsaa_status zsaa_op_attention(const void* qkv, int B, int N, int Hq, int Hkv, in
  * the lse that zsaa_op_attention wrote. */
 zsaa_status zsaa_op_colmass(const void* qkv, const float* lse, int B, int N, int Hq, int Hkv,
                             int hd, int dtype, float* colmass, zsaa_stream stream);
+
+/* The two steps above with the mask of Eq. 1 chosen: causal = 1 as above,
+ * causal = 0 for a bidirectional encoder (M = 0: every query sees every key,
+ * and the column mass sums P[i,j] over all queries i). */
+zsaa_status zsaa_op_attention_ex(const void* qkv, int B, int N, int Hq, int Hkv, int hd, int dtype,
+                                 int causal, void* out, float* lse, zsaa_stream stream);
+zsaa_status zsaa_op_colmass_ex(const void* qkv, const float* lse, int B, int N, int Hq, int Hkv,
+                               int hd, int dtype, int causal, float* colmass, zsaa_stream stream);
 
 /* Per-kernel timing of the forward pass.  After zsaa_trace_begin every
  * kernel the model launches is bracketed by CUDA events recorded on the launch

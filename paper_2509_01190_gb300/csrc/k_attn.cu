@@ -49,7 +49,8 @@ __device__ __forceinline__ void load_tile64(uint32_t sbase, const bf16* g, size_
 template <int HD>
 __global__ void __launch_bounds__(128)
     attn_fwd_bf16_kernel(const bf16* __restrict__ qkv, int N, int Hq, int Hkv,
-                         bf16* __restrict__ out, float* __restrict__ lse2, float scale_log2) {
+                         bf16* __restrict__ out, float* __restrict__ lse2, float scale_log2,
+                         int causal) {
   pdl_trigger();
   pdl_wait();
   constexpr int ROWB = HD * 2;
@@ -69,7 +70,7 @@ __global__ void __launch_bounds__(128)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gid = lane >> 2, tig = lane & 3;
 
-  const int kv_end = min(N, q0 + 64);
+  const int kv_end = causal ? min(N, q0 + 64) : N;
   const int n_kb = (kv_end + 63) / 64;
 
   load_tile64<HD>(sQ, Qg, ld, q0, N);
@@ -126,8 +127,8 @@ __global__ void __launch_bounds__(128)
       for (int e = 0; e < 2; ++e) {
         const int j = k0 + nt * 8 + 2 * tig + e;
         float a = s[nt][e] * scale_log2, c = s[nt][2 + e] * scale_log2;
-        if (j > i_lo || j >= N) a = -INFINITY;
-        if (j > i_hi || j >= N) c = -INFINITY;
+        if ((causal && j > i_lo) || j >= N) a = -INFINITY;
+        if ((causal && j > i_hi) || j >= N) c = -INFINITY;
         s[nt][e] = a;
         s[nt][2 + e] = c;
         mx_lo = fmaxf(mx_lo, a);
@@ -221,7 +222,7 @@ template <int HD>
 __global__ void __launch_bounds__(128)
     colmass_bf16_kernel(const bf16* __restrict__ qkv, const float* __restrict__ lse2, int N,
                         int Hq, int Hkv, int B, int q_per, int weight_vnorm,
-                        float* __restrict__ parts, float scale_log2) {
+                        float* __restrict__ parts, float scale_log2, int causal) {
   pdl_trigger();
   pdl_wait();
   constexpr int ROWB = HD * 2;
@@ -240,7 +241,7 @@ __global__ void __launch_bounds__(128)
   const int gid = lane >> 2, tig = lane & 3;
   const int j_lo = kb * 64 + warp * 16 + gid, j_hi = j_lo + 8;
   const int n_qb = (N + 63) / 64;
-  const int qb0 = max(kb, qc * q_per), qb1 = min(n_qb, (qc + 1) * q_per);
+  const int qb0 = max(causal ? kb : 0, qc * q_per), qb1 = min(n_qb, (qc + 1) * q_per);
   const int nq = qb1 > qb0 ? qb1 - qb0 : 0;
   const int steps = per * nq;
 
@@ -300,8 +301,8 @@ __global__ void __launch_bounds__(128)
           const int i = qb * 64 + qi;
           if (i < N) {
             const float l = Lq[qi];
-            if (i >= j_lo) acc_lo += exp2f(sacc[nt][e] * scale_log2 - l);
-            if (i >= j_hi) acc_hi += exp2f(sacc[nt][2 + e] * scale_log2 - l);
+            if (!causal || i >= j_lo) acc_lo += exp2f(sacc[nt][e] * scale_log2 - l);
+            if (!causal || i >= j_hi) acc_hi += exp2f(sacc[nt][2 + e] * scale_log2 - l);
           }
         }
       }
@@ -376,7 +377,7 @@ __global__ void colmass_reduce_kernel(const float* __restrict__ parts, int n_qc,
 // fp32 attention: one warp per (query i, head h, batch b).
 __global__ void attn_fwd_f32_kernel(const float* __restrict__ qkv, int N, int Hq, int Hkv, int hd,
                                     float* __restrict__ out, float* __restrict__ lse2,
-                                    float scale_log2) {
+                                    float scale_log2, int causal) {
   pdl_trigger();
   pdl_wait();
   const int i = blockIdx.x * 4 + (threadIdx.x >> 5);
@@ -386,9 +387,10 @@ __global__ void attn_fwd_f32_kernel(const float* __restrict__ qkv, int N, int Hq
   const size_t ld = static_cast<size_t>(Hq + 2 * Hkv) * hd;
   const float* base = qkv + static_cast<size_t>(b) * N * ld;
   const float* q = base + i * ld + h * hd;
+  const int jend = causal ? i + 1 : N;  // keys [0, jend)
   // pass 1: max and normaliser (per lane over its keys, then merged)
   float m = -INFINITY, l = 0.f;
-  for (int j = lane; j <= i; j += 32) {
+  for (int j = lane; j < jend; j += 32) {
     const float* k = base + j * ld + (Hq + g) * hd;
     float s = 0.f;
     for (int e = 0; e < hd; ++e) s = fmaf(q[e], k[e], s);
@@ -407,16 +409,16 @@ __global__ void attn_fwd_f32_kernel(const float* __restrict__ qkv, int N, int Hq
   const float lse = m + log2f(l);
   // pass 2: output, each lane owns dims lane, lane+32, ...
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int j0 = 0; j0 <= i; j0 += 32) {
+  for (int j0 = 0; j0 < jend; j0 += 32) {
     const int j = j0 + lane;
     float p = 0.f;
-    if (j <= i) {
+    if (j < jend) {
       const float* k = base + j * ld + (Hq + g) * hd;
       float s = 0.f;
       for (int e = 0; e < hd; ++e) s = fmaf(q[e], k[e], s);
       p = exp2f(s * scale_log2 - lse);
     }
-    const int cnt = min(32, i - j0 + 1);
+    const int cnt = min(32, jend - j0);
     for (int t = 0; t < cnt; ++t) {
       const float pt = __shfl_sync(0xffffffffu, p, t);
       const float* v = base + (j0 + t) * ld + (Hq + Hkv + g) * hd;
@@ -431,7 +433,7 @@ __global__ void attn_fwd_f32_kernel(const float* __restrict__ qkv, int N, int Hq
 // fp32 column mass: one warp per (key j, KV head g, batch b); one query chunk.
 __global__ void colmass_f32_kernel(const float* __restrict__ qkv, const float* __restrict__ lse2,
                                    int N, int Hq, int Hkv, int hd, int B, int weight_vnorm,
-                                   float* __restrict__ parts, float scale_log2) {
+                                   float* __restrict__ parts, float scale_log2, int causal) {
   pdl_trigger();
   pdl_wait();
   const int j = blockIdx.x * 4 + (threadIdx.x >> 5);
@@ -444,7 +446,7 @@ __global__ void colmass_f32_kernel(const float* __restrict__ qkv, const float* _
   float acc = 0.f;
   for (int hh = 0; hh < per; ++hh) {
     const int h = g * per + hh;
-    for (int i = j + lane; i < N; i += 32) {
+    for (int i = (causal ? j : 0) + lane; i < N; i += 32) {
       const float* q = base + i * ld + h * hd;
       float s = 0.f;
       for (int e = 0; e < hd; ++e) s = fmaf(q[e], k[e], s);
@@ -469,12 +471,12 @@ cudaError_t set_smem(Kern k, int bytes) {
 }  // namespace
 
 cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, int Hkv, int hd,
-                             void* out, float* lse, cudaStream_t s) {
+                             void* out, float* lse, int causal, cudaStream_t s) {
   const float scale_log2 = kLog2e / sqrtf(static_cast<float>(hd));
   if (dtype == ZSAA_F32) {
     dim3 grid((N + 3) / 4, Hq, B);
     ZSAA_LAUNCH(attn_fwd_f32_kernel, dim3(grid), dim3(128), 0, s, static_cast<const float*>(qkv), N, Hq, Hkv, hd,
-                                             static_cast<float*>(out), lse, scale_log2);
+                                             static_cast<float*>(out), lse, scale_log2, causal);
     return cudaGetLastError();
   }
   dim3 grid((N + 63) / 64, Hq, B);
@@ -483,13 +485,13 @@ cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, i
     static cudaError_t e = set_smem(attn_fwd_bf16_kernel<64>, smem);
     if (e != cudaSuccess) return e;
     ZSAA_LAUNCH(attn_fwd_bf16_kernel<64>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), N, Hq, Hkv,
-                                                      static_cast<bf16*>(out), lse, scale_log2);
+                                                      static_cast<bf16*>(out), lse, scale_log2, causal);
   } else if (hd == 128) {
     const int smem = 5 * 64 * 256;
     static cudaError_t e = set_smem(attn_fwd_bf16_kernel<128>, smem);
     if (e != cudaSuccess) return e;
     ZSAA_LAUNCH(attn_fwd_bf16_kernel<128>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), N, Hq, Hkv,
-                                                       static_cast<bf16*>(out), lse, scale_log2);
+                                                       static_cast<bf16*>(out), lse, scale_log2, causal);
   } else {
     return cudaErrorInvalidValue;
   }
@@ -510,17 +512,17 @@ size_t colmass_parts_elems(int B, int N, int Hq, int Hkv) {
 namespace {
 cudaError_t colmass_parts(int dtype, const void* qkv, const float* lse, const float* vnorm, int B,
                           int N, int Hq, int Hkv, int hd, int weight_vnorm, float* parts, int* n_qc,
-                          int* status, cudaStream_t s) {
+                          int* status, int causal, cudaStream_t s) {
   // tensor-core path (with precomputed norms when they are needed)
   if (dtype == ZSAA_BF16 && status != nullptr && (!weight_vnorm || vnorm != nullptr))
     return launch_colmass_tc(qkv, lse, weight_vnorm ? vnorm : nullptr, B, N, Hq, Hkv, hd, parts,
-                             status, n_qc, s);
+                             status, n_qc, causal, s);
   const float scale_log2 = kLog2e / sqrtf(static_cast<float>(hd));
   if (dtype == ZSAA_F32) {
     *n_qc = 1;
     dim3 grid((N + 3) / 4, Hkv, B);
     ZSAA_LAUNCH(colmass_f32_kernel, dim3(grid), dim3(128), 0, s, static_cast<const float*>(qkv), lse, N, Hq, Hkv, hd, B,
-                                            weight_vnorm, parts, scale_log2);
+                                            weight_vnorm, parts, scale_log2, causal);
     return cudaGetLastError();
   }
   *n_qc = colmass_chunks(N);
@@ -531,14 +533,14 @@ cudaError_t colmass_parts(int dtype, const void* qkv, const float* lse, const fl
     if (e != cudaSuccess) return e;
     ZSAA_LAUNCH(colmass_bf16_kernel<64>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), lse, N, Hq,
                                                      Hkv, B, kColmassQPer, weight_vnorm, parts,
-                                                     scale_log2);
+                                                     scale_log2, causal);
   } else if (hd == 128) {
     const int smem = 3 * 64 * 256 + 2 * 64 * 4;
     static cudaError_t e = set_smem(colmass_bf16_kernel<128>, smem);
     if (e != cudaSuccess) return e;
     ZSAA_LAUNCH(colmass_bf16_kernel<128>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), lse, N, Hq,
                                                       Hkv, B, kColmassQPer, weight_vnorm, parts,
-                                                      scale_log2);
+                                                      scale_log2, causal);
   } else {
     return cudaErrorInvalidValue;
   }
@@ -547,9 +549,11 @@ cudaError_t colmass_parts(int dtype, const void* qkv, const float* lse, const fl
 }  // namespace
 
 cudaError_t launch_colmass(int dtype, const void* qkv, const float* lse, int B, int N, int Hq,
-                           int Hkv, int hd, float* parts, float* C, int* status, cudaStream_t s) {
+                           int Hkv, int hd, float* parts, float* C, int* status, int causal,
+                           cudaStream_t s) {
   int n_qc = 1;
-  cudaError_t e = colmass_parts(dtype, qkv, lse, nullptr, B, N, Hq, Hkv, hd, 0, parts, &n_qc, status, s);
+  cudaError_t e = colmass_parts(dtype, qkv, lse, nullptr, B, N, Hq, Hkv, hd, 0, parts, &n_qc, status,
+                                causal, s);
   if (e != cudaSuccess) return e;
   const int total = B * Hkv * N;
   ZSAA_LAUNCH(colmass_reduce_kernel, dim3((total + 255) / 256), dim3(256), 0, s, parts, n_qc, B, Hkv, N, 0, C);
@@ -558,17 +562,18 @@ cudaError_t launch_colmass(int dtype, const void* qkv, const float* lse, int B, 
 
 cudaError_t launch_position_parts(int dtype, const void* qkv, const float* lse, const float* vnorm,
                                   int B, int N, int Hq, int Hkv, int hd, int mode, float* parts,
-                                  int* n_qc, int* status, cudaStream_t s) {
+                                  int* n_qc, int* status, int causal, cudaStream_t s) {
   return colmass_parts(dtype, qkv, lse, vnorm, B, N, Hq, Hkv, hd,
-                       mode == ZSAA_SCORE_SOFTSCORE_VNORM ? 1 : 0, parts, n_qc, status, s);
+                       mode == ZSAA_SCORE_SOFTSCORE_VNORM ? 1 : 0, parts, n_qc, status, causal, s);
 }
 
 cudaError_t launch_position_scores(int dtype, const void* qkv, const float* lse, const float* vnorm,
                                    int B, int N, int Hq, int Hkv, int hd, int mode, float* parts,
-                                   float* scores, int* status, cudaStream_t s) {
+                                   float* scores, int* status, int causal, cudaStream_t s) {
   int n_qc = 1;
   cudaError_t e = colmass_parts(dtype, qkv, lse, vnorm, B, N, Hq, Hkv, hd,
-                                mode == ZSAA_SCORE_SOFTSCORE_VNORM ? 1 : 0, parts, &n_qc, status, s);
+                                mode == ZSAA_SCORE_SOFTSCORE_VNORM ? 1 : 0, parts, &n_qc, status,
+                                causal, s);
   if (e != cudaSuccess) return e;
   const int total = B * N;
   ZSAA_LAUNCH(colmass_reduce_kernel, dim3((total + 255) / 256), dim3(256), 0, s, parts, n_qc, B, Hkv, N, 1, scores);

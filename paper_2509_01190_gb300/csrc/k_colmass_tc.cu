@@ -4,7 +4,8 @@
 // For every sequence b, KV group g, query head h of g and block of 128 keys,
 // the CTA computes S^T = K Q^T (M = 128 keys, N = 128 queries, K = hd) with
 // tcgen05.mma into TMEM, one query block at a time (only blocks at or after
-// the key block: the mask is causal), and its epilogue warps -- one TMEM lane,
+// the key block when the mask is causal; every block for a bidirectional
+// encoder), and its epilogue warps -- one TMEM lane,
 // i.e. one key, per thread -- accumulate exp2(s * c - lse2[q]) over the
 // queries q >= key of each block.  That is the column sum of the normalised
 // soft-score P (the row normalisers lse2 come from the attention kernel).
@@ -49,6 +50,7 @@ struct CmArgs {
   const float* vnorm;  // [B*N, Hkv] ||v|| per row and group (used when weight_vnorm)
   float* parts;        // [per][B][G][N]
   int B, N, Hq, Hkv, ld, n_kb, total, weight_vnorm;
+  int causal;  // 0: bidirectional (every query block, no causal mask)
   float scale_log2;
   int* status;
 };
@@ -133,7 +135,7 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
         for (int c = 0; c < C::CHUNKS; ++c)
           tma_load_2d(sK + kbuf * C::TILE_BYTES + c * (C::TILE_BYTES / C::CHUNKS), &tm,
                       (a.Hq + g) * HD + c * 64, row0 + kb * CM_BM, &kfull[kbuf]);
-        for (int qb = kb; qb < a.n_kb; ++qb, ++it) {
+        for (int qb = a.causal ? kb : 0; qb < a.n_kb; ++qb, ++it) {
           const int s = it % CM_STAGES;
           const uint32_t ph = (it / CM_STAGES) & 1;
           if (!mbar_wait_ab(&empty[s], ph ^ 1, a.status, abort_flag)) {
@@ -169,7 +171,7 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
         if (!mbar_wait_ab(&kfull[kbuf], (tiles >> 1) & 1, a.status, abort_flag)) break;
         tc_fence_after();
         const uint32_t k_base = smem_u32(sK + kbuf * C::TILE_BYTES);
-        for (int qb = kb; qb < a.n_kb; ++qb, ++it, ++i) {
+        for (int qb = a.causal ? kb : 0; qb < a.n_kb; ++qb, ++it, ++i) {
           const int ab = i & 1;
           const uint32_t use = static_cast<uint32_t>(i >> 1);
           if (!mbar_wait_ab(&acc_empty[ab], (use & 1) ^ 1, a.status, abort_flag)) {
@@ -227,14 +229,14 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
     if (static_cast<int>(blockIdx.x) < a.total) {
       int b, g, hh, kb;
       cm_tile(blockIdx.x, a, b, g, hh, kb);
-      fetch(blockIdx.x, kb, 0);
+      fetch(blockIdx.x, a.causal ? kb : 0, 0);
     }
     for (int t = blockIdx.x; t < a.total; t += gridDim.x) {
       int b, g, hh, kb;
       cm_tile(t, a, b, g, hh, kb);
       const int key = kb * CM_BM + krow;
       float acc = 0.f;
-      for (int qb = kb; qb < a.n_kb; ++qb, ++i) {
+      for (int qb = a.causal ? kb : 0; qb < a.n_kb; ++qb, ++i) {
         const int ab = i & 1;
         const uint32_t use = static_cast<uint32_t>(i >> 1);
         cp_async_wait<0>();
@@ -245,7 +247,7 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
         } else if (t + static_cast<int>(gridDim.x) < a.total) {
           int b2, g2, hh2, kb2;
           cm_tile(t + gridDim.x, a, b2, g2, hh2, kb2);
-          fetch(t + gridDim.x, kb2, ab ^ 1);
+          fetch(t + gridDim.x, a.causal ? kb2 : 0, ab ^ 1);
         }
         const float* L = s_lse + ab * CM_BN;
         ok = ok && __all_sync(0xffffffffu, mbar_wait_ab(&acc_full[ab], use & 1, a.status, abort_flag));
@@ -262,14 +264,15 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
             tmem_ld_wait();
             const int qc0 = half * 64 + c;
             const int q0 = qb * CM_BN + qc0;
-            if (q0 > key && q0 + 32 <= a.N) {  // whole chunk inside the causal region
+            if ((!a.causal || q0 > key) && q0 + 32 <= a.N) {  // whole chunk inside the mask
 #pragma unroll
               for (int e = 0; e < 32; ++e) acc += ex2_ftz(__uint_as_float(r[e]) * a.scale_log2 - L[qc0 + e]);
             } else {
 #pragma unroll
               for (int e = 0; e < 32; ++e) {
                 const int q = q0 + e;
-                if (q >= key && q < a.N) acc += ex2_ftz(__uint_as_float(r[e]) * a.scale_log2 - L[qc0 + e]);
+                if ((!a.causal || q >= key) && q < a.N)
+                  acc += ex2_ftz(__uint_as_float(r[e]) * a.scale_log2 - L[qc0 + e]);
               }
             }
           }
@@ -328,7 +331,7 @@ cudaError_t run_cm(const CUtensorMap& tm, const CmArgs& a, int sms, cudaStream_t
 
 cudaError_t launch_colmass_tc(const void* qkv, const float* lse, const float* vnorm, int B, int N,
                               int Hq, int Hkv, int hd, float* parts, int* status, int* n_chunks,
-                              cudaStream_t s) {
+                              int causal, cudaStream_t s) {
   if (hd != 64 && hd != 128) return cudaErrorInvalidValue;
   const int ld = (Hq + 2 * Hkv) * hd;
   EncodeTiledFn enc = get_encode_tiled();
@@ -354,6 +357,7 @@ cudaError_t launch_colmass_tc(const void* qkv, const float* lse, const float* vn
   a.n_kb = (N + CM_BM - 1) / CM_BM;
   a.total = a.n_kb * B * Hq;
   a.weight_vnorm = vnorm != nullptr;
+  a.causal = causal;
   a.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(hd));
   a.status = status;
   *n_chunks = Hq / Hkv;

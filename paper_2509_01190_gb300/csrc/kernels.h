@@ -92,8 +92,10 @@ cudaError_t launch_gemm_f32(const float* A, int lda, const float* W, const float
                             const GemmParams& p, cudaStream_t s);
 
 // ---- attention (k_attn.cu)
+// causal = 0: bidirectional (Eq. 1 with M = 0); the column-mass kernels below
+// take the same flag.
 cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, int Hkv, int hd,
-                             void* out, float* lse, cudaStream_t s);
+                             void* out, float* lse, int causal, cudaStream_t s);
 // Column mass C[B, Hkv, N] (via partial sums in `parts`, which must hold
 // colmass_parts_elems(B, N, Hq, Hkv) floats).  bf16 with a status word runs
 // the tensor-core kernel (k_colmass_tc.cu); otherwise the mma.sync / fp32 ones.
@@ -101,7 +103,8 @@ constexpr int kColmassQPer = 2;  // query blocks of 64 per mma.sync column-mass 
 int colmass_chunks(int N);
 size_t colmass_parts_elems(int B, int N, int Hq, int Hkv);
 cudaError_t launch_colmass(int dtype, const void* qkv, const float* lse, int B, int N, int Hq,
-                           int Hkv, int hd, float* parts, float* C, int* status, cudaStream_t s);
+                           int Hkv, int hd, float* parts, float* C, int* status, int causal,
+                           cudaStream_t s);
 // The score paths below take vnorm = ||v|| per row and group ([B*N, Hkv], from
 // the QKV epilogue) for the bf16 tensor-core kernel; NULL makes the kernels
 // compute the norms from qkv themselves.
@@ -109,17 +112,17 @@ cudaError_t launch_colmass(int dtype, const void* qkv, const float* lse, int B, 
 // ||v|| per group, summed over groups; same workspace as launch_colmass.
 cudaError_t launch_position_scores(int dtype, const void* qkv, const float* lse, const float* vnorm,
                                    int B, int N, int Hq, int Hkv, int hd, int mode, float* parts,
-                                   float* scores, int* status, cudaStream_t s);
+                                   float* scores, int* status, int causal, cudaStream_t s);
 // Only the partials of the position scores (for launch_select_parts); *n_qc
 // receives the number of partial chunks.
 cudaError_t launch_position_parts(int dtype, const void* qkv, const float* lse, const float* vnorm,
                                   int B, int N, int Hq, int Hkv, int hd, int mode, float* parts,
-                                  int* n_qc, int* status, cudaStream_t s);
+                                  int* n_qc, int* status, int causal, cudaStream_t s);
 // Tensor-core column-mass partials: parts[Hq/Hkv][B][Hkv][N] (per head of the
 // group), times vnorm when it is not NULL; hd 64 or 128.
 cudaError_t launch_colmass_tc(const void* qkv, const float* lse, const float* vnorm, int B, int N,
                               int Hq, int Hkv, int hd, float* parts, int* status, int* n_chunks,
-                              cudaStream_t s);
+                              int causal, cudaStream_t s);
 
 // ---- generation over the pruned KV cache (k_decode.cu)
 // Cache of one layer: K and V bf16 [B, Hkv, cap, hd], positions int32 [B, cap].

@@ -124,6 +124,7 @@ zsaa_status validate_config(const zsaa_config& c) {
     return fail(ZSAA_ERR_INVALID_ARG, "bad score_mode");
   if (c.plan_mode != ZSAA_PLAN_COST && c.plan_mode != ZSAA_PLAN_RATE)
     return fail(ZSAA_ERR_INVALID_ARG, "bad plan_mode");
+  if (c.bidirectional != 0 && c.bidirectional != 1) return fail(ZSAA_ERR_INVALID_ARG, "bidirectional must be 0 or 1");
   if (c.n_layers < 64 && (c.prune_mask >> c.n_layers) != 0)
     return fail(ZSAA_ERR_INVALID_ARG, "prune_mask names layers beyond n_layers");
   if (c.dtype == ZSAA_BF16) {
@@ -439,6 +440,9 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
 
   const int d = c.d_model, hd = c.head_dim, Hq = c.n_heads, Hkv = c.n_kv_heads;
   const int dt = c.dtype;
+  const int causal = c.bidirectional ? 0 : 1;
+  // query-key pairs of Eq. 1 per sequence and head
+  auto n_pairs = [&](int n) { return causal ? static_cast<double>(n) * (n + 1) / 2.0 : static_cast<double>(n) * n; };
   int cur = 0;
   const double es = static_cast<double>(m->esz);
 #define TRACE(name, fl, by) TraceScope trace_scope_(m, name, fl, by, s)
@@ -526,9 +530,9 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
       ZCK(launch_kv_write(m->qkv, m->ld_qkv, m->pos[cur], B, N, Hq, Hkv, hd, kc->layers[li], s));
     }
     {
-      const double pairs = static_cast<double>(B) * Hq * (static_cast<double>(N) * (N + 1) / 2.0);
+      const double pairs = static_cast<double>(B) * Hq * n_pairs(N);
       TRACE("attention", 4.0 * pairs * hd, Md * (m->ld_qkv + m->dq) * es + static_cast<double>(B) * Hq * N * 4.0);
-      ZCK(launch_attention(dt, m->qkv, B, N, Hq, Hkv, hd, m->attn, m->lse, s));
+      ZCK(launch_attention(dt, m->qkv, B, N, Hq, Hkv, hd, m->attn, m->lse, causal, s));
     }
     {
       GemmParams q{};
@@ -556,7 +560,7 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
       const bool want_idx = opts && opts->idx_out;
       if (k < N || want_scores || want_idx) {
         float* sc = want_scores ? opts->scores_out + off_scores : m->scores;
-        const double pairs = static_cast<double>(B) * Hq * (static_cast<double>(N) * (N + 1) / 2.0);
+        const double pairs = static_cast<double>(B) * Hq * n_pairs(N);
         const int32_t* idx = m->idx;
         if (dt == ZSAA_BF16 && !forced && k < N && N <= kSelectPartsMaxN) {
           // column-mass partials, then top-k with the score reduction fused in
@@ -565,7 +569,8 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
             TRACE("colmass", 2.0 * pairs * hd,
                   Md * (m->dq + 2 * m->dkv) * es + static_cast<double>(B) * Hq * N * 4.0);
             ZCK(launch_position_parts(dt, m->qkv, m->lse, dt == ZSAA_BF16 ? m->vnorm : nullptr, B, N,
-                                      Hq, Hkv, hd, c.score_mode, m->colmass, &n_qc, m->status, s));
+                                      Hq, Hkv, hd, c.score_mode, m->colmass, &n_qc, m->status,
+                                      causal, s));
           }
           TRACE("select", 0.0, static_cast<double>(n_qc) * B * Hkv * N * 4.0 + static_cast<double>(B) * k * 4.0);
           ZCK(launch_select_parts(m->colmass, n_qc, B, Hkv, N, k, c.force_keep_last, m->idx,
@@ -576,7 +581,8 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
                   Md * (m->dq + 2 * m->dkv) * es + static_cast<double>(B) * Hq * N * 4.0 + Md * 4.0);
             trace_scope_.kernels = 2;
             ZCK(launch_position_scores(dt, m->qkv, m->lse, dt == ZSAA_BF16 ? m->vnorm : nullptr, B, N,
-                                       Hq, Hkv, hd, c.score_mode, m->colmass, sc, m->status, s));
+                                       Hq, Hkv, hd, c.score_mode, m->colmass, sc, m->status,
+                                       causal, s));
           }
           if (forced) {
             idx = opts->forced_idx + off_forced;
@@ -1237,16 +1243,27 @@ zsaa_status zsaa_op_linear(const void* A, const void* W, const void* W2, const v
 
 zsaa_status zsaa_op_attention(const void* qkv, int B, int N, int Hq, int Hkv, int hd, int dtype,
                               void* out, float* lse, zsaa_stream stream) {
+  return zsaa_op_attention_ex(qkv, B, N, Hq, Hkv, hd, dtype, 1, out, lse, stream);
+}
+
+zsaa_status zsaa_op_attention_ex(const void* qkv, int B, int N, int Hq, int Hkv, int hd, int dtype,
+                                 int causal, void* out, float* lse, zsaa_stream stream) {
   if (qkv == nullptr || out == nullptr || lse == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null argument");
   if (B < 1 || N < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv) return fail(ZSAA_ERR_INVALID_ARG, "bad shape");
   if (dtype == ZSAA_BF16 && hd != 64 && hd != 128) return fail(ZSAA_ERR_UNSUPPORTED, "bf16 attention needs hd 64 or 128");
   if (dtype == ZSAA_F32 && (hd < 1 || hd > 128)) return fail(ZSAA_ERR_UNSUPPORTED, "f32 attention needs hd <= 128");
-  ZCK(launch_attention(dtype, qkv, B, N, Hq, Hkv, hd, out, lse, reinterpret_cast<cudaStream_t>(stream)));
+  ZCK(launch_attention(dtype, qkv, B, N, Hq, Hkv, hd, out, lse, causal ? 1 : 0,
+                       reinterpret_cast<cudaStream_t>(stream)));
   return ZSAA_OK;
 }
 
 zsaa_status zsaa_op_colmass(const void* qkv, const float* lse, int B, int N, int Hq, int Hkv,
                             int hd, int dtype, float* colmass, zsaa_stream stream) {
+  return zsaa_op_colmass_ex(qkv, lse, B, N, Hq, Hkv, hd, dtype, 1, colmass, stream);
+}
+
+zsaa_status zsaa_op_colmass_ex(const void* qkv, const float* lse, int B, int N, int Hq, int Hkv,
+                               int hd, int dtype, int causal, float* colmass, zsaa_stream stream) {
   if (qkv == nullptr || lse == nullptr || colmass == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null argument");
   if (B < 1 || N < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv) return fail(ZSAA_ERR_INVALID_ARG, "bad shape");
   if (dtype == ZSAA_BF16 && hd != 64 && hd != 128) return fail(ZSAA_ERR_UNSUPPORTED, "bf16 column mass needs hd 64 or 128");
@@ -1256,7 +1273,8 @@ zsaa_status zsaa_op_colmass(const void* qkv, const float* lse, int B, int N, int
   if (status == nullptr) return fail(ZSAA_ERR_CUDA, "status word allocation failed");
   ZCK(cudaMallocAsync(reinterpret_cast<void**>(&parts),
                       colmass_parts_elems(B, N, Hq, Hkv) * sizeof(float), s));
-  cudaError_t e = launch_colmass(dtype, qkv, lse, B, N, Hq, Hkv, hd, parts, colmass, status, s);
+  cudaError_t e = launch_colmass(dtype, qkv, lse, B, N, Hq, Hkv, hd, parts, colmass, status,
+                                 causal ? 1 : 0, s);
   cudaError_t e2 = cudaFreeAsync(parts, s);
   ZCK(e);
   ZCK(e2);
@@ -1304,8 +1322,9 @@ zsaa_status zsaa_cache_create(zsaa_model* m, int B, int L, double accel, int max
   *out = nullptr;
   if (m == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null model");
   const zsaa_config& c = m->cfg;
-  if (c.dtype != ZSAA_BF16 || c.n_classes != 0 || !c.force_keep_last)
-    return fail(ZSAA_ERR_UNSUPPORTED, "generation needs a bf16 model with the LM head and force_keep_last");
+  if (c.dtype != ZSAA_BF16 || c.n_classes != 0 || !c.force_keep_last || c.bidirectional)
+    return fail(ZSAA_ERR_UNSUPPORTED,
+                "generation needs a causal bf16 model with the LM head and force_keep_last");
   if (B < 1 || B > m->max_B || L < 1 || L > m->max_L)
     return fail(ZSAA_ERR_INVALID_ARG, "B=%d L=%d outside [1,%d] x [1,%d]", B, L, m->max_B, m->max_L);
   if (max_new < 1 || max_new > (1 << 20))

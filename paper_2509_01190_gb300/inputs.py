@@ -46,6 +46,8 @@ class ModelShape:
     tie_embeddings: bool = False
     prune: str = "all_but_last"  # or a comma list of 1-based layers, e.g. "1"
     plan_mode: str = "cost"
+    bidirectional: bool = False  # encoder variant: Eq. 1 without the causal mask
+    score_mode: str = "softscore_vnorm"  # or "softscore" (column mass alone)
 
     def prune_layers(self) -> List[int]:
         if self.prune == "all_but_last":

@@ -29,6 +29,7 @@ EXPORTED = [
     "zsaa_last_error", "zsaa_version", "zsaa_trace_begin", "zsaa_trace_end",
     "zsaa_score_select_noalloc", "zsaa_model_set_graphs", "zsaa_cache_create", "zsaa_cache_destroy",
     "zsaa_prefill", "zsaa_decode_step", "zsaa_cache_layer", "zsaa_cache_bytes",
+    "zsaa_op_attention_ex", "zsaa_op_colmass_ex",
 ]
 
 
@@ -44,7 +45,7 @@ class zsaa_config(C.Structure):
         ("head_dim", C.c_int), ("ffn_dim", C.c_int), ("vocab", C.c_int), ("n_classes", C.c_int),
         ("rope_theta", C.c_float), ("rms_eps", C.c_float), ("dtype", C.c_int), ("tau", C.c_int),
         ("prune_mask", C.c_uint64), ("force_keep_last", C.c_int), ("score_mode", C.c_int),
-        ("plan_mode", C.c_int),
+        ("plan_mode", C.c_int), ("bidirectional", C.c_int),
     ]
 
 
@@ -93,6 +94,8 @@ def lib():
             "zsaa_op_linear": ([_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _I, _I, C.c_float, _P], _I),
             "zsaa_op_attention": ([_P, _I, _I, _I, _I, _I, _I, _P, _P, _P], _I),
             "zsaa_op_colmass": ([_P, _P, _I, _I, _I, _I, _I, _I, _P, _P], _I),
+            "zsaa_op_attention_ex": ([_P, _I, _I, _I, _I, _I, _I, _I, _P, _P, _P], _I),
+            "zsaa_op_colmass_ex": ([_P, _P, _I, _I, _I, _I, _I, _I, _I, _P, _P], _I),
             "zsaa_sync": ([_P, _P], _I),
             "zsaa_device_status": ([], _I),
             "zsaa_last_error": ([], C.c_char_p),
@@ -142,7 +145,7 @@ def _stream(stream) -> Optional[int]:
 def make_config(n_layers, d_model, n_heads, n_kv_heads, head_dim, ffn_dim, vocab, n_classes=0,
                 rope_theta=500000.0, rms_eps=1e-5, dtype="bf16", tau=5,
                 prune_layers: Sequence[int] = (), force_keep_last=True,
-                score_mode="softscore_vnorm", plan_mode="cost") -> zsaa_config:
+                score_mode="softscore_vnorm", plan_mode="cost", bidirectional=False) -> zsaa_config:
     mask = 0
     for layer in prune_layers:
         mask |= 1 << (int(layer) - 1)
@@ -151,7 +154,7 @@ def make_config(n_layers, d_model, n_heads, n_kv_heads, head_dim, ffn_dim, vocab
         float(rope_theta), float(rms_eps), ZSAA_BF16 if dtype == "bf16" else ZSAA_F32, tau, mask,
         1 if force_keep_last else 0,
         ZSAA_SCORE_SOFTSCORE_VNORM if score_mode == "softscore_vnorm" else ZSAA_SCORE_SOFTSCORE,
-        ZSAA_PLAN_COST if plan_mode == "cost" else ZSAA_PLAN_RATE)
+        ZSAA_PLAN_COST if plan_mode == "cost" else ZSAA_PLAN_RATE, 1 if bidirectional else 0)
 
 
 def config_from_shape(shape, prune_layers: Optional[Sequence[int]] = None, **overrides) -> zsaa_config:
@@ -161,7 +164,8 @@ def config_from_shape(shape, prune_layers: Optional[Sequence[int]] = None, **ove
               vocab=shape.vocab, n_classes=shape.n_classes, rope_theta=shape.rope_theta,
               rms_eps=shape.rms_eps, dtype=shape.dtype,
               prune_layers=shape.prune_layers() if prune_layers is None else prune_layers,
-              plan_mode=shape.plan_mode)
+              plan_mode=shape.plan_mode, bidirectional=getattr(shape, "bidirectional", False),
+              score_mode=getattr(shape, "score_mode", "softscore_vnorm"))
     kw.update(overrides)
     return make_config(**kw)
 
@@ -379,6 +383,18 @@ def zsaa_op_colmass(qkv, lse, B: int, N: int, Hq: int, Hkv: int, hd: int, dtype:
                     stream=None):
     _check(lib().zsaa_op_colmass(_ptr(qkv), _ptr(lse), B, N, Hq, Hkv, hd, dtype, _ptr(colmass),
                                  _stream(stream)))
+
+
+def zsaa_op_attention_ex(qkv, B: int, N: int, Hq: int, Hkv: int, hd: int, dtype: int, causal: bool,
+                         out, lse, stream=None):
+    _check(lib().zsaa_op_attention_ex(_ptr(qkv), B, N, Hq, Hkv, hd, dtype, 1 if causal else 0,
+                                      _ptr(out), _ptr(lse), _stream(stream)))
+
+
+def zsaa_op_colmass_ex(qkv, lse, B: int, N: int, Hq: int, Hkv: int, hd: int, dtype: int,
+                       causal: bool, colmass, stream=None):
+    _check(lib().zsaa_op_colmass_ex(_ptr(qkv), _ptr(lse), B, N, Hq, Hkv, hd, dtype,
+                                    1 if causal else 0, _ptr(colmass), _stream(stream)))
 
 
 def zsaa_device_status():

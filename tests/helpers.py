@@ -26,7 +26,8 @@ def oracle_cfg(shape, prune_layers=None, n_layers=None):
         ffn_dim=shape.ffn_dim, vocab=shape.vocab, n_classes=shape.n_classes,
         rope_theta=shape.rope_theta, rms_eps=shape.rms_eps, dtype=shape.dtype,
         prune_layers=shape.prune_layers() if prune_layers is None else prune_layers,
-        plan_mode=shape.plan_mode)
+        plan_mode=shape.plan_mode, causal=not getattr(shape, "bidirectional", False),
+        score_mode=getattr(shape, "score_mode", "softscore_vnorm"))
 
 
 def bf16_ulp_close(got, ref, ulps=1, atol=0.0):

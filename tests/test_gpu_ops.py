@@ -241,7 +241,7 @@ def _qkv(B, N, Hq, Hkv, hd, seed, dtype):
     return _rand((B * N, (Hq + 2 * Hkv) * hd), seed, 1.0, dtype)
 
 
-def _oracle_attention(qkv, B, N, Hq, Hkv, hd):
+def _oracle_attention(qkv, B, N, Hq, Hkv, hd, causal=True):
     x = _np(qkv).reshape(B, N, Hq + 2 * Hkv, hd)
     per = Hq // Hkv
     outs, lses, Ps = [], [], []
@@ -252,10 +252,11 @@ def _oracle_attention(qkv, B, N, Hq, Hkv, hd):
         lse = np.empty((Hq, N))
         for h in range(Hq):
             g = h // per
-            P[h] = O.attention_probs(q[:, h], k[:, g])
+            P[h] = O.attention_probs(q[:, h], k[:, g], causal=causal)
             o[:, h] = P[h] @ v[:, g]
             s = (q[:, h] @ k[:, g].T) / math.sqrt(hd)
-            s = np.where(np.tril(np.ones((N, N), bool)), s, -np.inf)
+            if causal:
+                s = np.where(np.tril(np.ones((N, N), bool)), s, -np.inf)
             mx = s.max(axis=1)
             lse[h] = (mx + np.log(np.exp(s - mx[:, None]).sum(axis=1))) / math.log(2.0)
         outs.append(o.reshape(N, Hq * hd))
