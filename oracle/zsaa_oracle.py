@@ -16,7 +16,8 @@ Every function follows one passage of the paper:
 * ``select_topk`` -- Sec. 3.3 (keep the highest-contribution rows).
 * ``schedule`` -- Eq. 2 (Sec. 3.3) with tau = 5 (Sec. 4.2).
 * ``plan`` -- Sec. 3.4 / Sec. 4.4: the preservation rate is picked at inference
-  time, per requested acceleration, without retraining.
+  time, per requested acceleration, without retraining; ``plan_varlen`` picks
+  one rate for a batch of different lengths (R17) and ``forward_varlen`` runs it.
 * ``forward`` -- Appendix A: a pre-norm decoder (RMSNorm, GQA, RoPE, SwiGLU),
   with the Sec. 3.3 elimination applied after each pruning layer.
 * ``forward_masked`` -- Appendix B: the "marked as pruned but not removed"
@@ -299,6 +300,45 @@ def plan(cfg: OracleConfig, L: int, accel: float):
     return alpha, schedule(L, alpha, cfg.n_layers, cfg.prune_layers, cfg.tau)
 
 
+def plan_varlen(cfg: OracleConfig, lengths: Sequence[int], accel: float):
+    """One preservation rate for a batch of sequences of different lengths (R17).
+
+    Sec. 3.4 picks alpha per inference call; with several lengths in one call
+    the "cost" mode bisects (60 steps, as ``plan``) for the largest alpha whose
+    modelled FLOPs summed over the batch are at most 1/accel of the unpruned
+    sum, and every sequence follows Eq. 2 from its own length with that alpha.
+    "rate": alpha = 1/accel.  Returns (alpha, [schedule per sequence]).
+    """
+    lengths = [int(x) for x in lengths]
+    if not lengths or min(lengths) < 1:
+        raise ValueError("lengths must be >= 1")
+    if not accel >= 1.0:
+        raise ValueError("accel must be >= 1")
+
+    def scheds(a):
+        return [schedule(L, a, cfg.n_layers, cfg.prune_layers, cfg.tau) for L in lengths]
+
+    if cfg.plan_mode == "rate":
+        alpha = 1.0 / accel
+        return alpha, scheds(alpha)
+    if cfg.plan_mode != "cost":
+        raise ValueError(cfg.plan_mode)
+    full = sum(model_cost(cfg, sc) for sc in scheds(1.0))
+    target = full / accel
+    if accel == 1.0:
+        alpha = 1.0
+    else:
+        lo, hi = 0.0, 1.0
+        for _ in range(60):
+            mid = 0.5 * (lo + hi)
+            if sum(model_cost(cfg, sc) for sc in scheds(mid)) <= target:
+                lo = mid
+            else:
+                hi = mid
+        alpha = lo
+    return alpha, scheds(alpha)
+
+
 # --------------------------------------------------------------------------
 # forward pass
 # --------------------------------------------------------------------------
@@ -483,6 +523,33 @@ def forward_masked(cfg: OracleConfig, weights, tokens: np.ndarray, sched: Sequen
         "kept_pos": np.stack(kept_pos),
         "kept_by_layer": {k: np.stack(v) for k, v in kept_by_layer.items()},
     }
+
+
+def forward_varlen(cfg: OracleConfig, weights, seqs: Sequence[np.ndarray], accel: Optional[float] = None,
+                   alpha: Optional[float] = None, forced_idx: Optional[Dict[int, list]] = None):
+    """Pruned prefill of sequences of different lengths in one call.
+
+    The rate comes from ``plan_varlen`` (or ``alpha``); each sequence then
+    runs ``forward`` on its own (a sequence never attends to another one).
+    ``forced_idx`` maps a pruning layer to a list of per-sequence index arrays.
+    Returns a dict of per-sequence lists (``logits``, ``kept_pos``,
+    ``schedule``, ``idx`` {layer: [..]}, ``scores`` {layer: [..]}) and ``alpha``.
+    """
+    lengths = [len(t) for t in seqs]
+    if alpha is None:
+        alpha, _ = plan_varlen(cfg, lengths, 1.0 if accel is None else accel)
+    out = {"alpha": alpha, "logits": [], "kept_pos": [], "schedule": [], "idx": {}, "scores": {}}
+    for b, t in enumerate(seqs):
+        fi = None if forced_idx is None else {l: np.asarray(v[b])[None] for l, v in forced_idx.items()}
+        r = forward(cfg, weights, np.asarray(t)[None], alpha=alpha, forced_idx=fi)
+        out["logits"].append(r["logits"][0])
+        out["kept_pos"].append(r["kept_pos"][0])
+        out["schedule"].append(r["schedule"])
+        for l, v in r["idx"].items():
+            out["idx"].setdefault(l, []).append(v[0])
+        for l, v in r["scores"].items():
+            out["scores"].setdefault(l, []).append(v[0])
+    return out
 
 
 # --------------------------------------------------------------------------

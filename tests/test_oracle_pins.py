@@ -555,3 +555,50 @@ def test_bidirectional_compacted_equals_masked_formulation():
     with pytest.raises(ValueError):
         O.decode_step(cfg, w, O.forward(cfg, w, tokens, alpha=0.6, collect_cache=True)["cache"],
                       tokens[:, 0])
+
+
+# ---------------------------------------------------------------- variable-length batches
+
+def test_plan_varlen_reduces_to_plan_and_meets_target():
+    cfg = _cfg(n_layers=16, d_model=2048, n_heads=32, n_kv_heads=8, head_dim=64, ffn_dim=8192,
+               vocab=128256, prune_layers=list(range(1, 16)))
+    for accel in (1.0, 2.0, 4.0, 8.0):
+        a1, s1 = O.plan(cfg, 512, accel)
+        a2, s2 = O.plan_varlen(cfg, [512], accel)
+        assert a1 == a2 and s2 == [s1]
+        a3, s3 = O.plan_varlen(cfg, [512] * 5, accel)
+        assert s3 == [s1] * 5 and abs(a3 - a1) < 1e-12
+    lengths = [512, 37, 2048, 1, 300]
+    full = sum(O.model_cost(cfg, O.schedule(L, 1.0, 16, cfg.prune_layers, 5)) for L in lengths)
+    prev = 1.0
+    for accel in (1.5, 3.0, 6.0):
+        alpha, scheds = O.plan_varlen(cfg, lengths, accel)
+        cost = sum(O.model_cost(cfg, sc) for sc in scheds)
+        assert cost <= full / accel
+        worse = [O.schedule(L, min(1.0, alpha + 1e-9), 16, cfg.prune_layers, 5) for L in lengths]
+        assert sum(O.model_cost(cfg, sc) for sc in worse) > full / accel or worse == scheds
+        for L, sc in zip(lengths, scheds):
+            assert sc == O.schedule(L, alpha, 16, cfg.prune_layers, 5)
+        assert alpha < prev
+        prev = alpha
+    # the longest sequence dominates the batch cost: its rate is close to its own
+    a_long, _ = O.plan(cfg, 2048, 3.0)
+    a_mix, _ = O.plan_varlen(cfg, lengths, 3.0)
+    assert abs(a_mix - a_long) < 0.05
+    with pytest.raises(ValueError):
+        O.plan_varlen(cfg, [10, 0], 2.0)
+
+
+def test_forward_varlen_runs_each_sequence_at_the_batch_rate():
+    cfg = _cfg()
+    w = _tiny_weights(cfg, seed=11)
+    rng = np.random.default_rng(20)
+    seqs = [rng.integers(0, cfg.vocab, n) for n in (23, 5, 40)]
+    out = O.forward_varlen(cfg, w, seqs, accel=3.0)
+    alpha, scheds = O.plan_varlen(cfg, [23, 5, 40], 3.0)
+    assert out["alpha"] == alpha and out["schedule"] == scheds
+    for b, t in enumerate(seqs):
+        r = O.forward(cfg, w, t[None], alpha=alpha)
+        np.testing.assert_array_equal(out["logits"][b], r["logits"][0])
+        np.testing.assert_array_equal(out["kept_pos"][b], r["kept_pos"][0])
+        assert out["kept_pos"][b][-1] == len(t) - 1
