@@ -153,6 +153,57 @@ def time_oracle(shape, weights_np, tokens, accel, budget_s, max_seqs):
     return n, time.perf_counter() - t0
 
 
+VARLEN_LENGTHS = [128, 256, 384, 512, 640, 768, 896, 512]  # 4096 tokens, 8 sequences
+
+
+def varlen_leg(zsaa, weights, cfg, shape, accel, flush, stream, max_over_ranks, world, steps):
+    """zsaa_forward_varlen on 8 sequences of 128..896 tokens (4096 in all, the
+    headline's token count), against the fixed-length forward of the same batch
+    padded to the longest sequence (B=8, L=896: the cost of padding; its
+    outputs are not those of the unpadded sequences).  A model made for
+    max_L=896 on the same weights; CUDA events on the launch stream, L2 flushed
+    between steps; the variable-length forward launches eagerly."""
+    import numpy as np
+    import torch
+    from paper_2509_01190_gb300 import inputs as I
+    lengths = VARLEN_LENGTHS
+    T, B, Lp = sum(lengths), len(lengths), max(lengths)
+    dev = flush.device
+    model = zsaa.Model(cfg, weights, B, Lp)
+    toks = I.make_tokens(B, Lp, shape.vocab, seed=11)
+    packed = torch.from_numpy(np.concatenate([toks[b, :L] for b, L in enumerate(lengths)])).to(dev)
+    padded = torch.from_numpy(toks).to(dev)
+    sched, alpha = zsaa.zsaa_plan_varlen(model, lengths, accel)
+    n_fin = sum(sc[-1] for sc in sched)
+    lg_v = torch.empty(n_fin, shape.vocab, device=dev, dtype=torch.float32)
+    psched, _ = zsaa.zsaa_plan(model, Lp, accel)
+    lg_p = torch.empty(B, psched[-1], shape.vocab, device=dev, dtype=torch.float32)
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(steps)]
+        for e0, e1 in evs:
+            flush.zero_()
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        zsaa.zsaa_sync(model)
+        return max_over_ranks(sum(a.elapsed_time(b) for a, b in evs) / steps)
+
+    ms_v = timed(lambda: zsaa.zsaa_forward_varlen(model, packed, lengths, accel, lg_v, stream=stream))
+    ms_p = timed(lambda: zsaa.zsaa_forward(model, padded, B, Lp, accel, lg_p, None, stream=stream))
+    model.close()
+    return {"lengths": lengths, "accel": accel, "alpha": alpha, "final_rows": n_fin,
+            "ms_per_step": ms_v, "tokens_per_s": world * T / (ms_v / 1e3),
+            "padded_ms_per_step": ms_p, "padded_real_tokens_per_s": world * T / (ms_p / 1e3),
+            "speedup_vs_padded": ms_p / ms_v,
+            "note": "packed rows, one alpha for the batch (zsaa_plan_varlen); eager launches"}
+
+
 def decode_leg(zsaa, model, weights, shape, B, L, accel, tok_dev, stream, barrier, max_over_ranks,
                world, steps=48, warmup=8):
     """Decode steps after a pruned prefill (CUDA-graph replay, events on the
@@ -459,6 +510,11 @@ def main():
                        "d2h_bytes_per_step": n_logit * 4, "ms_per_step": e2e_s * 1e3,
                        "note": "zsaa_forward_host: pinned host tokens in, host float32 logits out; "
                                "the 256 MiB L2 flush runs inside this span"}
+
+        # ---- variable-length batch: the same 4096 tokens as B x L, in mixed lengths
+        if shape.n_classes == 0 and B * L == 4096:
+            line["varlen"] = varlen_leg(zsaa, weights, cfg, shape, args.accel, flush, stream,
+                                        max_over_ranks, world, args.steps)
 
         # ---- generation over the pruned KV cache (LM head only): B tokens per step
         if not shape.n_classes:

@@ -182,6 +182,42 @@ zsaa_status zsaa_forward_host(zsaa_model* m, const int32_t* token_ids, int B, in
                               double accel, float* logits_out, int32_t* kept_pos_out,
                               zsaa_stream stream);
 
+/* ---- Variable-length batches.
+ *
+ * Sec. 3.4 picks the preservation rate per inference call.  For one call over
+ * sequences of different lengths the library reads it as one alpha for the
+ * whole batch: ZSAA_PLAN_COST bisects (as zsaa_plan) for the largest alpha
+ * whose modelled FLOPs summed over the batch are at most 1/accel of the
+ * unpruned sum, and each sequence then follows Eq. 2 from its own length, so
+ * sequence b keeps N_{l,b} rows after layer l.  ZSAA_PLAN_RATE: alpha = 1/accel.
+ *
+ * zsaa_plan_varlen(_config): lengths host int32 [B] (each >= 1); sched_out
+ * host int [B][n_layers+1], row b = N_{0,b} .. N_{n,b}; alpha_out may be NULL.
+ * Host only, no device work. */
+zsaa_status zsaa_plan_varlen_config(const zsaa_config* cfg, const int32_t* lengths, int B,
+                                    double accel, int* sched_out, double* alpha_out);
+zsaa_status zsaa_plan_varlen(const zsaa_model* m, const int32_t* lengths, int B, double accel,
+                             int* sched_out, double* alpha_out);
+
+/* zsaa_forward_varlen: the pruned prefill of B sequences packed back to back.
+ *   token_ids   : device int32 [T], T = sum of lengths, sequence b after b-1
+ *   lengths     : host int32 [B], each in [1, max_L]; B <= max_B; T <= max_B*max_L
+ *   logits_out  : device float32: LM head: the final kept rows of every
+ *                 sequence, packed in order [sum_b N_{n,b}, vocab]; classifier:
+ *                 [B, n_classes] from each sequence's last kept row
+ *   kept_pos_out: device int32 [sum_b N_{n,b}] (positions within each sequence) or NULL
+ *   opts        : NULL, or the forced_idx / scores_out / idx_out hooks of
+ *                 zsaa_forward_ex with packed layouts: per pruning layer l,
+ *                 indices [sum_b N_{l,b}] (within each sequence's rows) and
+ *                 scores [sum_b N_{l-1,b}]; every other field zero.
+ * A sequence attends only to its own rows.  bf16 models with d_model <= 4096
+ * and lengths <= 12288 (ZSAA_ERR_UNSUPPORTED otherwise).  Runs eagerly; the
+ * row offsets are uploaded from pinned memory the model owns (allocated on the
+ * first call), and the call waits for the previous call's upload to finish. */
+zsaa_status zsaa_forward_varlen(zsaa_model* m, const int32_t* token_ids, const int32_t* lengths,
+                                int B, double accel, float* logits_out, int32_t* kept_pos_out,
+                                const zsaa_forward_opts* opts, zsaa_stream stream);
+
 /* ---- Generation over the pruned KV cache.
  *
  * Sec. 3.3 removes an eliminated row from every later layer, so after a pruned

@@ -61,6 +61,20 @@ __device__ __forceinline__ unsigned long long globaltimer_ns() {
   return t;
 }
 
+// Variable-length batches keep the rows of B sequences packed, sequence b at
+// rows [cu[b], cu[b+1]) (cu[0] = 0, strictly increasing).  Sequence of row r:
+__device__ __forceinline__ int seq_of_row(const int* __restrict__ cu, int B, int r) {
+  int lo = 0, hi = B;  // cu[lo] <= r < cu[hi]
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (__ldg(cu + mid) <= r)
+      lo = mid;
+    else
+      hi = mid;
+  }
+  return lo;
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);

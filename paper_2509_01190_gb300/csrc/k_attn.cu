@@ -48,9 +48,9 @@ __device__ __forceinline__ void load_tile64(uint32_t sbase, const bf16* g, size_
 
 template <int HD>
 __global__ void __launch_bounds__(128)
-    attn_fwd_bf16_kernel(const bf16* __restrict__ qkv, int N, int Hq, int Hkv,
+    attn_fwd_bf16_kernel(const bf16* __restrict__ qkv, int Ns, int Hq, int Hkv,
                          bf16* __restrict__ out, float* __restrict__ lse2, float scale_log2,
-                         int causal) {
+                         int causal, const int* __restrict__ cu) {
   pdl_trigger();
   pdl_wait();
   constexpr int ROWB = HD * 2;
@@ -60,9 +60,14 @@ __global__ void __launch_bounds__(128)
   const uint32_t sK0 = sQ + TILE, sV0 = sQ + 3 * TILE;  // K: 2 buffers, V: 2 buffers
 
   const int qb = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  // fixed length: N = Ns rows per sequence; packed variable length: this
+  // sequence's rows [cu[b], cu[b+1]) (Ns = the longest: grid and lse stride)
+  const size_t row0 = cu ? static_cast<size_t>(cu[b]) : static_cast<size_t>(b) * Ns;
+  const int N = cu ? cu[b + 1] - cu[b] : Ns;
+  if (qb * 64 >= N) return;
   const int g = h / (Hq / Hkv);
   const size_t ld = static_cast<size_t>(Hq + 2 * Hkv) * HD;
-  const bf16* base = qkv + static_cast<size_t>(b) * N * ld;
+  const bf16* base = qkv + row0 * ld;
   const bf16* Qg = base + h * HD;
   const bf16* Kg = base + (Hq + g) * HD;
   const bf16* Vg = base + (Hq + Hkv + g) * HD;
@@ -194,20 +199,20 @@ __global__ void __launch_bounds__(128)
   const float inv_lo = l_lo > 0.f ? 1.f / l_lo : 0.f, inv_hi = l_hi > 0.f ? 1.f / l_hi : 0.f;
   const size_t ldo = static_cast<size_t>(Hq) * HD;
   if (i_lo < N) {
-    bf16* orow = out + (static_cast<size_t>(b) * N + i_lo) * ldo + h * HD;
+    bf16* orow = out + (row0 + i_lo) * ldo + h * HD;
 #pragma unroll
     for (int nt = 0; nt < HD / 8; ++nt)
       *reinterpret_cast<uint32_t*>(orow + nt * 8 + 2 * tig) =
           pack_bf16x2(o[nt][0] * inv_lo, o[nt][1] * inv_lo);
-    if (tig == 0) lse2[(static_cast<size_t>(b) * Hq + h) * N + i_lo] = m_lo + log2f(l_lo);
+    if (tig == 0) lse2[(static_cast<size_t>(b) * Hq + h) * Ns + i_lo] = m_lo + log2f(l_lo);
   }
   if (i_hi < N) {
-    bf16* orow = out + (static_cast<size_t>(b) * N + i_hi) * ldo + h * HD;
+    bf16* orow = out + (row0 + i_hi) * ldo + h * HD;
 #pragma unroll
     for (int nt = 0; nt < HD / 8; ++nt)
       *reinterpret_cast<uint32_t*>(orow + nt * 8 + 2 * tig) =
           pack_bf16x2(o[nt][2] * inv_hi, o[nt][3] * inv_hi);
-    if (tig == 0) lse2[(static_cast<size_t>(b) * Hq + h) * N + i_hi] = m_hi + log2f(l_hi);
+    if (tig == 0) lse2[(static_cast<size_t>(b) * Hq + h) * Ns + i_hi] = m_hi + log2f(l_hi);
   }
 }
 
@@ -471,7 +476,8 @@ cudaError_t set_smem(Kern k, int bytes) {
 }  // namespace
 
 cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, int Hkv, int hd,
-                             void* out, float* lse, int causal, cudaStream_t s) {
+                             void* out, float* lse, int causal, cudaStream_t s, const int* cu) {
+  if (cu != nullptr && dtype != ZSAA_BF16) return cudaErrorInvalidValue;
   const float scale_log2 = kLog2e / sqrtf(static_cast<float>(hd));
   if (dtype == ZSAA_F32) {
     dim3 grid((N + 3) / 4, Hq, B);
@@ -485,13 +491,13 @@ cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, i
     static cudaError_t e = set_smem(attn_fwd_bf16_kernel<64>, smem);
     if (e != cudaSuccess) return e;
     ZSAA_LAUNCH(attn_fwd_bf16_kernel<64>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), N, Hq, Hkv,
-                                                      static_cast<bf16*>(out), lse, scale_log2, causal);
+                                                      static_cast<bf16*>(out), lse, scale_log2, causal, cu);
   } else if (hd == 128) {
     const int smem = 5 * 64 * 256;
     static cudaError_t e = set_smem(attn_fwd_bf16_kernel<128>, smem);
     if (e != cudaSuccess) return e;
     ZSAA_LAUNCH(attn_fwd_bf16_kernel<128>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), N, Hq, Hkv,
-                                                       static_cast<bf16*>(out), lse, scale_log2, causal);
+                                                       static_cast<bf16*>(out), lse, scale_log2, causal, cu);
   } else {
     return cudaErrorInvalidValue;
   }
@@ -512,11 +518,13 @@ size_t colmass_parts_elems(int B, int N, int Hq, int Hkv) {
 namespace {
 cudaError_t colmass_parts(int dtype, const void* qkv, const float* lse, const float* vnorm, int B,
                           int N, int Hq, int Hkv, int hd, int weight_vnorm, float* parts, int* n_qc,
-                          int* status, int causal, cudaStream_t s) {
+                          int* status, int causal, cudaStream_t s, const int* cu = nullptr,
+                          int rows = 0) {
   // tensor-core path (with precomputed norms when they are needed)
   if (dtype == ZSAA_BF16 && status != nullptr && (!weight_vnorm || vnorm != nullptr))
     return launch_colmass_tc(qkv, lse, weight_vnorm ? vnorm : nullptr, B, N, Hq, Hkv, hd, parts,
-                             status, n_qc, causal, s);
+                             status, n_qc, causal, s, cu, rows);
+  if (cu != nullptr) return cudaErrorInvalidValue;  // packed sequences: tensor-core path only
   const float scale_log2 = kLog2e / sqrtf(static_cast<float>(hd));
   if (dtype == ZSAA_F32) {
     *n_qc = 1;
@@ -562,9 +570,11 @@ cudaError_t launch_colmass(int dtype, const void* qkv, const float* lse, int B, 
 
 cudaError_t launch_position_parts(int dtype, const void* qkv, const float* lse, const float* vnorm,
                                   int B, int N, int Hq, int Hkv, int hd, int mode, float* parts,
-                                  int* n_qc, int* status, int causal, cudaStream_t s) {
+                                  int* n_qc, int* status, int causal, cudaStream_t s, const int* cu,
+                                  int rows) {
   return colmass_parts(dtype, qkv, lse, vnorm, B, N, Hq, Hkv, hd,
-                       mode == ZSAA_SCORE_SOFTSCORE_VNORM ? 1 : 0, parts, n_qc, status, causal, s);
+                       mode == ZSAA_SCORE_SOFTSCORE_VNORM ? 1 : 0, parts, n_qc, status, causal, s,
+                       cu, rows);
 }
 
 cudaError_t launch_position_scores(int dtype, const void* qkv, const float* lse, const float* vnorm,

@@ -51,6 +51,7 @@ struct CmArgs {
   float* parts;        // [per][B][G][N]
   int B, N, Hq, Hkv, ld, n_kb, total, weight_vnorm;
   int causal;  // 0: bidirectional (every query block, no causal mask)
+  const int* cu;  // packed sequences of different lengths: rows [cu[b], cu[b+1]); N = the longest
   float scale_log2;
   int* status;
 };
@@ -72,6 +73,31 @@ __device__ __forceinline__ void cm_tile(int t, const CmArgs& a, int& b, int& g, 
   r /= per;
   g = r % a.Hkv;
   b = r / a.Hkv;
+}
+
+// Rows of sequence b: first packed row and length.
+__device__ __forceinline__ void cm_seq(const CmArgs& a, int b, int& row0, int& n) {
+  if (a.cu) {
+    row0 = a.cu[b];
+    n = a.cu[b + 1] - row0;
+  } else {
+    row0 = b * a.N;
+    n = a.N;
+  }
+}
+
+// Tile t holds keys of its sequence (a shorter sequence has fewer key blocks).
+__device__ __forceinline__ bool cm_live(int t, const CmArgs& a) {
+  int b, g, hh, kb, row0, n;
+  cm_tile(t, a, b, g, hh, kb);
+  cm_seq(a, b, row0, n);
+  return kb * CM_BM < n;
+}
+
+// The next tile of this CTA at or after t that holds keys (a.total if none).
+__device__ __forceinline__ int cm_next(int t, const CmArgs& a) {
+  while (t < a.total && !cm_live(t, a)) t += gridDim.x;
+  return t < a.total ? t : a.total;
 }
 
 template <int HD>
@@ -123,11 +149,12 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
     if (lane == 0) {
       uint32_t it = 0, tiles = 0, issued_last = 0;
       bool ok = true;
-      for (int t = blockIdx.x; t < a.total && ok; t += gridDim.x, ++tiles) {
-        int b, g, hh, kb;
+      for (int t = cm_next(blockIdx.x, a); t < a.total && ok; t = cm_next(t + gridDim.x, a), ++tiles) {
+        int b, g, hh, kb, row0, n_b;
         cm_tile(t, a, b, g, hh, kb);
+        cm_seq(a, b, row0, n_b);
+        const int n_qb = (n_b + CM_BN - 1) / CM_BN;
         const int h = g * (a.Hq / a.Hkv) + hh;
-        const int row0 = b * a.N;
         // K tile (two buffers): wait until the MMAs of two tiles ago are done with it
         const int kbuf = tiles & 1;
         if (!mbar_wait_ab(&kempty[kbuf], ((tiles >> 1) & 1) ^ 1, a.status, abort_flag)) break;
@@ -135,7 +162,7 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
         for (int c = 0; c < C::CHUNKS; ++c)
           tma_load_2d(sK + kbuf * C::TILE_BYTES + c * (C::TILE_BYTES / C::CHUNKS), &tm,
                       (a.Hq + g) * HD + c * 64, row0 + kb * CM_BM, &kfull[kbuf]);
-        for (int qb = a.causal ? kb : 0; qb < a.n_kb; ++qb, ++it) {
+        for (int qb = a.causal ? kb : 0; qb < n_qb; ++qb, ++it) {
           const int s = it % CM_STAGES;
           const uint32_t ph = (it / CM_STAGES) & 1;
           if (!mbar_wait_ab(&empty[s], ph ^ 1, a.status, abort_flag)) {
@@ -164,14 +191,16 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
       uint32_t it = 0, tiles = 0;
       int i = 0;
       bool ok = true;
-      for (int t = blockIdx.x; t < a.total && ok; t += gridDim.x, ++tiles) {
-        int b, g, hh, kb;
+      for (int t = cm_next(blockIdx.x, a); t < a.total && ok; t = cm_next(t + gridDim.x, a), ++tiles) {
+        int b, g, hh, kb, row0, n_b;
         cm_tile(t, a, b, g, hh, kb);
+        cm_seq(a, b, row0, n_b);
+        const int n_qb = (n_b + CM_BN - 1) / CM_BN;
         const int kbuf = tiles & 1;
         if (!mbar_wait_ab(&kfull[kbuf], (tiles >> 1) & 1, a.status, abort_flag)) break;
         tc_fence_after();
         const uint32_t k_base = smem_u32(sK + kbuf * C::TILE_BYTES);
-        for (int qb = a.causal ? kb : 0; qb < a.n_kb; ++qb, ++it, ++i) {
+        for (int qb = a.causal ? kb : 0; qb < n_qb; ++qb, ++it, ++i) {
           const int ab = i & 1;
           const uint32_t use = static_cast<uint32_t>(i >> 1);
           if (!mbar_wait_ab(&acc_empty[ab], (use & 1) ^ 1, a.status, abort_flag)) {
@@ -209,12 +238,13 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
     // fetch the normalisers of step (t, qb) into s_lse[buf]
     auto fetch = [&](int t, int qb, int buf) {
       if (et < CM_BN) {
-        int b, g, hh, kb;
+        int b, g, hh, kb, row0, n_b;
         cm_tile(t, a, b, g, hh, kb);
+        cm_seq(a, b, row0, n_b);
         const int h = g * (a.Hq / a.Hkv) + hh;
         const int q = qb * CM_BN + et;
         float* dst = s_lse + buf * CM_BN + et;
-        if (q < a.N) {
+        if (q < n_b) {
           asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)),
                        "l"(a.lse2 + (static_cast<size_t>(b) * a.Hq + h) * a.N + q)
                        : "memory");
@@ -226,28 +256,34 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
     };
     int i = 0;
     bool ok = true;
-    if (static_cast<int>(blockIdx.x) < a.total) {
+    const int t_first = cm_next(blockIdx.x, a);
+    if (t_first < a.total) {
       int b, g, hh, kb;
-      cm_tile(blockIdx.x, a, b, g, hh, kb);
-      fetch(blockIdx.x, a.causal ? kb : 0, 0);
+      cm_tile(t_first, a, b, g, hh, kb);
+      fetch(t_first, a.causal ? kb : 0, 0);
     }
-    for (int t = blockIdx.x; t < a.total; t += gridDim.x) {
-      int b, g, hh, kb;
+    for (int t = t_first; t < a.total; t = cm_next(t + gridDim.x, a)) {
+      int b, g, hh, kb, row0, n_b;
       cm_tile(t, a, b, g, hh, kb);
+      cm_seq(a, b, row0, n_b);
+      const int n_qb = (n_b + CM_BN - 1) / CM_BN;
       const int key = kb * CM_BM + krow;
       float acc = 0.f;
-      for (int qb = a.causal ? kb : 0; qb < a.n_kb; ++qb, ++i) {
+      for (int qb = a.causal ? kb : 0; qb < n_qb; ++qb, ++i) {
         const int ab = i & 1;
         const uint32_t use = static_cast<uint32_t>(i >> 1);
         cp_async_wait<0>();
         // this step's normalisers are in s_lse[ab]; every warp is done with step i-1
         asm volatile("bar.sync 1, %0;" ::"n"(CM_EPI_WARPS * 32) : "memory");
-        if (qb + 1 < a.n_kb) {
+        if (qb + 1 < n_qb) {
           fetch(t, qb + 1, ab ^ 1);
-        } else if (t + static_cast<int>(gridDim.x) < a.total) {
-          int b2, g2, hh2, kb2;
-          cm_tile(t + gridDim.x, a, b2, g2, hh2, kb2);
-          fetch(t + gridDim.x, a.causal ? kb2 : 0, ab ^ 1);
+        } else {
+          const int tn = cm_next(t + gridDim.x, a);
+          if (tn < a.total) {
+            int b2, g2, hh2, kb2;
+            cm_tile(tn, a, b2, g2, hh2, kb2);
+            fetch(tn, a.causal ? kb2 : 0, ab ^ 1);
+          }
         }
         const float* L = s_lse + ab * CM_BN;
         ok = ok && __all_sync(0xffffffffu, mbar_wait_ab(&acc_full[ab], use & 1, a.status, abort_flag));
@@ -264,14 +300,14 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
             tmem_ld_wait();
             const int qc0 = half * 64 + c;
             const int q0 = qb * CM_BN + qc0;
-            if ((!a.causal || q0 > key) && q0 + 32 <= a.N) {  // whole chunk inside the mask
+            if ((!a.causal || q0 > key) && q0 + 32 <= n_b) {  // whole chunk inside the mask
 #pragma unroll
               for (int e = 0; e < 32; ++e) acc += ex2_ftz(__uint_as_float(r[e]) * a.scale_log2 - L[qc0 + e]);
             } else {
 #pragma unroll
               for (int e = 0; e < 32; ++e) {
                 const int q = q0 + e;
-                if ((!a.causal || q >= key) && q < a.N)
+                if ((!a.causal || q >= key) && q < n_b)
                   acc += ex2_ftz(__uint_as_float(r[e]) * a.scale_log2 - L[qc0 + e]);
               }
             }
@@ -284,9 +320,9 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
       // add the two column halves (fixed order: half 0 + half 1)
       if (half == 1) s_half[krow] = acc;
       asm volatile("bar.sync 1, %0;" ::"n"(CM_EPI_WARPS * 32) : "memory");
-      if (half == 0 && key < a.N) {
+      if (half == 0 && key < n_b) {
         float v = acc + s_half[krow];
-        if (a.weight_vnorm) v *= a.vnorm[(static_cast<size_t>(b) * a.N + key) * a.Hkv + g];
+        if (a.weight_vnorm) v *= a.vnorm[(static_cast<size_t>(row0) + key) * a.Hkv + g];
         a.parts[((static_cast<size_t>(hh) * a.B + b) * a.Hkv + g) * a.N + key] = v;
       }
       // s_half is rewritten only after the next tile's first barrier
@@ -331,13 +367,14 @@ cudaError_t run_cm(const CUtensorMap& tm, const CmArgs& a, int sms, cudaStream_t
 
 cudaError_t launch_colmass_tc(const void* qkv, const float* lse, const float* vnorm, int B, int N,
                               int Hq, int Hkv, int hd, float* parts, int* status, int* n_chunks,
-                              int causal, cudaStream_t s) {
+                              int causal, cudaStream_t s, const int* cu, int rows) {
   if (hd != 64 && hd != 128) return cudaErrorInvalidValue;
   const int ld = (Hq + 2 * Hkv) * hd;
   EncodeTiledFn enc = get_encode_tiled();
   if (enc == nullptr) return cudaErrorInvalidValue;
   CUtensorMap tm;
-  cuuint64_t dims[2] = {static_cast<cuuint64_t>(ld), static_cast<cuuint64_t>(B) * N};
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(ld),
+                        cu ? static_cast<cuuint64_t>(rows) : static_cast<cuuint64_t>(B) * N};
   cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
   cuuint32_t box[2] = {64, static_cast<cuuint32_t>(CM_BM)};
   cuuint32_t es[2] = {1, 1};
@@ -358,6 +395,7 @@ cudaError_t launch_colmass_tc(const void* qkv, const float* lse, const float* vn
   a.total = a.n_kb * B * Hq;
   a.weight_vnorm = vnorm != nullptr;
   a.causal = causal;
+  a.cu = cu;
   a.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(hd));
   a.status = status;
   *n_chunks = Hq / Hkv;

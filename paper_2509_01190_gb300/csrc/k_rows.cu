@@ -173,29 +173,36 @@ constexpr int kSelThreads = 1024;
 // scores_out when it is not null); otherwise they are read from `scores`.
 template <bool FROM_PARTS>
 __global__ void __launch_bounds__(kSelThreads)
-    select_topk_kernel(const float* __restrict__ scores, int N, int k, int force_last,
+    select_topk_kernel(const float* __restrict__ scores, int Ns, int ks, int force_last,
                        int32_t* __restrict__ idx_out, const float* __restrict__ parts, int n_qc,
-                       int B, int G, float* __restrict__ scores_out) {
+                       int B, int G, float* __restrict__ scores_out, const int* __restrict__ cu_in,
+                       const int* __restrict__ cu_out) {
   pdl_trigger();
   pdl_wait();
   const int b = blockIdx.x;
+  // fixed length: N = Ns rows in, k = ks kept per sequence; variable length
+  // (FROM_PARTS only): this sequence's counts from the packed row offsets,
+  // partials still at stride Ns (the longest sequence)
+  const int N = cu_in ? cu_in[b + 1] - cu_in[b] : Ns;
+  const int k = cu_out ? cu_out[b + 1] - cu_out[b] : ks;
+  const size_t sc_row0 = cu_in ? static_cast<size_t>(cu_in[b]) : static_cast<size_t>(b) * Ns;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int nwarps = kSelThreads / 32;
   extern __shared__ float sscore[];
   const float* s = scores + static_cast<size_t>(b) * N;
   if (FROM_PARTS) {
-    const size_t plane = static_cast<size_t>(B) * G * N;
+    const size_t plane = static_cast<size_t>(B) * G * Ns;
     for (int j = tid; j < N; j += kSelThreads) {
       float acc = 0.f;
       for (int qc = 0; qc < n_qc; ++qc)
-        for (int g = 0; g < G; ++g) acc += parts[qc * plane + (static_cast<size_t>(b) * G + g) * N + j];
+        for (int g = 0; g < G; ++g) acc += parts[qc * plane + (static_cast<size_t>(b) * G + g) * Ns + j];
       sscore[j] = acc;
-      if (scores_out != nullptr) scores_out[static_cast<size_t>(b) * N + j] = acc;
+      if (scores_out != nullptr) scores_out[sc_row0 + j] = acc;
     }
     __syncthreads();
     s = sscore;
   }
-  int32_t* out = idx_out + static_cast<size_t>(b) * k;
+  int32_t* out = idx_out + (cu_out ? static_cast<size_t>(cu_out[b]) : static_cast<size_t>(b) * k);
   const int n_cand = force_last ? N - 1 : N;
   const int need = force_last ? k - 1 : k;
 
@@ -341,7 +348,9 @@ __global__ void rows_norm_bf16_kernel(const uint4* __restrict__ src, const int32
                                       int k, const int32_t* __restrict__ pos_in, int rows, int vec,
                                       const uint4* __restrict__ w, float eps,
                                       uint4* __restrict__ h_out, uint4* __restrict__ x_out,
-                                      int32_t* __restrict__ pos_out, int* status) {
+                                      int32_t* __restrict__ pos_out, int* status,
+                                      const int* __restrict__ cu_src, const int* __restrict__ cu_dst,
+                                      int nseq) {
   pdl_trigger();
   pdl_wait();
   const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
@@ -356,15 +365,25 @@ __global__ void rows_norm_bf16_kernel(const uint4* __restrict__ src, const int32
       t = 0;
     }
     srow = static_cast<size_t>(t);
-    p = r % L;
+    p = cu_dst ? r - __ldg(cu_dst + seq_of_row(cu_dst, nseq, r)) : r % L;
   } else {
-    const int b = r / k;
+    int b, n_b;
+    size_t row0;
+    if (cu_dst) {  // packed sequences of different lengths
+      b = seq_of_row(cu_dst, nseq, r);
+      row0 = static_cast<size_t>(__ldg(cu_src + b));
+      n_b = __ldg(cu_src + b + 1) - __ldg(cu_src + b);
+    } else {
+      b = r / k;
+      row0 = static_cast<size_t>(b) * N;
+      n_b = N;
+    }
     int j = idx[r];
-    if (j < 0 || j >= N) {
+    if (j < 0 || j >= n_b) {
       if (lane == 0 && status != nullptr) atomicOr(status, kStatusBadIndex);
       j = 0;
     }
-    srow = static_cast<size_t>(b) * N + j;
+    srow = row0 + j;
     p = pos_in[srow];
   }
   const uint4* sr = src + srow * vec;
@@ -434,13 +453,14 @@ __global__ void rope_f32_kernel(float* __restrict__ qkv, int rows, int ld, int r
 template <typename T>
 __global__ void cls_head_kernel(const T* __restrict__ h, int N, int d,
                                 const T* __restrict__ norm_w, float eps, const T* __restrict__ W,
-                                int n_classes, float* __restrict__ out) {
+                                int n_classes, float* __restrict__ out, const int* __restrict__ cu) {
   pdl_trigger();
   pdl_wait();
   extern __shared__ float xs[];  // d floats
   __shared__ float red[32];
   const int b = blockIdx.x;
-  const T* row = h + (static_cast<size_t>(b) * N + (N - 1)) * d;
+  const size_t last = cu ? static_cast<size_t>(cu[b + 1] - 1) : static_cast<size_t>(b) * N + (N - 1);
+  const T* row = h + last * d;
   float ss = 0.f;
   for (int i = threadIdx.x; i < d; i += blockDim.x) {
     float v = to_f(row[i]);
@@ -513,30 +533,34 @@ cudaError_t launch_row_norm(int dtype, const void* h, int rows, int d, float* sc
 cudaError_t launch_select(const float* scores, int B, int N, int k, int force_last, int32_t* idx,
                           cudaStream_t s) {
   ZSAA_LAUNCH(select_topk_kernel<false>, dim3(B), dim3(kSelThreads), 0, s, scores, N, k, force_last,
-              idx, static_cast<const float*>(nullptr), 0, B, 0, static_cast<float*>(nullptr));
+              idx, static_cast<const float*>(nullptr), 0, B, 0, static_cast<float*>(nullptr),
+              static_cast<const int*>(nullptr), static_cast<const int*>(nullptr));
   return cudaGetLastError();
 }
 
 cudaError_t launch_select_parts(const float* parts, int n_qc, int B, int G, int N, int k,
-                                int force_last, int32_t* idx, float* scores_out, cudaStream_t s) {
+                                int force_last, int32_t* idx, float* scores_out, cudaStream_t s,
+                                const int* cu_in, const int* cu_out) {
   const size_t smem = static_cast<size_t>(N) * sizeof(float);
   static cudaError_t attr = cudaFuncSetAttribute(select_topk_kernel<true>,
                                                  cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                  static_cast<int>(kSelectPartsMaxN * sizeof(float)));
   if (attr != cudaSuccess) return attr;
   ZSAA_LAUNCH(select_topk_kernel<true>, dim3(B), dim3(kSelThreads), smem, s,
-              static_cast<const float*>(nullptr), N, k, force_last, idx, parts, n_qc, B, G, scores_out);
+              static_cast<const float*>(nullptr), N, k, force_last, idx, parts, n_qc, B, G, scores_out,
+              cu_in, cu_out);
   return cudaGetLastError();
 }
 
 cudaError_t launch_rows_norm(const void* src, const int32_t* tok, int vocab, int L,
                              const int32_t* idx, int N, int k, const int32_t* pos_in, int rows,
                              int d, const void* w, float eps, void* h_out, void* x_out,
-                             int32_t* pos_out, int* status, cudaStream_t s) {
+                             int32_t* pos_out, int* status, cudaStream_t s, const int* cu_src,
+                             const int* cu_dst, int nseq) {
   ZSAA_LAUNCH(rows_norm_bf16_kernel, dim3(row_blocks(rows)), dim3(32 * kWarpsPerBlock), 0, s,
               static_cast<const uint4*>(src), tok, vocab, L, idx, N, k, pos_in, rows, d / 8,
               static_cast<const uint4*>(w), eps, static_cast<uint4*>(h_out),
-              static_cast<uint4*>(x_out), pos_out, status);
+              static_cast<uint4*>(x_out), pos_out, status, cu_src, cu_dst, nseq);
   return cudaGetLastError();
 }
 
@@ -560,16 +584,17 @@ cudaError_t launch_rope_f32(float* qkv, int rows, int ld, int rope_cols, int hd,
 }
 
 cudaError_t launch_cls_head(int dtype, const void* h, int B, int N, int d, const void* norm_w,
-                            float eps, const void* W, int n_classes, float* out, cudaStream_t s) {
+                            float eps, const void* W, int n_classes, float* out, cudaStream_t s,
+                            const int* cu) {
   const size_t smem = static_cast<size_t>(d) * sizeof(float);
   if (dtype == ZSAA_BF16)
     ZSAA_LAUNCH(cls_head_kernel<bf16>, dim3(B), dim3(256), smem, s, static_cast<const bf16*>(h), N, d,
                                                static_cast<const bf16*>(norm_w), eps,
-                                               static_cast<const bf16*>(W), n_classes, out);
+                                               static_cast<const bf16*>(W), n_classes, out, cu);
   else
     ZSAA_LAUNCH(cls_head_kernel<float>, dim3(B), dim3(256), smem, s, static_cast<const float*>(h), N, d,
                                                 static_cast<const float*>(norm_w), eps,
-                                                static_cast<const float*>(W), n_classes, out);
+                                                static_cast<const float*>(W), n_classes, out, cu);
   return cudaGetLastError();
 }
 

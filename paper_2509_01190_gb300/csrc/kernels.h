@@ -19,17 +19,27 @@ cudaError_t launch_select(const float* scores, int B, int N, int k, int force_la
 // Top-k from column-mass partials parts[n_qc][B][G][N] (scores summed in shared
 // memory, copied to scores_out when not null); N <= kSelectPartsMaxN.
 constexpr int kSelectPartsMaxN = 12288;
+// Variable length (cu_in / cu_out: packed row offsets [B+1] before / after the
+// selection): sequence b has cu_in[b+1]-cu_in[b] candidates, keeps
+// cu_out[b+1]-cu_out[b], partials at stride N (the longest), idx and scores
+// written packed at cu_out[b] / cu_in[b].
 cudaError_t launch_select_parts(const float* parts, int n_qc, int B, int G, int N, int k,
-                                int force_last, int32_t* idx, float* scores_out, cudaStream_t s);
+                                int force_last, int32_t* idx, float* scores_out, cudaStream_t s,
+                                const int* cu_in = nullptr, const int* cu_out = nullptr);
 // bf16 rows: h_out[r] = source row, x_out[r] = RMSNorm(h_out[r]) * w, pos_out[r].
 // Embedding when idx == nullptr (rows = B*L, source row tok[r] of E);
 // otherwise compaction (rows = B*k, source row b*N + idx[r] of h).
 // d % 8 == 0 and d <= kRowsNormMaxD.
 constexpr int kRowsNormMaxD = 8 * 32 * 16;
+// Variable length: cu_dst (offsets of the written rows; nseq sequences) gives
+// the sequence of a row and, for the embedding, pos = r - cu_dst[b]; cu_src
+// (offsets of the source rows) places compaction index j at row cu_src[b] + j.
 cudaError_t launch_rows_norm(const void* src, const int32_t* tok, int vocab, int L,
                              const int32_t* idx, int N, int k, const int32_t* pos_in, int rows,
                              int d, const void* w, float eps, void* h_out, void* x_out,
-                             int32_t* pos_out, int* status, cudaStream_t s);
+                             int32_t* pos_out, int* status, cudaStream_t s,
+                             const int* cu_src = nullptr, const int* cu_dst = nullptr,
+                             int nseq = 0);
 cudaError_t launch_gather(const void* src, int B, int N, int k, int row_bytes, const int32_t* idx,
                           void* dst, const int32_t* pos_in, int32_t* pos_out, int* status,
                           cudaStream_t s);
@@ -37,7 +47,8 @@ cudaError_t launch_rope_f32(float* qkv, int rows, int ld, int rope_cols, int hd,
                             const int32_t* pos, const float* cos_t, const float* sin_t,
                             cudaStream_t s);
 cudaError_t launch_cls_head(int dtype, const void* h, int B, int N, int d, const void* norm_w,
-                            float eps, const void* W, int n_classes, float* out, cudaStream_t s);
+                            float eps, const void* W, int n_classes, float* out, cudaStream_t s,
+                            const int* cu = nullptr);  // cu: last row of b is cu[b+1]-1
 
 // ---- GEMMs (k_gemm_tc.cu, k_gemm_simt.cu)
 enum Epilogue : int { kEpiStore = 0, kEpiResid = 1, kEpiSwiGLU = 2, kEpiStoreF32 = 3, kEpiRope = 4 };
@@ -94,8 +105,11 @@ cudaError_t launch_gemm_f32(const float* A, int lda, const float* W, const float
 // ---- attention (k_attn.cu)
 // causal = 0: bidirectional (Eq. 1 with M = 0); the column-mass kernels below
 // take the same flag.
+// cu (bf16 only): packed sequences of different lengths, rows [cu[b], cu[b+1]);
+// N is then the longest length (grid size and the stride of lse).
 cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, int Hkv, int hd,
-                             void* out, float* lse, int causal, cudaStream_t s);
+                             void* out, float* lse, int causal, cudaStream_t s,
+                             const int* cu = nullptr);
 // Column mass C[B, Hkv, N] (via partial sums in `parts`, which must hold
 // colmass_parts_elems(B, N, Hq, Hkv) floats).  bf16 with a status word runs
 // the tensor-core kernel (k_colmass_tc.cu); otherwise the mma.sync / fp32 ones.
@@ -117,12 +131,15 @@ cudaError_t launch_position_scores(int dtype, const void* qkv, const float* lse,
 // receives the number of partial chunks.
 cudaError_t launch_position_parts(int dtype, const void* qkv, const float* lse, const float* vnorm,
                                   int B, int N, int Hq, int Hkv, int hd, int mode, float* parts,
-                                  int* n_qc, int* status, int causal, cudaStream_t s);
+                                  int* n_qc, int* status, int causal, cudaStream_t s,
+                                  const int* cu = nullptr, int rows = 0);
 // Tensor-core column-mass partials: parts[Hq/Hkv][B][Hkv][N] (per head of the
-// group), times vnorm when it is not NULL; hd 64 or 128.
+// group), times vnorm when it is not NULL; hd 64 or 128.  With cu: packed
+// sequences of different lengths (rows [cu[b], cu[b+1]), `rows` in all, N the
+// longest); vnorm is then per packed row.
 cudaError_t launch_colmass_tc(const void* qkv, const float* lse, const float* vnorm, int B, int N,
                               int Hq, int Hkv, int hd, float* parts, int* status, int* n_chunks,
-                              int causal, cudaStream_t s);
+                              int causal, cudaStream_t s, const int* cu = nullptr, int rows = 0);
 
 // ---- generation over the pruned KV cache (k_decode.cu)
 // Cache of one layer: K and V bf16 [B, Hkv, cap, hd], positions int32 [B, cap].

@@ -109,6 +109,45 @@ zsaa_status plan_impl(const zsaa_config& c, int L, double accel, int* sched, dou
   return ZSAA_OK;
 }
 
+// One rate for B sequences of different lengths (R17): the "cost" mode bisects
+// on the modelled FLOPs summed over the batch; each sequence then follows
+// Eq. 2 from its own length.  sched: [B][n_layers + 1].  Sums stay exact
+// integers below 2^53, so the oracle's planner agrees bit for bit.
+zsaa_status plan_varlen_impl(const zsaa_config& c, const int32_t* lengths, int B, double accel,
+                             int* sched, double* alpha_out) {
+  if (!(accel >= 1.0)) return fail(ZSAA_ERR_INVALID_ARG, "accel must be >= 1 (got %g)", accel);
+  if (B < 1 || lengths == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "need B >= 1 lengths");
+  for (int b = 0; b < B; ++b)
+    if (lengths[b] < 1) return fail(ZSAA_ERR_INVALID_ARG, "length %d of sequence %d is < 1", lengths[b], b);
+  const int n1 = c.n_layers + 1;
+  auto fill = [&](double a) {
+    long long total = 0;
+    for (int b = 0; b < B; ++b) {
+      eq2_schedule(c, lengths[b], a, sched + static_cast<size_t>(b) * n1);
+      total += model_cost(c, sched + static_cast<size_t>(b) * n1);
+    }
+    return total;
+  };
+  double alpha = 1.0;
+  if (c.plan_mode == ZSAA_PLAN_RATE) {
+    alpha = 1.0 / accel;
+  } else if (accel != 1.0) {
+    const double target = static_cast<double>(fill(1.0)) / accel;
+    double lo = 0.0, hi = 1.0;
+    for (int it = 0; it < 60; ++it) {
+      const double mid = 0.5 * (lo + hi);
+      if (static_cast<double>(fill(mid)) <= target)
+        lo = mid;
+      else
+        hi = mid;
+    }
+    alpha = lo;
+  }
+  fill(alpha);
+  if (alpha_out) *alpha_out = alpha;
+  return ZSAA_OK;
+}
+
 zsaa_status validate_config(const zsaa_config& c) {
   if (c.n_layers < 1 || c.n_layers > 64) return fail(ZSAA_ERR_INVALID_ARG, "n_layers must be 1..64");
   if (c.dtype != ZSAA_F32 && c.dtype != ZSAA_BF16) return fail(ZSAA_ERR_INVALID_ARG, "bad dtype");
@@ -278,6 +317,11 @@ struct zsaa_model {
   float* stage_logits = nullptr;
   int32_t* stage_pos = nullptr;
   size_t stage_logits_cap = 0;
+  // packed-sequence row offsets of zsaa_forward_varlen (device, and the pinned
+  // host copy they are uploaded from; the event guards its reuse)
+  int32_t* vl_cu = nullptr;
+  int32_t* vl_cu_host = nullptr;
+  cudaEvent_t vl_done = nullptr;
   // tracing (zsaa_trace_begin / _end)
   struct TraceRec {
     int cls;
@@ -385,6 +429,9 @@ void free_model(zsaa_model* m) {
                   m->stage_pos};
   for (void* p : ptrs)
     if (p) cudaFree(p);
+  if (m->vl_cu) cudaFree(m->vl_cu);
+  if (m->vl_cu_host) cudaFreeHost(m->vl_cu_host);
+  if (m->vl_done) cudaEventDestroy(m->vl_done);
   delete m;
 }
 
@@ -708,6 +755,228 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
   }
   if (kept_pos)
     ZCK(cudaMemcpyAsync(kept_pos, m->pos[cur], sizeof(int32_t) * M, cudaMemcpyDeviceToDevice, s));
+#undef TRACE
+  return ZSAA_OK;
+}
+
+// Pruned prefill of B sequences of different lengths packed back to back
+// (sequence b at rows [cu_l[b], cu_l[b+1]) of layer l's buffers).  The dense
+// steps (GEMMs, norms) run on all packed rows at once; attention, column mass,
+// selection and compaction take the offsets.  bf16 and the fused row path only.
+zsaa_status run_forward_varlen(zsaa_model* m, const int32_t* tok, const int32_t* lengths, int B,
+                               double accel, float* logits, int32_t* kept_pos,
+                               const zsaa_forward_opts* opts, cudaStream_t s) {
+  const zsaa_config& c = m->cfg;
+  const int d = c.d_model, hd = c.head_dim, Hq = c.n_heads, Hkv = c.n_kv_heads, n = c.n_layers;
+  if (c.dtype != ZSAA_BF16 || d % 8 != 0 || d > kRowsNormMaxD)
+    return fail(ZSAA_ERR_UNSUPPORTED, "variable-length batches need a bf16 model with d_model <= %d", kRowsNormMaxD);
+  if (tok == nullptr || logits == nullptr || lengths == nullptr)
+    return fail(ZSAA_ERR_INVALID_ARG, "null token, lengths or logits pointer");
+  if (B < 1 || B > m->max_B) return fail(ZSAA_ERR_INVALID_ARG, "B=%d outside [1,%d]", B, m->max_B);
+  if (opts && (opts->hidden_out || opts->n_layers_run || opts->hidden_in || opts->pos_in ||
+               opts->first_layer || opts->plan_L))
+    return fail(ZSAA_ERR_INVALID_ARG, "variable-length forwards take only the forced_idx/scores_out/idx_out hooks");
+  long long T0 = 0;
+  for (int b = 0; b < B; ++b) {
+    if (lengths[b] < 1 || lengths[b] > m->max_L)
+      return fail(ZSAA_ERR_INVALID_ARG, "length %d of sequence %d outside [1,%d]", lengths[b], b, m->max_L);
+    T0 += lengths[b];
+  }
+  if (T0 > static_cast<long long>(m->max_B) * m->max_L)
+    return fail(ZSAA_ERR_INVALID_ARG, "%lld packed rows exceed max_B*max_L", T0);
+  const int n1 = n + 1;
+  std::vector<int> sched(static_cast<size_t>(B) * n1);
+  double alpha = 1.0;
+  zsaa_status st = plan_varlen_impl(c, lengths, B, accel, sched.data(), &alpha);
+  if (st != ZSAA_OK) return st;
+  // row offsets per layer boundary, the longest sequence, and the row counts
+  std::vector<int> rows(n1), nmax(n1, 0);
+  if (m->vl_cu == nullptr) {
+    ZCK(cudaMalloc(reinterpret_cast<void**>(&m->vl_cu), sizeof(int32_t) * n1 * (m->max_B + 1)));
+    ZCK(cudaMallocHost(reinterpret_cast<void**>(&m->vl_cu_host), sizeof(int32_t) * n1 * (m->max_B + 1)));
+    ZCK(cudaEventCreateWithFlags(&m->vl_done, cudaEventDisableTiming));
+  } else {
+    ZCK(cudaEventSynchronize(m->vl_done));  // the previous call's upload has read the host copy
+  }
+  for (int l = 0; l < n1; ++l) {
+    int32_t* cu = m->vl_cu_host + static_cast<size_t>(l) * (B + 1);
+    cu[0] = 0;
+    for (int b = 0; b < B; ++b) {
+      const int nb = sched[static_cast<size_t>(b) * n1 + l];
+      cu[b + 1] = cu[b] + nb;
+      nmax[l] = nb > nmax[l] ? nb : nmax[l];
+    }
+    rows[l] = cu[B];
+  }
+  ZCK(cudaMemcpyAsync(m->vl_cu, m->vl_cu_host, sizeof(int32_t) * n1 * (B + 1), cudaMemcpyHostToDevice, s));
+  ZCK(cudaEventRecord(m->vl_done, s));
+  auto cu_dev = [&](int l) { return m->vl_cu + static_cast<size_t>(l) * (B + 1); };
+
+  const int dt = c.dtype;
+  const int causal = c.bidirectional ? 0 : 1;
+  const double es = static_cast<double>(m->esz);
+  int cur = 0;
+#define TRACE(name, fl, by) TraceScope trace_scope_(m, name, fl, by, s)
+  {
+    TRACE("embed_norm", 0.0, static_cast<double>(T0) * (3.0 * d * es + 8.0));
+    ZCK(launch_rows_norm(m->embed, tok, c.vocab, 1, nullptr, 0, 0, nullptr, rows[0], d,
+                         LW(m, 0, kAttnNorm), c.rms_eps, m->h[cur], m->x, m->pos[cur], m->status,
+                         s, nullptr, cu_dev(0), B));
+  }
+  bool x_ready = true;
+  size_t off_forced = 0, off_scores = 0, off_idx = 0;
+  for (int l = 1; l <= n; ++l) {
+    const int li = l - 1;
+    const int M = rows[li], Nm = nmax[li];
+    const double Md = static_cast<double>(M);
+    void* h = m->h[cur];
+    if (!x_ready) {
+      TRACE("rmsnorm", 0.0, 2.0 * Md * d * es);
+      ZCK(launch_rmsnorm(dt, h, LW(m, li, kAttnNorm), M, d, c.rms_eps, m->x, s));
+    }
+    {
+      GemmParams p{};
+      p.M = M;
+      p.N = m->ld_qkv;
+      p.K = d;
+      p.out = m->qkv;
+      p.ldo = m->ld_qkv;
+      p.pos = m->pos[cur];
+      p.cos_t = m->rope_cos;
+      p.sin_t = m->rope_sin;
+      p.rope_cols = m->dq + m->dkv;
+      p.hd = hd;
+      p.vnorm_out = m->vnorm;
+      TcWeights W{LW(m, li, kWq), LW(m, li, kWk), LW(m, li, kWv), m->dq, m->dq + m->dkv};
+      TRACE("gemm_qkv_rope", 2.0 * Md * m->ld_qkv * d, (Md * d + static_cast<double>(m->ld_qkv) * d + Md * m->ld_qkv) * es);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->x, d, W, kEpiRope, p, s, &trace_scope_.kernels);
+      if (st != ZSAA_OK) return st;
+    }
+    {
+      double pairs = 0.0;
+      for (int b = 0; b < B; ++b) {
+        const double nb = sched[static_cast<size_t>(b) * n1 + li];
+        pairs += causal ? nb * (nb + 1) / 2.0 : nb * nb;
+      }
+      TRACE("attention", 4.0 * pairs * Hq * hd, Md * (m->ld_qkv + m->dq) * es + static_cast<double>(B) * Hq * Nm * 4.0);
+      ZCK(launch_attention(dt, m->qkv, B, Nm, Hq, Hkv, hd, m->attn, m->lse, causal, s, cu_dev(li)));
+    }
+    {
+      GemmParams q{};
+      q.M = M;
+      q.N = d;
+      q.K = m->dq;
+      q.out = h;
+      q.ldo = d;
+      q.resid = h;
+      TcWeights W{LW(m, li, kWo), nullptr, nullptr, d, d};
+      TRACE("gemm_o_resid", 2.0 * Md * d * m->dq, (Md * m->dq + static_cast<double>(d) * m->dq + 2.0 * Md * d) * es);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->attn, m->dq, W, kEpiResid, q, s, &trace_scope_.kernels);
+      if (st != ZSAA_OK) return st;
+    }
+    // elimination between attention and MLP (see run_forward), per sequence
+    bool mlp_x_ready = false;
+    if (prunes(c, l)) {
+      const bool want_scores = opts && opts->scores_out;
+      const bool forced = opts && opts->forced_idx;
+      const bool want_idx = opts && opts->idx_out;
+      const bool shrinks = rows[l] < M;
+      if (shrinks || want_scores || want_idx) {
+        if (Nm > kSelectPartsMaxN)
+          return fail(ZSAA_ERR_UNSUPPORTED, "variable-length selection needs lengths <= %d", kSelectPartsMaxN);
+        int n_qc = 1;
+        {
+          TRACE("colmass", 2.0 * Md * Nm * Hq * hd, Md * (m->dq + 2 * m->dkv) * es);
+          ZCK(launch_position_parts(dt, m->qkv, m->lse, m->vnorm, B, Nm, Hq, Hkv, hd, c.score_mode,
+                                    m->colmass, &n_qc, m->status, causal, s, cu_dev(li), M));
+        }
+        {
+          TRACE("select", 0.0, static_cast<double>(n_qc) * B * Hkv * Nm * 4.0 + rows[l] * 4.0);
+          ZCK(launch_select_parts(m->colmass, n_qc, B, Hkv, Nm, 0, c.force_keep_last, m->idx,
+                                  want_scores ? opts->scores_out + off_scores : nullptr, s, cu_dev(li),
+                                  cu_dev(l)));
+        }
+        const int32_t* idx = forced ? opts->forced_idx + off_forced : m->idx;
+        if (want_idx)
+          ZCK(cudaMemcpyAsync(opts->idx_out + off_idx, idx, sizeof(int32_t) * rows[l],
+                              cudaMemcpyDeviceToDevice, s));
+        if (shrinks) {
+          TRACE("gather_norm", 0.0, static_cast<double>(rows[l]) * (3.0 * d * es + 12.0));
+          ZCK(launch_rows_norm(h, nullptr, 0, 0, idx, Nm, 0, m->pos[cur], rows[l], d,
+                               LW(m, li, kMlpNorm), c.rms_eps, m->h[cur ^ 1], m->x, m->pos[cur ^ 1],
+                               m->status, s, cu_dev(li), cu_dev(l), B));
+          mlp_x_ready = true;
+          cur ^= 1;
+        }
+      }
+      off_forced += rows[l];
+      off_idx += rows[l];
+      off_scores += M;
+    }
+    const int Mm = rows[l];
+    const double Mmd = static_cast<double>(Mm);
+    void* hm = m->h[cur];
+    if (!mlp_x_ready) {
+      TRACE("rmsnorm", 0.0, 2.0 * Mmd * d * es);
+      ZCK(launch_rmsnorm(dt, hm, LW(m, li, kMlpNorm), Mm, d, c.rms_eps, m->x, s));
+    }
+    const double F = c.ffn_dim;
+    {
+      GemmParams q{};
+      q.M = Mm;
+      q.N = c.ffn_dim;
+      q.K = d;
+      q.out = m->act;
+      q.ldo = c.ffn_dim;
+      TcWeights W{LW(m, li, kWg), LW(m, li, kWu), nullptr, c.ffn_dim, c.ffn_dim};
+      TRACE("gemm_gate_up_swiglu", 4.0 * Mmd * F * d, (Mmd * d + 2.0 * F * d + Mmd * F) * es);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->x, d, W, kEpiSwiGLU, q, s, &trace_scope_.kernels);
+      if (st != ZSAA_OK) return st;
+    }
+    {
+      GemmParams q{};
+      q.M = Mm;
+      q.N = d;
+      q.K = c.ffn_dim;
+      q.out = hm;
+      q.ldo = d;
+      q.resid = hm;
+      TcWeights W{LW(m, li, kWd), nullptr, nullptr, d, d};
+      TRACE("gemm_down_resid", 2.0 * Mmd * d * F, (Mmd * F + F * d + 2.0 * Mmd * d) * es);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->act, c.ffn_dim, W, kEpiResid, q, s, &trace_scope_.kernels);
+      if (st != ZSAA_OK) return st;
+    }
+    x_ready = false;
+  }
+  const int Mf = rows[n];
+  if (c.n_classes > 0) {
+    TRACE("cls_head", 2.0 * B * d * c.n_classes, (static_cast<double>(B) * d + static_cast<double>(c.n_classes) * d) * es);
+    ZCK(launch_cls_head(dt, m->h[cur], B, 0, d, m->final_norm, c.rms_eps, m->head, c.n_classes,
+                        logits, s, cu_dev(n)));
+  } else {
+    {
+      TRACE("rmsnorm", 0.0, 2.0 * static_cast<double>(Mf) * d * es);
+      ZCK(launch_rmsnorm(dt, m->h[cur], m->final_norm, Mf, d, c.rms_eps, m->x, s));
+    }
+    GemmParams q{};
+    q.M = Mf;
+    q.N = c.vocab;
+    q.K = d;
+    q.out = logits;
+    q.ldo = c.vocab;
+    TcWeights W{m->head, nullptr, nullptr, c.vocab, c.vocab};
+    const double V = c.vocab, Mh = Mf;
+    TRACE("gemm_lm_head", 2.0 * Mh * V * d, (Mh * d + V * d) * es + Mh * V * 4.0);
+    trace_scope_.kernels = 0;
+    st = linear(m, m->x, d, W, kEpiStoreF32, q, s, &trace_scope_.kernels);
+    if (st != ZSAA_OK) return st;
+  }
+  if (kept_pos)
+    ZCK(cudaMemcpyAsync(kept_pos, m->pos[cur], sizeof(int32_t) * Mf, cudaMemcpyDeviceToDevice, s));
 #undef TRACE
   return ZSAA_OK;
 }
@@ -1314,6 +1583,28 @@ zsaa_status zsaa_trace_end(zsaa_model* m, zsaa_trace_row* rows, int max_rows, in
   m->trace.clear();
   m->ev_used = 0;
   return ZSAA_OK;
+}
+
+zsaa_status zsaa_plan_varlen_config(const zsaa_config* cfg, const int32_t* lengths, int B,
+                                    double accel, int* sched_out, double* alpha_out) {
+  if (cfg == nullptr || sched_out == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null config or output");
+  zsaa_status st = validate_config(*cfg);
+  if (st != ZSAA_OK) return st;
+  return plan_varlen_impl(*cfg, lengths, B, accel, sched_out, alpha_out);
+}
+
+zsaa_status zsaa_plan_varlen(const zsaa_model* m, const int32_t* lengths, int B, double accel,
+                             int* sched_out, double* alpha_out) {
+  if (m == nullptr || sched_out == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null model or output");
+  return plan_varlen_impl(m->cfg, lengths, B, accel, sched_out, alpha_out);
+}
+
+zsaa_status zsaa_forward_varlen(zsaa_model* m, const int32_t* token_ids, const int32_t* lengths,
+                                int B, double accel, float* logits_out, int32_t* kept_pos_out,
+                                const zsaa_forward_opts* opts, zsaa_stream stream) {
+  if (m == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null model");
+  return run_forward_varlen(m, token_ids, lengths, B, accel, logits_out, kept_pos_out, opts,
+                            reinterpret_cast<cudaStream_t>(stream));
 }
 
 zsaa_status zsaa_cache_create(zsaa_model* m, int B, int L, double accel, int max_new,

@@ -29,7 +29,8 @@ EXPORTED = [
     "zsaa_last_error", "zsaa_version", "zsaa_trace_begin", "zsaa_trace_end",
     "zsaa_score_select_noalloc", "zsaa_model_set_graphs", "zsaa_cache_create", "zsaa_cache_destroy",
     "zsaa_prefill", "zsaa_decode_step", "zsaa_cache_layer", "zsaa_cache_bytes",
-    "zsaa_op_attention_ex", "zsaa_op_colmass_ex",
+    "zsaa_op_attention_ex", "zsaa_op_colmass_ex", "zsaa_plan_varlen_config", "zsaa_plan_varlen",
+    "zsaa_forward_varlen",
 ]
 
 
@@ -95,6 +96,9 @@ def lib():
             "zsaa_op_attention": ([_P, _I, _I, _I, _I, _I, _I, _P, _P, _P], _I),
             "zsaa_op_colmass": ([_P, _P, _I, _I, _I, _I, _I, _I, _P, _P], _I),
             "zsaa_op_attention_ex": ([_P, _I, _I, _I, _I, _I, _I, _I, _P, _P, _P], _I),
+            "zsaa_plan_varlen_config": ([C.POINTER(zsaa_config), _P, _I, _D, C.POINTER(_I), C.POINTER(_D)], _I),
+            "zsaa_plan_varlen": ([_P, _P, _I, _D, C.POINTER(_I), C.POINTER(_D)], _I),
+            "zsaa_forward_varlen": ([_P, _P, _P, _I, _D, _P, _P, C.POINTER(zsaa_forward_opts), _P], _I),
             "zsaa_op_colmass_ex": ([_P, _P, _I, _I, _I, _I, _I, _I, _I, _P, _P], _I),
             "zsaa_sync": ([_P, _P], _I),
             "zsaa_device_status": ([], _I),
@@ -247,6 +251,44 @@ def zsaa_forward_ex(model: Model, token_ids, B: int, L: int, accel: float, logit
     _check(lib().zsaa_forward_ex(model.handle, _ptr(token_ids), B, L, float(accel),
                                  _ptr(logits_out), _ptr(kept_pos_out), C.byref(opts),
                                  _stream(stream)))
+
+
+def _lengths(lengths):
+    arr = (C.c_int32 * len(lengths))(*[int(x) for x in lengths])
+    return arr, len(lengths)
+
+
+def zsaa_plan_varlen_config(cfg: zsaa_config, lengths, accel: float) -> Tuple[List[List[int]], float]:
+    arr, B = _lengths(lengths)
+    n1 = cfg.n_layers + 1
+    sched = (C.c_int * (B * n1))()
+    alpha = C.c_double()
+    _check(lib().zsaa_plan_varlen_config(C.byref(cfg), C.cast(arr, C.c_void_p), B, float(accel), sched,
+                                         C.byref(alpha)))
+    return [list(sched[b * n1:(b + 1) * n1]) for b in range(B)], alpha.value
+
+
+def zsaa_plan_varlen(model: Model, lengths, accel: float) -> Tuple[List[List[int]], float]:
+    arr, B = _lengths(lengths)
+    n1 = model.cfg.n_layers + 1
+    sched = (C.c_int * (B * n1))()
+    alpha = C.c_double()
+    _check(lib().zsaa_plan_varlen(model.handle, C.cast(arr, C.c_void_p), B, float(accel), sched,
+                                  C.byref(alpha)))
+    return [list(sched[b * n1:(b + 1) * n1]) for b in range(B)], alpha.value
+
+
+def zsaa_forward_varlen(model: Model, token_ids, lengths, accel: float, logits_out, kept_pos_out=None,
+                        forced_idx=None, scores_out=None, idx_out=None, stream=None):
+    """token_ids: device int32 [sum(lengths)] packed; lengths: host sequence of ints."""
+    arr, B = _lengths(lengths)
+    opts = None
+    if forced_idx is not None or scores_out is not None or idx_out is not None:
+        opts = C.byref(zsaa_forward_opts(_ptr(forced_idx), _ptr(scores_out), _ptr(idx_out), None,
+                                         0, None, None, 0, 0))
+    _check(lib().zsaa_forward_varlen(model.handle, _ptr(token_ids), C.cast(arr, C.c_void_p), B,
+                                     float(accel), _ptr(logits_out), _ptr(kept_pos_out), opts,
+                                     _stream(stream)))
 
 
 def zsaa_forward_host(model: Model, token_ids, B: int, L: int, accel: float, logits_out,

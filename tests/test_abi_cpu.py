@@ -118,3 +118,21 @@ def test_generation_entry_points_reject_null_handles(zlib):
     assert L.zsaa_cache_layer(None, 1, None, None, None, None, None, None) == zlib.ZSAA_ERR_INVALID_ARG
     assert L.zsaa_cache_bytes(None, None, None) == zlib.ZSAA_ERR_INVALID_ARG
     L.zsaa_cache_destroy(None)  # no-op
+
+
+def test_varlen_planner_matches_oracle_exactly(zlib):
+    rng = np.random.default_rng(3)
+    for name in ("1b", "1b_cls", "8b", "tiny"):
+        shape = I.WORKLOADS[name]["shape"]
+        cfg = zlib.config_from_shape(shape)
+        ocfg = _oracle_cfg(shape)
+        for _ in range(6):
+            B = int(rng.integers(1, 9))
+            lengths = [int(x) for x in rng.integers(1, 2049, B)]
+            for accel in (1.0, 1.7, 4.0, 11.0):
+                sched, alpha = zlib.zsaa_plan_varlen_config(cfg, lengths, accel)
+                oalpha, osched = O.plan_varlen(ocfg, lengths, accel)
+                assert alpha == oalpha and sched == osched, (name, lengths, accel)
+    with pytest.raises(zlib.ZsaaError) as e:
+        zlib.zsaa_plan_varlen_config(zlib.config_from_shape(I.LLAMA_1B), [5, 0], 2.0)
+    assert e.value.status == zlib.ZSAA_ERR_INVALID_ARG
