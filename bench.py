@@ -511,6 +511,32 @@ def main():
                        "note": "zsaa_forward_host: pinned host tokens in, host float32 logits out; "
                                "the 256 MiB L2 flush runs inside this span"}
 
+        # ---- Appendix B's masked mode on the same batch: nothing removed, so the
+        # cost of the unpruned forward (the speedup comes from compaction)
+        if shape.dtype == "bf16":
+            n_fin = sched[-1]
+            lg_m = torch.empty(max_out, device=dev, dtype=torch.float32)
+
+            def run_masked():
+                zsaa.zsaa_forward_masked(model, tok_dev, B, L, args.accel, lg_m, None, stream=stream)
+            for _ in range(3):
+                run_masked()
+            torch.cuda.synchronize()
+            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                   for _ in range(args.steps)]
+            for e0, e1 in evs:
+                flush.zero_()
+                e0.record(stream)
+                run_masked()
+                e1.record(stream)
+            torch.cuda.synchronize()
+            zsaa.zsaa_sync(model)
+            ms_m = max_over_ranks(sum(a.elapsed_time(b) for a, b in evs) / args.steps)
+            line["masked_mode"] = {"accel": args.accel, "ms_per_step": ms_m,
+                                   "tokens_per_s": world * B * L / (ms_m / 1e3),
+                                   "vs_compacted": ms_m / ms_head, "final_rows": n_fin,
+                                   "note": "zsaa_forward_masked, eager launches"}
+
         # ---- variable-length batch: the same 4096 tokens as B x L, in mixed lengths
         if shape.n_classes == 0 and B * L == 4096:
             line["varlen"] = varlen_leg(zsaa, weights, cfg, shape, args.accel, flush, stream,

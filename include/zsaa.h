@@ -182,6 +182,22 @@ zsaa_status zsaa_forward_host(zsaa_model* m, const int32_t* token_ids, int B, in
                               double accel, float* logits_out, int32_t* kept_pos_out,
                               zsaa_stream stream);
 
+/* zsaa_forward_masked: Appendix B's "marked, not removed" formulation as an
+ * inference mode.  Every layer runs on all B*L rows; at a pruning layer the
+ * scores come from the unmarked queries and keys, the top N_l unmarked rows
+ * stay unmarked (Eq. 2 schedule, as zsaa_forward), and a marked row is hidden
+ * as a key from every later layer.  Outputs have the layout of zsaa_forward
+ * (logits of the final unmarked rows, their positions) and equal its values
+ * up to rounding; the cost is that of the unpruned forward (nothing is
+ * removed).  opts: NULL or the forced_idx / scores_out / idx_out hooks, with
+ * indices given as POSITIONS [B, N_l] per pruning layer and scores [B, L] per
+ * pruning layer (entries of marked rows unspecified); other fields zero.
+ * bf16 models, d_model <= 4096, L <= 12288.  Row flags are owned by the
+ * model (allocated on the first call). */
+zsaa_status zsaa_forward_masked(zsaa_model* m, const int32_t* token_ids, int B, int L, double accel,
+                                float* logits_out, int32_t* kept_pos_out,
+                                const zsaa_forward_opts* opts, zsaa_stream stream);
+
 /* ---- Variable-length batches.
  *
  * Sec. 3.4 picks the preservation rate per inference call.  For one call over

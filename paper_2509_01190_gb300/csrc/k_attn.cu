@@ -50,7 +50,8 @@ template <int HD>
 __global__ void __launch_bounds__(128)
     attn_fwd_bf16_kernel(const bf16* __restrict__ qkv, int Ns, int Hq, int Hkv,
                          bf16* __restrict__ out, float* __restrict__ lse2, float scale_log2,
-                         int causal, const int* __restrict__ cu) {
+                         int causal, const int* __restrict__ cu,
+                         const uint8_t* __restrict__ key_alive) {
   pdl_trigger();
   pdl_wait();
   constexpr int ROWB = HD * 2;
@@ -65,6 +66,8 @@ __global__ void __launch_bounds__(128)
   const size_t row0 = cu ? static_cast<size_t>(cu[b]) : static_cast<size_t>(b) * Ns;
   const int N = cu ? cu[b + 1] - cu[b] : Ns;
   if (qb * 64 >= N) return;
+  // masked mode (Appendix B): keys whose flag is 0 are hidden from every query
+  const uint8_t* ka = key_alive ? key_alive + static_cast<size_t>(b) * Ns : nullptr;
   const int g = h / (Hq / Hkv);
   const size_t ld = static_cast<size_t>(Hq + 2 * Hkv) * HD;
   const bf16* base = qkv + row0 * ld;
@@ -132,8 +135,9 @@ __global__ void __launch_bounds__(128)
       for (int e = 0; e < 2; ++e) {
         const int j = k0 + nt * 8 + 2 * tig + e;
         float a = s[nt][e] * scale_log2, c = s[nt][2 + e] * scale_log2;
-        if ((causal && j > i_lo) || j >= N) a = -INFINITY;
-        if ((causal && j > i_hi) || j >= N) c = -INFINITY;
+        const bool dead = j >= N || (ka != nullptr && ka[j] == 0);
+        if ((causal && j > i_lo) || dead) a = -INFINITY;
+        if ((causal && j > i_hi) || dead) c = -INFINITY;
         s[nt][e] = a;
         s[nt][2 + e] = c;
         mx_lo = fmaxf(mx_lo, a);
@@ -476,8 +480,9 @@ cudaError_t set_smem(Kern k, int bytes) {
 }  // namespace
 
 cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, int Hkv, int hd,
-                             void* out, float* lse, int causal, cudaStream_t s, const int* cu) {
-  if (cu != nullptr && dtype != ZSAA_BF16) return cudaErrorInvalidValue;
+                             void* out, float* lse, int causal, cudaStream_t s, const int* cu,
+                             const uint8_t* key_alive) {
+  if ((cu != nullptr || key_alive != nullptr) && dtype != ZSAA_BF16) return cudaErrorInvalidValue;
   const float scale_log2 = kLog2e / sqrtf(static_cast<float>(hd));
   if (dtype == ZSAA_F32) {
     dim3 grid((N + 3) / 4, Hq, B);
@@ -491,13 +496,13 @@ cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, i
     static cudaError_t e = set_smem(attn_fwd_bf16_kernel<64>, smem);
     if (e != cudaSuccess) return e;
     ZSAA_LAUNCH(attn_fwd_bf16_kernel<64>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), N, Hq, Hkv,
-                                                      static_cast<bf16*>(out), lse, scale_log2, causal, cu);
+                                                      static_cast<bf16*>(out), lse, scale_log2, causal, cu, key_alive);
   } else if (hd == 128) {
     const int smem = 5 * 64 * 256;
     static cudaError_t e = set_smem(attn_fwd_bf16_kernel<128>, smem);
     if (e != cudaSuccess) return e;
     ZSAA_LAUNCH(attn_fwd_bf16_kernel<128>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), N, Hq, Hkv,
-                                                       static_cast<bf16*>(out), lse, scale_log2, causal, cu);
+                                                       static_cast<bf16*>(out), lse, scale_log2, causal, cu, key_alive);
   } else {
     return cudaErrorInvalidValue;
   }
@@ -519,12 +524,12 @@ namespace {
 cudaError_t colmass_parts(int dtype, const void* qkv, const float* lse, const float* vnorm, int B,
                           int N, int Hq, int Hkv, int hd, int weight_vnorm, float* parts, int* n_qc,
                           int* status, int causal, cudaStream_t s, const int* cu = nullptr,
-                          int rows = 0) {
+                          int rows = 0, const uint8_t* q_alive = nullptr) {
   // tensor-core path (with precomputed norms when they are needed)
   if (dtype == ZSAA_BF16 && status != nullptr && (!weight_vnorm || vnorm != nullptr))
     return launch_colmass_tc(qkv, lse, weight_vnorm ? vnorm : nullptr, B, N, Hq, Hkv, hd, parts,
-                             status, n_qc, causal, s, cu, rows);
-  if (cu != nullptr) return cudaErrorInvalidValue;  // packed sequences: tensor-core path only
+                             status, n_qc, causal, s, cu, rows, q_alive);
+  if (cu != nullptr || q_alive != nullptr) return cudaErrorInvalidValue;  // tensor-core path only
   const float scale_log2 = kLog2e / sqrtf(static_cast<float>(hd));
   if (dtype == ZSAA_F32) {
     *n_qc = 1;
@@ -571,10 +576,10 @@ cudaError_t launch_colmass(int dtype, const void* qkv, const float* lse, int B, 
 cudaError_t launch_position_parts(int dtype, const void* qkv, const float* lse, const float* vnorm,
                                   int B, int N, int Hq, int Hkv, int hd, int mode, float* parts,
                                   int* n_qc, int* status, int causal, cudaStream_t s, const int* cu,
-                                  int rows) {
+                                  int rows, const uint8_t* q_alive) {
   return colmass_parts(dtype, qkv, lse, vnorm, B, N, Hq, Hkv, hd,
                        mode == ZSAA_SCORE_SOFTSCORE_VNORM ? 1 : 0, parts, n_qc, status, causal, s,
-                       cu, rows);
+                       cu, rows, q_alive);
 }
 
 cudaError_t launch_position_scores(int dtype, const void* qkv, const float* lse, const float* vnorm,

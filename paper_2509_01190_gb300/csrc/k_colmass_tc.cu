@@ -52,6 +52,7 @@ struct CmArgs {
   int B, N, Hq, Hkv, ld, n_kb, total, weight_vnorm;
   int causal;  // 0: bidirectional (every query block, no causal mask)
   const int* cu;  // packed sequences of different lengths: rows [cu[b], cu[b+1]); N = the longest
+  const uint8_t* q_alive;  // masked mode: [B, N] flags, queries with 0 add nothing
   float scale_log2;
   int* status;
 };
@@ -244,7 +245,9 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
         const int h = g * (a.Hq / a.Hkv) + hh;
         const int q = qb * CM_BN + et;
         float* dst = s_lse + buf * CM_BN + et;
-        if (q < n_b) {
+        if (q < n_b && a.q_alive != nullptr && a.q_alive[static_cast<size_t>(b) * a.N + q] == 0) {
+          *dst = INFINITY;  // exp2(s * c - inf) = 0: a hidden query contributes nothing
+        } else if (q < n_b) {
           asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)),
                        "l"(a.lse2 + (static_cast<size_t>(b) * a.Hq + h) * a.N + q)
                        : "memory");
@@ -367,7 +370,8 @@ cudaError_t run_cm(const CUtensorMap& tm, const CmArgs& a, int sms, cudaStream_t
 
 cudaError_t launch_colmass_tc(const void* qkv, const float* lse, const float* vnorm, int B, int N,
                               int Hq, int Hkv, int hd, float* parts, int* status, int* n_chunks,
-                              int causal, cudaStream_t s, const int* cu, int rows) {
+                              int causal, cudaStream_t s, const int* cu, int rows,
+                              const uint8_t* q_alive) {
   if (hd != 64 && hd != 128) return cudaErrorInvalidValue;
   const int ld = (Hq + 2 * Hkv) * hd;
   EncodeTiledFn enc = get_encode_tiled();
@@ -396,6 +400,7 @@ cudaError_t launch_colmass_tc(const void* qkv, const float* lse, const float* vn
   a.weight_vnorm = vnorm != nullptr;
   a.causal = causal;
   a.cu = cu;
+  a.q_alive = q_alive;
   a.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(hd));
   a.status = status;
   *n_chunks = Hq / Hkv;

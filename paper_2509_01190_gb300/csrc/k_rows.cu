@@ -176,7 +176,7 @@ __global__ void __launch_bounds__(kSelThreads)
     select_topk_kernel(const float* __restrict__ scores, int Ns, int ks, int force_last,
                        int32_t* __restrict__ idx_out, const float* __restrict__ parts, int n_qc,
                        int B, int G, float* __restrict__ scores_out, const int* __restrict__ cu_in,
-                       const int* __restrict__ cu_out) {
+                       const int* __restrict__ cu_out, uint8_t* __restrict__ alive) {
   pdl_trigger();
   pdl_wait();
   const int b = blockIdx.x;
@@ -203,6 +203,9 @@ __global__ void __launch_bounds__(kSelThreads)
     s = sscore;
   }
   int32_t* out = idx_out + (cu_out ? static_cast<size_t>(cu_out[b]) : static_cast<size_t>(b) * k);
+  // masked mode (Appendix B, fixed length): rows are never removed; the
+  // candidates are the rows still unmarked, and the flags are updated here
+  uint8_t* al = alive ? alive + static_cast<size_t>(b) * Ns : nullptr;
   const int n_cand = force_last ? N - 1 : N;
   const int need = force_last ? k - 1 : k;
 
@@ -218,6 +221,7 @@ __global__ void __launch_bounds__(kSelThreads)
       for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0;
       __syncthreads();
       for (int j = tid; j < n_cand; j += kSelThreads) {
+        if (al != nullptr && al[j] == 0) continue;  // masked mode: only unmarked rows compete
         const uint32_t key = order_key(s[j]);
         if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
       }
@@ -257,7 +261,7 @@ __global__ void __launch_bounds__(kSelThreads)
   int base_gt = 0, base_eq = 0;
   for (int j0 = 0; j0 < n_cand && need > 0; j0 += kSelThreads) {
     const int j = j0 + tid;
-    const bool in = j < n_cand;
+    const bool in = j < n_cand && (al == nullptr || al[j] != 0);
     const uint32_t key = in ? order_key(s[j]) : 0u;
     const bool gt = in && key > T;
     const bool eq = in && key == T;
@@ -295,6 +299,29 @@ __global__ void __launch_bounds__(kSelThreads)
     __syncthreads();
   }
   if (force_last && tid == 0) out[k - 1] = N - 1;
+  if (al != nullptr) {  // the kept rows stay unmarked, every other row is marked
+    __syncthreads();
+    for (int j = tid; j < N; j += kSelThreads) al[j] = 0;
+    __syncthreads();
+    for (int r = tid; r < k; r += kSelThreads) al[out[r]] = 1;
+  }
+}
+
+// Masked mode with given kept positions: flags[b, :] = 0, then 1 at idx[b, :k].
+__global__ void flags_from_idx_kernel(const int32_t* __restrict__ idx, int N, int k,
+                                      uint8_t* __restrict__ flags, int* status) {
+  pdl_trigger();
+  pdl_wait();
+  uint8_t* f = flags + static_cast<size_t>(blockIdx.x) * N;
+  for (int j = threadIdx.x; j < N; j += blockDim.x) f[j] = 0;
+  __syncthreads();
+  for (int r = threadIdx.x; r < k; r += blockDim.x) {
+    const int j = idx[static_cast<size_t>(blockIdx.x) * k + r];
+    if (j >= 0 && j < N)
+      f[j] = 1;
+    else if (status != nullptr)
+      atomicOr(status, kStatusBadIndex);
+  }
 }
 
 // ---------------------------------------------------------------- gather
@@ -534,13 +561,14 @@ cudaError_t launch_select(const float* scores, int B, int N, int k, int force_la
                           cudaStream_t s) {
   ZSAA_LAUNCH(select_topk_kernel<false>, dim3(B), dim3(kSelThreads), 0, s, scores, N, k, force_last,
               idx, static_cast<const float*>(nullptr), 0, B, 0, static_cast<float*>(nullptr),
-              static_cast<const int*>(nullptr), static_cast<const int*>(nullptr));
+              static_cast<const int*>(nullptr), static_cast<const int*>(nullptr),
+              static_cast<uint8_t*>(nullptr));
   return cudaGetLastError();
 }
 
 cudaError_t launch_select_parts(const float* parts, int n_qc, int B, int G, int N, int k,
                                 int force_last, int32_t* idx, float* scores_out, cudaStream_t s,
-                                const int* cu_in, const int* cu_out) {
+                                const int* cu_in, const int* cu_out, uint8_t* alive) {
   const size_t smem = static_cast<size_t>(N) * sizeof(float);
   static cudaError_t attr = cudaFuncSetAttribute(select_topk_kernel<true>,
                                                  cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -548,7 +576,13 @@ cudaError_t launch_select_parts(const float* parts, int n_qc, int B, int G, int 
   if (attr != cudaSuccess) return attr;
   ZSAA_LAUNCH(select_topk_kernel<true>, dim3(B), dim3(kSelThreads), smem, s,
               static_cast<const float*>(nullptr), N, k, force_last, idx, parts, n_qc, B, G, scores_out,
-              cu_in, cu_out);
+              cu_in, cu_out, alive);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_flags_from_idx(const int32_t* idx, int B, int N, int k, uint8_t* flags,
+                                  int* status, cudaStream_t s) {
+  ZSAA_LAUNCH(flags_from_idx_kernel, dim3(B), dim3(256), 0, s, idx, N, k, flags, status);
   return cudaGetLastError();
 }
 

@@ -25,7 +25,11 @@ constexpr int kSelectPartsMaxN = 12288;
 // written packed at cu_out[b] / cu_in[b].
 cudaError_t launch_select_parts(const float* parts, int n_qc, int B, int G, int N, int k,
                                 int force_last, int32_t* idx, float* scores_out, cudaStream_t s,
-                                const int* cu_in = nullptr, const int* cu_out = nullptr);
+                                const int* cu_in = nullptr, const int* cu_out = nullptr,
+                                uint8_t* alive = nullptr);
+// alive (masked mode, fixed length): [B, N] flags; only flagged rows compete
+// (k includes the forced last row), and afterwards exactly the kept rows are
+// flagged.  idx then holds positions 0..N-1.
 // bf16 rows: h_out[r] = source row, x_out[r] = RMSNorm(h_out[r]) * w, pos_out[r].
 // Embedding when idx == nullptr (rows = B*L, source row tok[r] of E);
 // otherwise compaction (rows = B*k, source row b*N + idx[r] of h).
@@ -40,6 +44,9 @@ cudaError_t launch_rows_norm(const void* src, const int32_t* tok, int vocab, int
                              int32_t* pos_out, int* status, cudaStream_t s,
                              const int* cu_src = nullptr, const int* cu_dst = nullptr,
                              int nseq = 0);
+// flags[b, :N] = 0 except 1 at positions idx[b, :k] (masked mode, forced choice).
+cudaError_t launch_flags_from_idx(const int32_t* idx, int B, int N, int k, uint8_t* flags,
+                                  int* status, cudaStream_t s);
 cudaError_t launch_gather(const void* src, int B, int N, int k, int row_bytes, const int32_t* idx,
                           void* dst, const int32_t* pos_in, int32_t* pos_out, int* status,
                           cudaStream_t s);
@@ -109,7 +116,9 @@ cudaError_t launch_gemm_f32(const float* A, int lda, const float* W, const float
 // N is then the longest length (grid size and the stride of lse).
 cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, int Hkv, int hd,
                              void* out, float* lse, int causal, cudaStream_t s,
-                             const int* cu = nullptr);
+                             const int* cu = nullptr, const uint8_t* key_alive = nullptr);
+// key_alive (bf16, fixed length): [B, N] flags of the masked mode; keys with 0
+// are hidden from every query.
 // Column mass C[B, Hkv, N] (via partial sums in `parts`, which must hold
 // colmass_parts_elems(B, N, Hq, Hkv) floats).  bf16 with a status word runs
 // the tensor-core kernel (k_colmass_tc.cu); otherwise the mma.sync / fp32 ones.
@@ -132,14 +141,16 @@ cudaError_t launch_position_scores(int dtype, const void* qkv, const float* lse,
 cudaError_t launch_position_parts(int dtype, const void* qkv, const float* lse, const float* vnorm,
                                   int B, int N, int Hq, int Hkv, int hd, int mode, float* parts,
                                   int* n_qc, int* status, int causal, cudaStream_t s,
-                                  const int* cu = nullptr, int rows = 0);
+                                  const int* cu = nullptr, int rows = 0,
+                                  const uint8_t* q_alive = nullptr);
 // Tensor-core column-mass partials: parts[Hq/Hkv][B][Hkv][N] (per head of the
 // group), times vnorm when it is not NULL; hd 64 or 128.  With cu: packed
 // sequences of different lengths (rows [cu[b], cu[b+1]), `rows` in all, N the
 // longest); vnorm is then per packed row.
 cudaError_t launch_colmass_tc(const void* qkv, const float* lse, const float* vnorm, int B, int N,
                               int Hq, int Hkv, int hd, float* parts, int* status, int* n_chunks,
-                              int causal, cudaStream_t s, const int* cu = nullptr, int rows = 0);
+                              int causal, cudaStream_t s, const int* cu = nullptr, int rows = 0,
+                              const uint8_t* q_alive = nullptr);
 
 // ---- generation over the pruned KV cache (k_decode.cu)
 // Cache of one layer: K and V bf16 [B, Hkv, cap, hd], positions int32 [B, cap].

@@ -319,6 +319,7 @@ struct zsaa_model {
   size_t stage_logits_cap = 0;
   // packed-sequence row offsets of zsaa_forward_varlen (device, and the pinned
   // host copy they are uploaded from; the event guards its reuse)
+  uint8_t* alive = nullptr;  // masked mode: [max_B, max_L] row flags (allocated on first use)
   int32_t* vl_cu = nullptr;
   int32_t* vl_cu_host = nullptr;
   cudaEvent_t vl_done = nullptr;
@@ -430,6 +431,7 @@ void free_model(zsaa_model* m) {
   for (void* p : ptrs)
     if (p) cudaFree(p);
   if (m->vl_cu) cudaFree(m->vl_cu);
+  if (m->alive) cudaFree(m->alive);
   if (m->vl_cu_host) cudaFreeHost(m->vl_cu_host);
   if (m->vl_done) cudaEventDestroy(m->vl_done);
   delete m;
@@ -755,6 +757,194 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
   }
   if (kept_pos)
     ZCK(cudaMemcpyAsync(kept_pos, m->pos[cur], sizeof(int32_t) * M, cudaMemcpyDeviceToDevice, s));
+#undef TRACE
+  return ZSAA_OK;
+}
+
+// Appendix B's formulation as an inference mode: rows are marked instead of
+// removed.  Every layer runs on all B*L rows; a marked row is hidden as a key
+// from the layer after its marking on, its query adds nothing to later column
+// masses, and only unmarked rows compete at a selection.  The kept rows'
+// outputs equal those of the compacted forward; the cost is that of accel 1.
+zsaa_status run_forward_masked(zsaa_model* m, const int32_t* tok, int B, int L, double accel,
+                               float* logits, int32_t* kept_pos, const zsaa_forward_opts* opts,
+                               cudaStream_t s) {
+  const zsaa_config& c = m->cfg;
+  const int d = c.d_model, hd = c.head_dim, Hq = c.n_heads, Hkv = c.n_kv_heads, n = c.n_layers;
+  if (c.dtype != ZSAA_BF16 || d % 8 != 0 || d > kRowsNormMaxD)
+    return fail(ZSAA_ERR_UNSUPPORTED, "the masked mode needs a bf16 model with d_model <= %d", kRowsNormMaxD);
+  if (tok == nullptr || logits == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null token or logits pointer");
+  if (B < 1 || B > m->max_B || L < 1 || L > m->max_L)
+    return fail(ZSAA_ERR_INVALID_ARG, "B=%d L=%d outside [1,%d] x [1,%d]", B, L, m->max_B, m->max_L);
+  if (L > kSelectPartsMaxN) return fail(ZSAA_ERR_UNSUPPORTED, "the masked mode needs L <= %d", kSelectPartsMaxN);
+  if (opts && (opts->hidden_out || opts->n_layers_run || opts->hidden_in || opts->pos_in ||
+               opts->first_layer || opts->plan_L))
+    return fail(ZSAA_ERR_INVALID_ARG, "the masked mode takes only the forced_idx/scores_out/idx_out hooks");
+  std::vector<int> sched(n + 1);
+  double alpha = 1.0;
+  zsaa_status st = plan_impl(c, L, accel, sched.data(), &alpha);
+  if (st != ZSAA_OK) return st;
+  if (m->alive == nullptr)
+    ZCK(cudaMalloc(reinterpret_cast<void**>(&m->alive), static_cast<size_t>(m->max_B) * m->max_L));
+  ZCK(cudaMemsetAsync(m->alive, 1, static_cast<size_t>(B) * L, s));
+  const int dt = c.dtype;
+  const int causal = c.bidirectional ? 0 : 1;
+  const double es = static_cast<double>(m->esz);
+  const int M = B * L;
+  const double Md = static_cast<double>(M);
+  void* h = m->h[0];
+#define TRACE(name, fl, by) TraceScope trace_scope_(m, name, fl, by, s)
+  {
+    TRACE("embed_norm", 0.0, Md * (3.0 * d * es + 8.0));
+    ZCK(launch_rows_norm(m->embed, tok, c.vocab, L, nullptr, 0, 0, nullptr, M, d,
+                         LW(m, 0, kAttnNorm), c.rms_eps, h, m->x, m->pos[0], m->status, s));
+  }
+  const int32_t* kept = nullptr;  // positions of the unmarked rows after the last selection
+  size_t off_forced = 0, off_scores = 0, off_idx = 0;
+  const double pairs = static_cast<double>(B) * Hq * (causal ? L * (L + 1.0) / 2.0 : 1.0 * L * L);
+  for (int l = 1; l <= n; ++l) {
+    const int li = l - 1;
+    if (l > 1) {
+      TRACE("rmsnorm", 0.0, 2.0 * Md * d * es);
+      ZCK(launch_rmsnorm(dt, h, LW(m, li, kAttnNorm), M, d, c.rms_eps, m->x, s));
+    }
+    {
+      GemmParams p{};
+      p.M = M;
+      p.N = m->ld_qkv;
+      p.K = d;
+      p.out = m->qkv;
+      p.ldo = m->ld_qkv;
+      p.pos = m->pos[0];
+      p.cos_t = m->rope_cos;
+      p.sin_t = m->rope_sin;
+      p.rope_cols = m->dq + m->dkv;
+      p.hd = hd;
+      p.vnorm_out = m->vnorm;
+      TcWeights W{LW(m, li, kWq), LW(m, li, kWk), LW(m, li, kWv), m->dq, m->dq + m->dkv};
+      TRACE("gemm_qkv_rope", 2.0 * Md * m->ld_qkv * d, (Md * d + static_cast<double>(m->ld_qkv) * d + Md * m->ld_qkv) * es);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->x, d, W, kEpiRope, p, s, &trace_scope_.kernels);
+      if (st != ZSAA_OK) return st;
+    }
+    {
+      TRACE("attention", 4.0 * pairs * hd, Md * (m->ld_qkv + m->dq) * es + static_cast<double>(B) * Hq * L * 4.0);
+      ZCK(launch_attention(dt, m->qkv, B, L, Hq, Hkv, hd, m->attn, m->lse, causal, s, nullptr,
+                           m->alive));
+    }
+    {
+      GemmParams q{};
+      q.M = M;
+      q.N = d;
+      q.K = m->dq;
+      q.out = h;
+      q.ldo = d;
+      q.resid = h;
+      TcWeights W{LW(m, li, kWo), nullptr, nullptr, d, d};
+      TRACE("gemm_o_resid", 2.0 * Md * d * m->dq, (Md * m->dq + static_cast<double>(d) * m->dq + 2.0 * Md * d) * es);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->attn, m->dq, W, kEpiResid, q, s, &trace_scope_.kernels);
+      if (st != ZSAA_OK) return st;
+    }
+    if (prunes(c, l)) {
+      const int k = sched[l];
+      const bool want_scores = opts && opts->scores_out;
+      const bool forced = opts && opts->forced_idx;
+      const bool want_idx = opts && opts->idx_out;
+      if (k < sched[l - 1] || want_scores || want_idx) {
+        int n_qc = 1;
+        {
+          TRACE("colmass", 2.0 * pairs * hd, Md * (m->dq + 2 * m->dkv) * es);
+          ZCK(launch_position_parts(dt, m->qkv, m->lse, m->vnorm, B, L, Hq, Hkv, hd, c.score_mode,
+                                    m->colmass, &n_qc, m->status, causal, s, nullptr, 0, m->alive));
+        }
+        {
+          TRACE("select", 0.0, static_cast<double>(n_qc) * B * Hkv * L * 4.0 + static_cast<double>(B) * k * 4.0);
+          ZCK(launch_select_parts(m->colmass, n_qc, B, Hkv, L, k, c.force_keep_last, m->idx,
+                                  want_scores ? opts->scores_out + off_scores : nullptr, s, nullptr,
+                                  nullptr, forced ? nullptr : m->alive));
+        }
+        kept = m->idx;
+        if (forced) {
+          kept = opts->forced_idx + off_forced;
+          TRACE("select", 0.0, static_cast<double>(B) * (L + 4.0 * k));
+          ZCK(launch_flags_from_idx(kept, B, L, k, m->alive, m->status, s));
+        }
+        if (want_idx)
+          ZCK(cudaMemcpyAsync(opts->idx_out + off_idx, kept, sizeof(int32_t) * B * k,
+                              cudaMemcpyDeviceToDevice, s));
+      }
+      off_forced += static_cast<size_t>(B) * k;
+      off_idx += static_cast<size_t>(B) * k;
+      off_scores += static_cast<size_t>(B) * L;
+    }
+    // the MLP of every row, marked or not (the formulation removes nothing)
+    {
+      TRACE("rmsnorm", 0.0, 2.0 * Md * d * es);
+      ZCK(launch_rmsnorm(dt, h, LW(m, li, kMlpNorm), M, d, c.rms_eps, m->x, s));
+    }
+    const double F = c.ffn_dim;
+    {
+      GemmParams q{};
+      q.M = M;
+      q.N = c.ffn_dim;
+      q.K = d;
+      q.out = m->act;
+      q.ldo = c.ffn_dim;
+      TcWeights W{LW(m, li, kWg), LW(m, li, kWu), nullptr, c.ffn_dim, c.ffn_dim};
+      TRACE("gemm_gate_up_swiglu", 4.0 * Md * F * d, (Md * d + 2.0 * F * d + Md * F) * es);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->x, d, W, kEpiSwiGLU, q, s, &trace_scope_.kernels);
+      if (st != ZSAA_OK) return st;
+    }
+    {
+      GemmParams q{};
+      q.M = M;
+      q.N = d;
+      q.K = c.ffn_dim;
+      q.out = h;
+      q.ldo = d;
+      q.resid = h;
+      TcWeights W{LW(m, li, kWd), nullptr, nullptr, d, d};
+      TRACE("gemm_down_resid", 2.0 * Md * d * F, (Md * F + F * d + 2.0 * Md * d) * es);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->act, c.ffn_dim, W, kEpiResid, q, s, &trace_scope_.kernels);
+      if (st != ZSAA_OK) return st;
+    }
+  }
+  // the unmarked rows, in order, through the head
+  const int nf = sched[n];
+  void* hf = h;
+  const int32_t* posf = m->pos[0];
+  if (kept != nullptr) {
+    TRACE("gather_norm", 0.0, static_cast<double>(B) * nf * (3.0 * d * es + 12.0));
+    ZCK(launch_rows_norm(h, nullptr, 0, 0, kept, L, nf, m->pos[0], B * nf, d, m->final_norm,
+                         c.rms_eps, m->h[1], m->x, m->pos[1], m->status, s));
+    hf = m->h[1];
+    posf = m->pos[1];
+  } else if (c.n_classes == 0) {
+    TRACE("rmsnorm", 0.0, 2.0 * static_cast<double>(B) * nf * d * es);
+    ZCK(launch_rmsnorm(dt, h, m->final_norm, B * nf, d, c.rms_eps, m->x, s));
+  }
+  if (c.n_classes > 0) {
+    TRACE("cls_head", 2.0 * B * d * c.n_classes, (static_cast<double>(B) * d + static_cast<double>(c.n_classes) * d) * es);
+    ZCK(launch_cls_head(dt, hf, B, nf, d, m->final_norm, c.rms_eps, m->head, c.n_classes, logits, s));
+  } else {
+    GemmParams q{};
+    q.M = B * nf;
+    q.N = c.vocab;
+    q.K = d;
+    q.out = logits;
+    q.ldo = c.vocab;
+    TcWeights W{m->head, nullptr, nullptr, c.vocab, c.vocab};
+    const double V = c.vocab, Mh = static_cast<double>(B) * nf;
+    TRACE("gemm_lm_head", 2.0 * Mh * V * d, (Mh * d + V * d) * es + Mh * V * 4.0);
+    trace_scope_.kernels = 0;
+    st = linear(m, m->x, d, W, kEpiStoreF32, q, s, &trace_scope_.kernels);
+    if (st != ZSAA_OK) return st;
+  }
+  if (kept_pos)
+    ZCK(cudaMemcpyAsync(kept_pos, posf, sizeof(int32_t) * B * nf, cudaMemcpyDeviceToDevice, s));
 #undef TRACE
   return ZSAA_OK;
 }
@@ -1583,6 +1773,14 @@ zsaa_status zsaa_trace_end(zsaa_model* m, zsaa_trace_row* rows, int max_rows, in
   m->trace.clear();
   m->ev_used = 0;
   return ZSAA_OK;
+}
+
+zsaa_status zsaa_forward_masked(zsaa_model* m, const int32_t* token_ids, int B, int L, double accel,
+                                float* logits_out, int32_t* kept_pos_out,
+                                const zsaa_forward_opts* opts, zsaa_stream stream) {
+  if (m == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null model");
+  return run_forward_masked(m, token_ids, B, L, accel, logits_out, kept_pos_out, opts,
+                            reinterpret_cast<cudaStream_t>(stream));
 }
 
 zsaa_status zsaa_plan_varlen_config(const zsaa_config* cfg, const int32_t* lengths, int B,

@@ -1,0 +1,104 @@
+"""The masked ("marked, not removed") mode of Appendix B on the GPU
+(zsaa_forward_masked) against the oracle's forward_masked, and against the
+library's compacted forward.
+
+Protocol: a natural run (the first pruning layer sees identical rows, so its
+scores and kept positions are compared with the oracle's as in the compacted
+tests), then a run with the oracle's kept positions forced, whose logits must
+meet the stated bf16 tolerance and whose kept positions must be exact; the
+compacted forward with the same choice must agree to the same tolerance.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import zsaa_oracle as O
+from paper_2509_01190_gb300 import inputs as I
+from tests.helpers import BF16_MAX_ABS, BF16_MEAN_ABS, logits_report, need_gpu, oracle_cfg
+from tests.test_gpu_forward import SMALL_BF16, SMALL_BF16_128, SMALL_CLS
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def z(zlib):
+    need_gpu()
+    return zlib
+
+
+def run_masked(z, shape, B, L, accel, seed=42):
+    weights = I.make_weights(shape, device="cuda")
+    tokens = I.make_tokens(B, L, shape.vocab, seed=seed)
+    tok = torch.from_numpy(tokens).cuda()
+    model = z.Model(z.config_from_shape(shape), weights, B, L)
+    sched, alpha = z.zsaa_plan(model, L, accel)
+    ocfg = oracle_cfg(shape)
+    wnp = I.weights_to_numpy(weights)
+    om = O.forward_masked(ocfg, wnp, tokens, sched)
+    oc = O.forward(ocfg, wnp, tokens, alpha=alpha)
+    prune = shape.prune_layers()
+    n_fin = sched[-1]
+    out_shape = (B, shape.n_classes) if shape.n_classes else (B, n_fin, shape.vocab)
+    # natural run with hooks
+    lg = torch.empty(out_shape, device="cuda", dtype=torch.float32)
+    kept = torch.empty(B, n_fin, device="cuda", dtype=torch.int32)
+    idx_tot = sum(B * sched[l] for l in prune)
+    idx_out = torch.full((max(idx_tot, 1),), -1, device="cuda", dtype=torch.int32)
+    sc_out = torch.zeros(max(len(prune) * B * L, 1), device="cuda", dtype=torch.float32)
+    z.zsaa_forward_masked(model, tok, B, L, accel, lg, kept, scores_out=sc_out, idx_out=idx_out)
+    z.zsaa_sync(model)
+    # forced run with the oracle's positions
+    forced = [om["kept_by_layer"][l].reshape(-1) for l in prune if l in om["kept_by_layer"]]
+    fdev = torch.from_numpy(np.concatenate(forced).astype(np.int32)).cuda() if forced else None
+    lg2 = torch.empty_like(lg)
+    kept2 = torch.empty_like(kept)
+    z.zsaa_forward_masked(model, tok, B, L, accel, lg2, kept2, forced_pos=fdev)
+    # the compacted forward with the same choice (indices into the current rows)
+    lg3 = torch.empty_like(lg)
+    fi = [oc["idx"][l].reshape(-1) for l in prune if l in oc["idx"]]
+    fidev = torch.from_numpy(np.concatenate(fi).astype(np.int32)).cuda() if fi else None
+    z.zsaa_forward_ex(model, tok, B, L, accel, lg3, None, forced_idx=fidev)
+    z.zsaa_sync(model)
+    return dict(sched=sched, om=om, oc=oc, prune=prune, idx_out=idx_out.cpu().numpy(),
+                sc_out=sc_out.cpu().numpy(), nat_kept=kept.cpu().numpy(), forced_logits=lg2.cpu().numpy(),
+                forced_kept=kept2.cpu().numpy(), compact_logits=lg3.cpu().numpy(), B=B, L=L)
+
+
+def check_masked(res):
+    om, oc, B, L = res["om"], res["oc"], res["B"], res["L"]
+    np.testing.assert_array_equal(res["forced_kept"], om["kept_pos"])
+    np.testing.assert_array_equal(om["kept_pos"], oc["kept_pos"])  # the oracle's two formulations
+    for got in (res["forced_logits"], res["compact_logits"]):
+        mx, mean = logits_report(got, om["logits"])
+        assert mx <= BF16_MAX_ABS and mean <= BF16_MEAN_ABS, (mx, mean)
+    if not res["prune"]:
+        return
+    # first pruning layer: every row is unmarked, so scores and choices are the compacted ones
+    l = res["prune"][0]
+    k = res["sched"][l]
+    sc = res["sc_out"][: B * L].reshape(B, L)
+    pos = res["idx_out"][: B * k].reshape(B, k)
+    for b in range(B):
+        s_ref = oc["scores"][l][b]
+        np.testing.assert_allclose(sc[b], s_ref, rtol=2e-2, atol=2e-2 * s_ref.max())
+        if k == L:
+            np.testing.assert_array_equal(pos[b], np.arange(L))
+            continue
+        order = np.sort(s_ref[:-1])[::-1]
+        thr = order[k - 2] if k >= 2 else np.inf
+        amb = set(np.nonzero(np.abs(s_ref - thr) <= 1e-2 * abs(thr))[0].tolist())
+        assert set(pos[b].tolist()) - amb == set(om["kept_by_layer"][l][b].tolist()) - amb
+        assert np.all(np.diff(pos[b]) > 0) and pos[b][-1] == L - 1
+
+
+@pytest.mark.parametrize("accel", [1.0, 2.0, 4.0])
+def test_masked_small_lm(z, accel):
+    check_masked(run_masked(z, SMALL_BF16, 3, 150, accel))
+
+
+def test_masked_small_hd128_and_classifier(z):
+    check_masked(run_masked(z, SMALL_BF16_128, 2, 333, 3.0))
+    res = run_masked(z, SMALL_CLS, 4, 120, 3.0)
+    check_masked(res)
+    assert res["forced_logits"].shape == (4, 4)
