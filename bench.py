@@ -42,6 +42,37 @@ if ROOT not in sys.path:
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
+# DRAM bytes per launch of the dominant kernel class (gate/up + SwiGLU GEMM) in
+# this forward, from one ncu capture (profiles/gemm_gate_up_swiglu_1b_traffic.md):
+# the mean of dram__bytes_read.sum + dram__bytes_write.sum over the 16 launches
+# of one forward.  Reported only while the sources it was measured on are
+# unchanged (sha256 below), else null.
+GATE_UP_TRAFFIC = {
+    "bytes_per_launch": 73546608.0,
+    "sources": {
+        "paper_2509_01190_gb300/csrc/k_gemm_tc.cu": "4368111cbae07a2681e323fed306aced39043baceb1473ab1fec0b06c7770513",
+        "paper_2509_01190_gb300/csrc/common.cuh": "f6813b6c6ecf5b5ff1008a2df997d16e1360d7b3fc8561dde7e27e0fc4b06f8b",
+        "paper_2509_01190_gb300/csrc/kernels.h": "188dbe67722fad80bb3d870535f0df1e11bbf742b281097180bbad52716e2ab2",
+    },
+}
+
+
+def measured_traffic(kernel_name):
+    """The ncu-measured DRAM bytes per launch of `kernel_name`, or None."""
+    import hashlib
+    if kernel_name != "gemm_gate_up_swiglu":
+        return None
+    root = os.path.dirname(os.path.abspath(__file__))
+    for rel, digest in GATE_UP_TRAFFIC["sources"].items():
+        try:
+            with open(os.path.join(root, rel), "rb") as f:
+                if hashlib.sha256(f.read()).hexdigest() != digest:
+                    return None
+        except OSError:
+            return None
+    return GATE_UP_TRAFFIC["bytes_per_launch"]
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -477,7 +508,8 @@ def main():
             ach = dom["flops"] / (dom["ms"] / 1e3) / 1e12
             peak = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
             line["roofline"] = {"bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
-                                "frac": ach / peak, "traffic": None, "kernel": dom["name"],
+                                "frac": ach / peak, "traffic": measured_traffic(dom["name"]),
+                                "kernel": dom["name"],
                                 "per_launch_ms": dom["ms"] / dom["launches"],
                                 "peak_source": f"{src} bf16_tflops_sustained (kernel inside a long step)"}
         else:
