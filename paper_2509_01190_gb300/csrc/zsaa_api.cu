@@ -302,6 +302,7 @@ struct zsaa_model {
   void* attn = nullptr;
   void* act = nullptr;
   float* lse = nullptr;
+  void* vt = nullptr;        // V^T of the current layer for the tcgen05 attention (bf16, hd 64)
   float* colmass = nullptr;  // query-chunk partials of the column mass / scores
   float* vnorm = nullptr;    // ||v|| per row and KV group, from the QKV epilogue (bf16)
   float* scores = nullptr;
@@ -424,7 +425,7 @@ void free_model(zsaa_model* m) {
   for (auto& g : m->graphs)
     if (g.exec) cudaGraphExecDestroy(g.exec);
   if (m->capture_stream) cudaStreamDestroy(m->capture_stream);
-  void* ptrs[] = {m->h[0], m->h[1], m->x, m->qkv, m->attn, m->act, m->lse, m->colmass, m->vnorm,
+  void* ptrs[] = {m->h[0], m->h[1], m->x, m->qkv, m->attn, m->act, m->lse, m->vt, m->colmass, m->vnorm,
                   m->scores, m->idx, m->pos[0], m->pos[1], m->rope_cos, m->rope_sin,
                   m->splitk_ws, m->splitk_flags, m->status, m->stage_tok, m->stage_logits,
                   m->stage_pos};
@@ -581,7 +582,12 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
     {
       const double pairs = static_cast<double>(B) * Hq * n_pairs(N);
       TRACE("attention", 4.0 * pairs * hd, Md * (m->ld_qkv + m->dq) * es + static_cast<double>(B) * Hq * N * 4.0);
-      ZCK(launch_attention(dt, m->qkv, B, N, Hq, Hkv, hd, m->attn, m->lse, causal, s));
+      if (attention_tc_supported(dt, hd, nullptr, nullptr, m->status, m->vt) && attention_tc_preferred(N)) {
+        trace_scope_.kernels = 2;  // V transpose + attention
+        ZCK(launch_attention_tc(m->qkv, m->vt, B, N, Hq, Hkv, m->attn, m->lse, causal, m->status, s));
+      } else {
+        ZCK(launch_attention(dt, m->qkv, B, N, Hq, Hkv, hd, m->attn, m->lse, causal, s));
+      }
     }
     {
       GemmParams q{};
@@ -1527,6 +1533,8 @@ zsaa_status zsaa_model_create(const zsaa_config* cfg, const zsaa_weights* w, int
   alloc(&m->attn, rows * m->dq * esz);
   alloc(&m->act, rows * F * esz);
   alloc(reinterpret_cast<void**>(&m->lse), rows * cfg->n_heads * sizeof(float));
+  if (cfg->dtype == ZSAA_BF16 && cfg->head_dim == 64)
+    alloc(&m->vt, attention_tc_vt_elems(max_B, max_L, cfg->n_kv_heads) * 2);
   alloc(reinterpret_cast<void**>(&m->colmass),
         colmass_parts_elems(max_B, max_L, cfg->n_heads, cfg->n_kv_heads) * sizeof(float));
   alloc(reinterpret_cast<void**>(&m->vnorm), rows * cfg->n_kv_heads * sizeof(float));
@@ -1711,8 +1719,18 @@ zsaa_status zsaa_op_attention_ex(const void* qkv, int B, int N, int Hq, int Hkv,
   if (B < 1 || N < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv) return fail(ZSAA_ERR_INVALID_ARG, "bad shape");
   if (dtype == ZSAA_BF16 && hd != 64 && hd != 128) return fail(ZSAA_ERR_UNSUPPORTED, "bf16 attention needs hd 64 or 128");
   if (dtype == ZSAA_F32 && (hd < 1 || hd > 128)) return fail(ZSAA_ERR_UNSUPPORTED, "f32 attention needs hd <= 128");
-  ZCK(launch_attention(dtype, qkv, B, N, Hq, Hkv, hd, out, lse, causal ? 1 : 0,
-                       reinterpret_cast<cudaStream_t>(stream)));
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int* status = shared_status();
+  if (dtype == ZSAA_BF16 && hd == 64 && status != nullptr) {  // the tcgen05 kernel, V^T scratch
+    void* vt = nullptr;
+    ZCK(cudaMallocAsync(&vt, attention_tc_vt_elems(B, N, Hkv) * 2, s));
+    cudaError_t e = launch_attention_tc(qkv, vt, B, N, Hq, Hkv, out, lse, causal ? 1 : 0, status, s);
+    cudaError_t e2 = cudaFreeAsync(vt, s);
+    ZCK(e);
+    ZCK(e2);
+    return ZSAA_OK;
+  }
+  ZCK(launch_attention(dtype, qkv, B, N, Hq, Hkv, hd, out, lse, causal ? 1 : 0, s));
   return ZSAA_OK;
 }
 

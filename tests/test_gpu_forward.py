@@ -252,6 +252,12 @@ def layerwise_case(z, shape, B, L, accel, layers):
 
 
 def chained_check(z, model, shape, tokens, sched, ores, accel):
+    """The whole forward chained on the GPU's own outputs (oracle indices forced):
+    bf16 storage points drift ~1 ulp per layer, so the final rows and the logits
+    must stay within the noise floor 2^-7 sqrt(n_layers) of their scale.  Every
+    sequence of the batch is the same one (identical rows on the GPU), so the
+    classifier's logits are only n_classes distinct numbers: their mean error
+    is no statistic, and the final hidden row (d numbers) carries the check."""
     B, L = tokens.shape
     n = shape.n_layers
     forced = []
@@ -261,12 +267,19 @@ def chained_check(z, model, shape, tokens, sched, ores, accel):
     tok = torch.from_numpy(np.repeat(tokens[:1], B, 0)).cuda()
     lg = torch.empty((B, shape.n_classes) if shape.n_classes else (B, sched[-1], shape.vocab),
                      device="cuda", dtype=torch.float32)
-    z.zsaa_forward_ex(model, tok, B, L, accel, lg, None, forced_idx=fdev)
+    hout = torch.empty(B, sched[-1], shape.d_model, device="cuda", dtype=torch.bfloat16)
+    z.zsaa_forward_ex(model, tok, B, L, accel, lg, None, forced_idx=fdev, hidden_out=hout)
     z.zsaa_sync(model)
+    drift = 2.0 ** -7 * np.sqrt(n)
+    href = ores["final_hidden"][0]
+    herr = np.abs(hout[0].float().cpu().numpy().astype(np.float64) - href)
+    assert herr.mean() <= drift * np.abs(href).mean(), (herr.mean(), np.abs(href).mean())
     ref = np.repeat(ores["logits"], B, 0)
     mx, mean = logits_report(lg.cpu().numpy(), ref)
-    floor = 2.0 ** -7 * np.sqrt(n) * ref.std()
-    assert mean <= floor and mx <= 8 * floor, (mx, mean, floor)
+    floor = drift * ref.std()
+    assert mx <= 8 * floor, (mx, floor)
+    if not shape.n_classes:
+        assert mean <= floor, (mean, floor)
 
 
 def test_full_size_1b_layerwise_and_head(z):
