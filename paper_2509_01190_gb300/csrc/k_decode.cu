@@ -53,20 +53,26 @@ __global__ void kv_write_kernel(const bf16* __restrict__ qkv, int ld,
 
 // One CTA per (KV group, sequence): RoPE and bf16 rounding of the group's PER
 // query heads and of its key, append of key/value to the cache, then Eq. 1 of
-// the PER queries over the cached rows.  4 warps take interleaved blocks of 32
+// the PER queries over the cached rows.  8 warps take interleaved blocks of 32
 // keys (one key per lane for the dot products, then one head dimension slice
 // per lane for P V) with an online softmax in the log2 domain; the warps'
 // partial results are merged at the end.
+// W warps per CTA: the 32-key blocks are walked serially within a warp, so
+// more warps shorten the chain (8: registers stay unspilled at 255 a thread).
 template <int HD, int PER>
-__global__ void __launch_bounds__(128)
+constexpr int decode_warps() { return 8; }
+
+template <int HD, int PER>
+__global__ void __launch_bounds__(decode_warps<HD, PER>() * 32)
     decode_attn_kernel(const float* __restrict__ qkv32, int ld, int Hq, int Hkv, KvLayer c,
                        const int* __restrict__ step, int L0, const float* __restrict__ cos_t,
                        const float* __restrict__ sin_t, bf16* __restrict__ out) {
   pdl_trigger();
   constexpr int HALF = HD / 2, DPL = HD / 32;  // head dims per lane in P V
   __shared__ __align__(16) float qs[PER][HD];
-  __shared__ float wm[4][PER], wl[4][PER];
-  __shared__ float wacc[4][PER][HD];
+  constexpr int W = decode_warps<HD, PER>();
+  __shared__ float wm[W][PER], wl[W][PER];
+  __shared__ float wacc[W][PER][HD];
   const int g = blockIdx.x, b = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   pdl_wait();
@@ -108,7 +114,7 @@ __global__ void __launch_bounds__(128)
 #pragma unroll
     for (int e = 0; e < DPL; ++e) acc[h][e] = 0.f;
   }
-  for (int j0 = warp * 32; j0 < n_keys; j0 += 128) {
+  for (int j0 = warp * 32; j0 < n_keys; j0 += W * 32) {
     const int j = j0 + lane;
     float sc[PER];
     if (j < n_keys) {
@@ -191,10 +197,10 @@ __global__ void __launch_bounds__(128)
     const int h = i / HD, dd = i % HD;
     float mx = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < 4; ++w) mx = fmaxf(mx, wm[w][h]);
+    for (int w = 0; w < W; ++w) mx = fmaxf(mx, wm[w][h]);
     float num = 0.f, den = 0.f;
 #pragma unroll
-    for (int w = 0; w < 4; ++w) {
+    for (int w = 0; w < W; ++w) {
       const float f = wm[w][h] == -INFINITY ? 0.f : exp2f(wm[w][h] - mx);
       num = fmaf(f, wacc[w][h][dd], num);
       den = fmaf(f, wl[w][h], den);
@@ -215,10 +221,10 @@ cudaError_t run_decode(int per, dim3 grid, cudaStream_t s, const float* qkv32, i
                        int Hkv, const KvLayer& c, const int* step, int L0, const float* cos_t,
                        const float* sin_t, bf16* out) {
   switch (per) {
-    case 1: ZSAA_LAUNCH(decode_attn_kernel<HD, 1>, grid, dim3(128), 0, s, qkv32, ld, Hq, Hkv, c, step, L0, cos_t, sin_t, out); break;
-    case 2: ZSAA_LAUNCH(decode_attn_kernel<HD, 2>, grid, dim3(128), 0, s, qkv32, ld, Hq, Hkv, c, step, L0, cos_t, sin_t, out); break;
-    case 4: ZSAA_LAUNCH(decode_attn_kernel<HD, 4>, grid, dim3(128), 0, s, qkv32, ld, Hq, Hkv, c, step, L0, cos_t, sin_t, out); break;
-    case 8: ZSAA_LAUNCH(decode_attn_kernel<HD, 8>, grid, dim3(128), 0, s, qkv32, ld, Hq, Hkv, c, step, L0, cos_t, sin_t, out); break;
+    case 1: ZSAA_LAUNCH(decode_attn_kernel<HD, 1>, grid, dim3(decode_warps<HD, 1>() * 32), 0, s, qkv32, ld, Hq, Hkv, c, step, L0, cos_t, sin_t, out); break;
+    case 2: ZSAA_LAUNCH(decode_attn_kernel<HD, 2>, grid, dim3(decode_warps<HD, 2>() * 32), 0, s, qkv32, ld, Hq, Hkv, c, step, L0, cos_t, sin_t, out); break;
+    case 4: ZSAA_LAUNCH(decode_attn_kernel<HD, 4>, grid, dim3(decode_warps<HD, 4>() * 32), 0, s, qkv32, ld, Hq, Hkv, c, step, L0, cos_t, sin_t, out); break;
+    case 8: ZSAA_LAUNCH(decode_attn_kernel<HD, 8>, grid, dim3(decode_warps<HD, 8>() * 32), 0, s, qkv32, ld, Hq, Hkv, c, step, L0, cos_t, sin_t, out); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaSuccess;
