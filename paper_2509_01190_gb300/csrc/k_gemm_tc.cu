@@ -646,6 +646,9 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
   // a handful of rows: 128-row tiles would idle most of the tensor core and
   // most SMs; stream the weights instead
   if (skinny_supported(A, lda, W, epi, p)) return launch_gemm_skinny(A, lda, W, epi, p, s);
+  // a few hundred rows: weight band as the 128-row operand, K split over a cluster
+  if (swap_preferred(epi, p.M) && swap_supported(A, lda, W, epi, p))
+    return launch_gemm_swap(A, lda, W, epi, p, s);
   const int sms = num_sms();
   const int vn = epi == kEpiSwiGLU ? 2 * p.N : p.N;
   const int m_tiles = (p.M + BM - 1) / BM;

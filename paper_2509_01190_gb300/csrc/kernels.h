@@ -105,6 +105,21 @@ bool skinny_supported(const void* A, int lda, const TcWeights& W, int epi, const
 cudaError_t launch_gemm_skinny(const void* A, int lda, const TcWeights& W, int epi,
                                const GemmParams& p, cudaStream_t s);
 
+// bf16 GEMM with the operands swapped (k_gemm_swap.cu) for kSkinnyMaxM < M <=
+// kSwapMaxM: the weight band is the 128-row tcgen05 operand, the activation
+// rows (blocks of at most kSwapRowBlock) the MMA's N side, and K is split over
+// a thread-block cluster whose partial sums meet in distributed shared memory.
+// Every epilogue; K % 64 == 0, N % 16 == 0, lda % 8 == 0, ldo % 4 == 0,
+// 16-byte aligned pointers, weight row blocks on 128-row boundaries, RoPE with
+// hd dividing 128.  launch_gemm_tc routes such calls here.
+constexpr int kSwapMaxM = 1024;
+constexpr int kSwapRowBlock = 256;
+bool swap_supported(const void* A, int lda, const TcWeights& W, int epi, const GemmParams& p);
+// Whether launch_gemm_tc takes the swapped kernel for this epilogue and row count.
+bool swap_preferred(int epi, int M);
+cudaError_t launch_gemm_swap(const void* A, int lda, const TcWeights& W, int epi,
+                             const GemmParams& p, cudaStream_t s);
+
 // fp32 CUDA-core GEMM, same epilogues (kEpiRope is applied by launch_rope_f32).
 cudaError_t launch_gemm_f32(const float* A, int lda, const float* W, const float* W2, int epi,
                             const GemmParams& p, cudaStream_t s);
