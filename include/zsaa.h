@@ -328,8 +328,11 @@ zsaa_status zsaa_score_select_noalloc(const void* hidden, int B, int L, int d, i
 /* Single steps of the path, for per-kernel checks and timing.  All pointers
  * device; shapes as stated.
  * zsaa_op_linear: out[M,N] = epilogue(A[M,K] W[N,K]^T); dtype ZSAA_BF16 uses
- * the tcgen05 GEMM (M <= 16 without RoPE: the weight-streaming GEMM), ZSAA_F32
- * the fp32 CUDA-core GEMM.  The bf16 kernels start reading W before the
+ * the tcgen05 GEMMs (M <= 16 without RoPE: the weight-streaming GEMM; up to a
+ * few hundred rows, by epilogue: the swapped-operand GEMM whose thread-block
+ * cluster adds its split-K partials in a fixed order, so results do not depend
+ * on timing; larger M: the persistent tiled GEMM), ZSAA_F32 the fp32 CUDA-core
+ * GEMM.  The bf16 kernels start reading W before the
  * previous library kernel on the stream has finished: W and W2 must not be
  * written by that kernel.  epilogue:
  *   0 store (out has dtype; bf16 rounds once),
