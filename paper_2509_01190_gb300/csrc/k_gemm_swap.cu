@@ -50,7 +50,7 @@ constexpr int SW_WARPS = SW_THREADS / 32;
 constexpr int SW_DRAIN_WARPS = 8;  // warps 2..9 copy the accumulator out of TMEM
 constexpr int SW_W_BYTES = SW_BAND * SW_BK * 2;
 constexpr int SW_MAX_CLUSTER = 8;
-constexpr int SW_RING_BUDGET = 196 * 1024;  // bytes of stage ring per CTA
+constexpr int SW_RING_BUDGET = 220 * 1024;  // bytes of stage ring per CTA
 constexpr int SW_MAX_STAGES = 8;
 
 struct SwMaps {
@@ -549,10 +549,12 @@ cudaError_t run_swap(const void* A, int lda, const TcWeights& W, const GemmParam
   const int nrb2 = (p.M + sh.Mp - 1) / sh.Mp;
   // A pass of the producer and MMA loops costs several hundred cycles whatever
   // a stage holds, so a stage takes as many 64-wide k-blocks (up to 4) as
-  // still leaves two stages in the ring.
+  // still leaves two stages in the ring (a TMA probe on one SM streamed best
+  // with about 100 KB per stage).
   const int kblock = SW_W_BYTES + sh.Mp * SW_BK * 2;
-  sh.ksub = 4;
-  while (sh.ksub > 1 && 2 * sh.ksub * kblock > SW_RING_BUDGET) sh.ksub /= 2;
+  sh.ksub = SW_RING_BUDGET / (2 * kblock);
+  if (sh.ksub > 4) sh.ksub = 4;
+  if (sh.ksub < 1) sh.ksub = 1;
   sh.stages = SW_RING_BUDGET / (sh.ksub * kblock);
   if (sh.stages > SW_MAX_STAGES) sh.stages = SW_MAX_STAGES;
   sh.nkb = p.K / SW_BK;
