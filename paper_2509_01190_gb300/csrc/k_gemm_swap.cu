@@ -53,6 +53,14 @@ constexpr int SW_MAX_CLUSTER = 8;
 constexpr int SW_RING_BUDGET = 220 * 1024;  // bytes of stage ring per CTA
 constexpr int SW_MAX_STAGES = 8;
 
+// Internal epilogue id: float32 store for very wide outputs (the LM head):
+// each CTA owns sh.nb adjacent 128-row weight bands, one TMEM accumulator per
+// band at columns i * sh.band_cols, all fed by the same activation tile, no
+// split-K, logits written straight from TMEM.  The activation rows are then
+// streamed once per nb bands instead of once per band.
+constexpr int kSwapHeadF32 = 6;
+constexpr int kSwapHeadMinN = 32768;
+
 struct SwMaps {
   CUtensorMap x, w0, w1, w2;
 };
@@ -61,6 +69,8 @@ struct SwShape {
   int Mp;         // activation rows per row block (multiple of 16, <= 256): the MMA's N
   int stages;     // depth of the stage ring
   int ksub;       // k-blocks of 64 per stage
+  int nb;         // weight bands per CTA (kSwapHeadF32; else 1)
+  int band_cols;  // TMEM columns between the bands' accumulators
   int nkb;        // k-blocks of 64
   int n1, n2;     // weight row blocks (non-SwiGLU): w0 [0, n1), w1 [n1, n2), w2 [n2, N)
   uint32_t tmem_cols;
@@ -288,13 +298,15 @@ template <int EPI>
 __global__ void __launch_bounds__(SW_THREADS, 1)
     gemm_swap_kernel(const __grid_constant__ SwMaps maps, const SwShape sh, const GemmParams p) {
   constexpr bool DUAL = EPI == kEpiSwiGLU;
+  constexpr bool HEAD = EPI == kSwapHeadF32;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   const int X_BYTES = sh.Mp * SW_BK * 2;  // one activation sub-tile [Mp x 64]
+  const int WSUB = (HEAD ? sh.nb : 1) * SW_W_BYTES;  // weight bytes of one k-block
   const int STAGES = sh.stages, KSUB = sh.ksub;
   uint8_t* sW = smem;                                     // [STAGES][KSUB] weight sub-tiles
-  uint8_t* sX = smem + STAGES * KSUB * SW_W_BYTES;        // [STAGES][KSUB] activation sub-tiles
+  uint8_t* sX = smem + STAGES * KSUB * WSUB;              // [STAGES][KSUB] activation sub-tiles
   uint64_t* full = reinterpret_cast<uint64_t*>(sX + STAGES * KSUB * X_BYTES);
   uint64_t* empty = full + SW_MAX_STAGES;
   uint64_t* acc_full = empty + SW_MAX_STAGES;
@@ -341,6 +353,9 @@ __global__ void __launch_bounds__(SW_THREADS, 1)
       if (DUAL) {
         wm0 = &maps.w0;
         wy = band * (SW_BAND / 2);
+      } else if (HEAD) {
+        wm0 = &maps.w0;
+        wy = band * sh.nb * SW_BAND;
       } else {
         const int n0 = band * SW_BAND;
         wm0 = n0 >= sh.n2 ? &maps.w2 : (n0 >= sh.n1 ? &maps.w1 : &maps.w0);
@@ -350,14 +365,18 @@ __global__ void __launch_bounds__(SW_THREADS, 1)
       // weight sub-tiles of stage j into slot s
       auto load_w = [&](int s, int j) {
         for (int u = 0; u < nsub_of(j); ++u) {
-          uint8_t* d = sW + (s * KSUB + u) * SW_W_BYTES;
+          uint8_t* d = sW + (s * KSUB + u) * WSUB;
           const int x = (kb0 + j * KSUB + u) * SW_BK;
-          tma_load_2d(d, wm0, x, wy, &full[s]);
+          if (HEAD) {  // nb bands; rows past N read as zeros
+            for (int i = 0; i < sh.nb; ++i) tma_load_2d(d + i * SW_W_BYTES, wm0, x, wy + i * SW_BAND, &full[s]);
+          } else {
+            tma_load_2d(d, wm0, x, wy, &full[s]);
+          }
           if (DUAL) tma_load_2d(d + (SW_BAND / 2) * 128, wm1, x, wy, &full[s]);
         }
       };
       auto stage_bytes = [&](int j) {
-        return static_cast<uint32_t>(nsub_of(j) * (SW_W_BYTES + X_BYTES));
+        return static_cast<uint32_t>(nsub_of(j) * (WSUB + X_BYTES));
       };
       const int npre = min(STAGES, nst);
       for (int j = 0; j < npre; ++j) {
@@ -405,12 +424,20 @@ __global__ void __launch_bounds__(SW_THREADS, 1)
         tc_fence_after();
         const int nsub = min(KSUB, kb1 - (kb0 + j * KSUB));
         for (int u = 0; u < nsub; ++u) {
-          const uint32_t w_base = smem_u32(sW + (s * KSUB + u) * SW_W_BYTES);
+          const uint32_t w_base = smem_u32(sW + (s * KSUB + u) * WSUB);
           const uint32_t x_base = smem_u32(sX + (s * KSUB + u) * X_BYTES);
 #pragma unroll
-          for (int k = 0; k < SW_BK / 16; ++k)
-            tc_mma_bf16(tmem, sdesc_sw128(w_base + k * 32), sdesc_sw128(x_base + k * 32), idesc,
-                        (j > 0 || u > 0 || k > 0) ? 1u : 0u);
+          for (int k = 0; k < SW_BK / 16; ++k) {
+            const uint32_t acc = (j > 0 || u > 0 || k > 0) ? 1u : 0u;
+            if (HEAD) {
+              for (int i = 0; i < sh.nb; ++i)
+                tc_mma_bf16(tmem + static_cast<uint32_t>(i * sh.band_cols),
+                            sdesc_sw128(w_base + i * SW_W_BYTES + k * 32), sdesc_sw128(x_base + k * 32),
+                            idesc, acc);
+            } else {
+              tc_mma_bf16(tmem, sdesc_sw128(w_base + k * 32), sdesc_sw128(x_base + k * 32), idesc, acc);
+            }
+          }
         }
         tc_commit(&empty[s]);
       }
@@ -425,7 +452,28 @@ __global__ void __launch_bounds__(SW_THREADS, 1)
     const int h = (warp - 2) >> 2;
     const int n = quad * 32 + lane;
     const bool ok = __all_sync(0xffffffffu, mbar_wait_ab(acc_full, 0, p.status, abort_flag));
-    if (ok) {
+    if (ok && HEAD) {
+      // logits[row0 + m, (band*nb + i)*128 + n] straight from TMEM: a warp stores
+      // 32 adjacent floats of one row per instruction
+      pdl_wait();
+      tc_fence_after();
+      const uint32_t tb = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+      float* out = static_cast<float*>(p.out);
+      for (int i = 0; i < sh.nb; ++i) {
+        const int col = (band * sh.nb + i) * SW_BAND + n;
+#pragma unroll 1
+        for (int c = 16 * h; c < sh.Mp; c += 32) {
+          uint32_t r[16];
+          tmem_ld16(tb + static_cast<uint32_t>(i * sh.band_cols + c), r);
+          tmem_ld_wait();
+          if (col < p.N) {
+#pragma unroll
+            for (int e = 0; e < 16; ++e)
+              if (c + e < rows) out[static_cast<size_t>(row0 + c + e) * p.ldo + col] = __uint_as_float(r[e]);
+          }
+        }
+      }
+    } else if (ok) {
       tc_fence_after();
       fence_proxy_async_smem();  // the ring was last written by TMA, read by the MMAs
       const uint32_t tb = tmem + (static_cast<uint32_t>(quad * 32) << 16);
@@ -450,7 +498,7 @@ __global__ void __launch_bounds__(SW_THREADS, 1)
   // ---- reduction over the cluster and epilogue: CTA `rank` finishes rows
   // [rank rows / S, (rank + 1) rows / S) of this block.
   pdl_wait();
-  if (*abort_flag == 0) {
+  if (!HEAD && *abort_flag == 0) {
     uint32_t src[SW_MAX_CLUSTER];
     const uint32_t red_local = smem_u32(red);
 #pragma unroll
@@ -480,8 +528,8 @@ bool encode_sw(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t rows, u
   return r == CUDA_SUCCESS;
 }
 
-size_t smem_bytes(int Mp, int stages, int ksub) {
-  return static_cast<size_t>(stages) * ksub * (SW_W_BYTES + Mp * SW_BK * 2) + 1024 + 256;
+size_t smem_bytes(int wsub, int Mp, int stages, int ksub) {
+  return static_cast<size_t>(stages) * ksub * (wsub + Mp * SW_BK * 2) + 1024 + 256;
 }
 
 template <int EPI>
@@ -541,6 +589,7 @@ cudaError_t run_swap(const void* A, int lda, const TcWeights& W, const GemmParam
   cudaError_t e = ensure_attr<EPI>();
   if (e != cudaSuccess) return e;
   constexpr bool DUAL = EPI == kEpiSwiGLU;
+  constexpr bool HEAD = EPI == kSwapHeadF32;
   // row blocks of at most 256 rows, as even as 16-row granularity allows
   const int nrb = (p.M + kSwapRowBlock - 1) / kSwapRowBlock;
   const int per = (p.M + nrb - 1) / nrb;
@@ -551,7 +600,12 @@ cudaError_t run_swap(const void* A, int lda, const TcWeights& W, const GemmParam
   // a stage holds, so a stage takes as many 64-wide k-blocks (up to 4) as
   // still leaves two stages in the ring (a TMA probe on one SM streamed best
   // with about 100 KB per stage).
-  const int kblock = SW_W_BYTES + sh.Mp * SW_BK * 2;
+  // HEAD: as many 128-row bands per CTA as TMEM holds accumulators for (up to 4)
+  sh.band_cols = 32;
+  while (sh.band_cols < sh.Mp) sh.band_cols += 32;
+  sh.nb = HEAD ? 512 / sh.band_cols : 1;
+  if (sh.nb > 4) sh.nb = 4;
+  const int kblock = sh.nb * SW_W_BYTES + sh.Mp * SW_BK * 2;
   sh.ksub = SW_RING_BUDGET / (2 * kblock);
   if (sh.ksub > 4) sh.ksub = 4;
   if (sh.ksub < 1) sh.ksub = 1;
@@ -562,16 +616,18 @@ cudaError_t run_swap(const void* A, int lda, const TcWeights& W, const GemmParam
   sh.n2 = DUAL ? p.N : W.n2;
   uint32_t cols = 32;
   while (cols < static_cast<uint32_t>(sh.Mp)) cols <<= 1;
-  sh.tmem_cols = cols;
-  const int bands = DUAL ? (p.N + SW_BAND / 2 - 1) / (SW_BAND / 2) : (p.N + SW_BAND - 1) / SW_BAND;
-  const size_t smem = smem_bytes(sh.Mp, sh.stages, sh.ksub);
+  sh.tmem_cols = HEAD ? 512 : cols;
+  const int bands = DUAL   ? (p.N + SW_BAND / 2 - 1) / (SW_BAND / 2)
+                    : HEAD ? (p.N + sh.nb * SW_BAND - 1) / (sh.nb * SW_BAND)
+                           : (p.N + SW_BAND - 1) / SW_BAND;
+  const size_t smem = smem_bytes(sh.nb * SW_W_BYTES, sh.Mp, sh.stages, sh.ksub);
 
   // Cluster size: fewest k-blocks per CTA over the waves the clusters need;
   // a wave costs about two k-blocks of fixed work (launch, TMEM, reduction).
   const int units = bands * nrb2;
   int best = 1;
   double best_cost = 1e30;
-  for (int S = 1; S <= SW_MAX_CLUSTER && S <= sh.nkb; ++S) {
+  for (int S = 1; S <= (HEAD ? 1 : SW_MAX_CLUSTER) && S <= sh.nkb; ++S) {  // HEAD: no split-K
     const int mc = max_clusters<EPI>(S, smem);
     if (mc <= 0) continue;
     const int waves = (units + mc - 1) / mc;
@@ -647,7 +703,9 @@ cudaError_t launch_gemm_swap(const void* A, int lda, const TcWeights& W, int epi
     case kEpiStore: return run_swap<kEpiStore>(A, lda, W, p, s);
     case kEpiResid: return run_swap<kEpiResid>(A, lda, W, p, s);
     case kEpiSwiGLU: return run_swap<kEpiSwiGLU>(A, lda, W, p, s);
-    case kEpiStoreF32: return run_swap<kEpiStoreF32>(A, lda, W, p, s);
+    case kEpiStoreF32:  // very wide outputs (the LM head): several bands per CTA
+      return p.N >= kSwapHeadMinN ? run_swap<kSwapHeadF32>(A, lda, W, p, s)
+                                  : run_swap<kEpiStoreF32>(A, lda, W, p, s);
     case kEpiRope: return run_swap<kEpiRope>(A, lda, W, p, s);
     default: return cudaErrorInvalidValue;
   }
