@@ -346,6 +346,10 @@ struct zsaa_model {
   bool use_graphs = true;
   std::list<GraphEntry> graphs;
   cudaStream_t capture_stream = nullptr;  // graphs are recorded here, launched on the caller's
+  // side stream of a pruning layer's O-projection (forked after the attention,
+  // joined before the gather), created on first use
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
 };
 
 // Pruned KV cache for generation (zsaa_cache_create).
@@ -425,6 +429,9 @@ void free_model(zsaa_model* m) {
   for (auto& g : m->graphs)
     if (g.exec) cudaGraphExecDestroy(g.exec);
   if (m->capture_stream) cudaStreamDestroy(m->capture_stream);
+  if (m->side) cudaStreamDestroy(m->side);
+  if (m->ev_fork) cudaEventDestroy(m->ev_fork);
+  if (m->ev_join) cudaEventDestroy(m->ev_join);
   void* ptrs[] = {m->h[0], m->h[1], m->x, m->qkv, m->attn, m->act, m->lse, m->vt, m->colmass, m->vnorm,
                   m->scores, m->idx, m->pos[0], m->pos[1], m->rope_cos, m->rope_sin,
                   m->splitk_ws, m->splitk_flags, m->status, m->stage_tok, m->stage_logits,
@@ -589,6 +596,22 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
         ZCK(launch_attention(dt, m->qkv, B, N, Hq, Hkv, hd, m->attn, m->lse, causal, s));
       }
     }
+    // A pruning layer's column mass and selection need only q, k and the row
+    // normalisers, so its O-projection runs beside them on the side stream;
+    // the gather, which reads the updated rows, joins it.  (Not while tracing,
+    // which times each launch on the one stream.)
+    const bool fork = !m->tracing && prunes(c, l) && sched[l] < N;
+    cudaStream_t so = s;
+    if (fork) {
+      if (m->side == nullptr) {
+        ZCK(cudaStreamCreateWithFlags(&m->side, cudaStreamNonBlocking));
+        ZCK(cudaEventCreateWithFlags(&m->ev_fork, cudaEventDisableTiming));
+        ZCK(cudaEventCreateWithFlags(&m->ev_join, cudaEventDisableTiming));
+      }
+      ZCK(cudaEventRecord(m->ev_fork, s));
+      ZCK(cudaStreamWaitEvent(m->side, m->ev_fork, 0));
+      so = m->side;
+    }
     {
       GemmParams q{};
       q.M = M;
@@ -600,9 +623,10 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
       TcWeights W{LW(m, li, kWo), nullptr, nullptr, d, d};
       TRACE("gemm_o_resid", 2.0 * Md * d * m->dq, (Md * m->dq + static_cast<double>(d) * m->dq + 2.0 * Md * d) * es);
       trace_scope_.kernels = 0;
-      st = linear(m, m->attn, m->dq, W, kEpiResid, q, s, &trace_scope_.kernels);
+      st = linear(m, m->attn, m->dq, W, kEpiResid, q, so, &trace_scope_.kernels);
       if (st != ZSAA_OK) return st;
     }
+    if (fork) ZCK(cudaEventRecord(m->ev_join, so));
     // Elimination (Sec. 3.3), between attention and MLP: the scores come from
     // this layer's attention and the MLP acts on each row alone, so the kept
     // rows come out exactly as if the whole layer ran first -- but the MLP
@@ -650,6 +674,7 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
           ZCK(cudaMemcpyAsync(opts->idx_out + off_idx, idx, sizeof(int32_t) * B * k,
                               cudaMemcpyDeviceToDevice, s));
         if (k < N) {
+          if (fork) ZCK(cudaStreamWaitEvent(s, m->ev_join, 0));  // the O-projection has updated h
           if (fuse_norm) {  // the kept rows and their pre-MLP RMSNorm in one pass
             TRACE("gather_norm", 0.0, static_cast<double>(B) * k * (3.0 * d * es + 12.0));
             ZCK(launch_rows_norm(h, nullptr, 0, 0, idx, N, k, m->pos[cur], B * k, d,
