@@ -377,6 +377,20 @@ struct zsaa_cache {
 
 namespace {
 
+// Make the model's side stream wait for the work enqueued on s so far
+// (creating the stream and its events on first use).
+cudaError_t fork_side(zsaa_model* m, cudaStream_t s) {
+  if (m->side == nullptr) {
+    cudaError_t e = cudaStreamCreateWithFlags(&m->side, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&m->ev_fork, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&m->ev_join, cudaEventDisableTiming);
+    if (e != cudaSuccess) return e;
+  }
+  cudaError_t e = cudaEventRecord(m->ev_fork, s);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(m->side, m->ev_fork, 0);
+  return e;
+}
+
 const void* LW(const zsaa_model* m, int layer, int slot) {
   return m->layers[static_cast<size_t>(layer) * 9 + slot];
 }
@@ -603,13 +617,7 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
     const bool fork = !m->tracing && prunes(c, l) && sched[l] < N;
     cudaStream_t so = s;
     if (fork) {
-      if (m->side == nullptr) {
-        ZCK(cudaStreamCreateWithFlags(&m->side, cudaStreamNonBlocking));
-        ZCK(cudaEventCreateWithFlags(&m->ev_fork, cudaEventDisableTiming));
-        ZCK(cudaEventCreateWithFlags(&m->ev_join, cudaEventDisableTiming));
-      }
-      ZCK(cudaEventRecord(m->ev_fork, s));
-      ZCK(cudaStreamWaitEvent(m->side, m->ev_fork, 0));
+      ZCK(fork_side(m, s));
       so = m->side;
     }
     {
@@ -863,6 +871,14 @@ zsaa_status run_forward_masked(zsaa_model* m, const int32_t* tok, int B, int L, 
       ZCK(launch_attention(dt, m->qkv, B, L, Hq, Hkv, hd, m->attn, m->lse, causal, s, nullptr,
                            m->alive));
     }
+    // O-projection beside the column mass and selection (see run_forward);
+    // the MLP's RMSNorm joins it
+    const bool fork = !m->tracing && prunes(c, l);
+    cudaStream_t so = s;
+    if (fork) {
+      ZCK(fork_side(m, s));
+      so = m->side;
+    }
     {
       GemmParams q{};
       q.M = M;
@@ -874,9 +890,10 @@ zsaa_status run_forward_masked(zsaa_model* m, const int32_t* tok, int B, int L, 
       TcWeights W{LW(m, li, kWo), nullptr, nullptr, d, d};
       TRACE("gemm_o_resid", 2.0 * Md * d * m->dq, (Md * m->dq + static_cast<double>(d) * m->dq + 2.0 * Md * d) * es);
       trace_scope_.kernels = 0;
-      st = linear(m, m->attn, m->dq, W, kEpiResid, q, s, &trace_scope_.kernels);
+      st = linear(m, m->attn, m->dq, W, kEpiResid, q, so, &trace_scope_.kernels);
       if (st != ZSAA_OK) return st;
     }
+    if (fork) ZCK(cudaEventRecord(m->ev_join, so));
     if (prunes(c, l)) {
       const int k = sched[l];
       const bool want_scores = opts && opts->scores_out;
@@ -909,6 +926,7 @@ zsaa_status run_forward_masked(zsaa_model* m, const int32_t* tok, int B, int L, 
       off_idx += static_cast<size_t>(B) * k;
       off_scores += static_cast<size_t>(B) * L;
     }
+    if (fork) ZCK(cudaStreamWaitEvent(s, m->ev_join, 0));  // the O-projection has updated h
     // the MLP of every row, marked or not (the formulation removes nothing)
     {
       TRACE("rmsnorm", 0.0, 2.0 * Md * d * es);
@@ -1083,6 +1101,13 @@ zsaa_status run_forward_varlen(zsaa_model* m, const int32_t* tok, const int32_t*
       TRACE("attention", 4.0 * pairs * Hq * hd, Md * (m->ld_qkv + m->dq) * es + static_cast<double>(B) * Hq * Nm * 4.0);
       ZCK(launch_attention(dt, m->qkv, B, Nm, Hq, Hkv, hd, m->attn, m->lse, causal, s, cu_dev(li)));
     }
+    // O-projection beside the column mass and selection (see run_forward)
+    const bool fork = !m->tracing && prunes(c, l) && rows[l] < M && Nm <= kSelectPartsMaxN;
+    cudaStream_t so = s;
+    if (fork) {
+      ZCK(fork_side(m, s));
+      so = m->side;
+    }
     {
       GemmParams q{};
       q.M = M;
@@ -1094,9 +1119,10 @@ zsaa_status run_forward_varlen(zsaa_model* m, const int32_t* tok, const int32_t*
       TcWeights W{LW(m, li, kWo), nullptr, nullptr, d, d};
       TRACE("gemm_o_resid", 2.0 * Md * d * m->dq, (Md * m->dq + static_cast<double>(d) * m->dq + 2.0 * Md * d) * es);
       trace_scope_.kernels = 0;
-      st = linear(m, m->attn, m->dq, W, kEpiResid, q, s, &trace_scope_.kernels);
+      st = linear(m, m->attn, m->dq, W, kEpiResid, q, so, &trace_scope_.kernels);
       if (st != ZSAA_OK) return st;
     }
+    if (fork) ZCK(cudaEventRecord(m->ev_join, so));
     // elimination between attention and MLP (see run_forward), per sequence
     bool mlp_x_ready = false;
     if (prunes(c, l)) {
@@ -1124,6 +1150,7 @@ zsaa_status run_forward_varlen(zsaa_model* m, const int32_t* tok, const int32_t*
           ZCK(cudaMemcpyAsync(opts->idx_out + off_idx, idx, sizeof(int32_t) * rows[l],
                               cudaMemcpyDeviceToDevice, s));
         if (shrinks) {
+          if (fork) ZCK(cudaStreamWaitEvent(s, m->ev_join, 0));  // the O-projection has updated h
           TRACE("gather_norm", 0.0, static_cast<double>(rows[l]) * (3.0 * d * es + 12.0));
           ZCK(launch_rows_norm(h, nullptr, 0, 0, idx, Nm, 0, m->pos[cur], rows[l], d,
                                LW(m, li, kMlpNorm), c.rms_eps, m->h[cur ^ 1], m->x, m->pos[cur ^ 1],
