@@ -1,16 +1,17 @@
 // Causal (or bidirectional) grouped-query attention, Eq. 1, on the sm_103a
-// tensor cores, for bf16 heads of 64 dims.
+// tensor cores, for bf16 heads of 64 or 128 dims (HD).
 //
 // Persistent: one CTA per SM walks work items (query block of 128 rows, query
 // head, sequence; longest first) and streams their key blocks through one
 // pipeline, so TMA, MMA and softmax of consecutive items overlap.  For every
-// key block of 128 (causal: up to the diagonal):
-//   MMA1  S = Q K^T          (tcgen05, M = 128 queries, N = 128 keys, K = 64) -> TMEM
+// key block of BN (128 keys for HD = 64, 64 for HD = 128, so that both fit the
+// same shared-memory ring; causal: up to the diagonal):
+//   MMA1  S = Q K^T          (tcgen05, M = 128 queries, N = BN keys, K = HD) -> TMEM
 //   softmax warps (one query row per thread, TMEM lane = row): scale, mask,
 //         running max m and sum l in the log2 domain, P = exp2(s - m) split as
 //         a bf16 pair P_hi + P_lo (R13) written to shared memory in the 128-byte
 //         swizzled K-major layout the tensor core reads
-//   MMA2  O_blk = P_hi V + P_lo V  (M = 128, N = 64 head dims, K = 128 keys) -> TMEM,
+//   MMA2  O_blk = P_hi V + P_lo V  (M = 128, N = HD head dims, K = BN keys) -> TMEM,
 //         V given transposed (V^T[d][key], from a transpose kernel) so both
 //         operands are K-major
 //   softmax warps: O = O * exp2(m_prev - m) + O_blk in registers.
@@ -33,24 +34,34 @@ namespace zsaa {
 namespace {
 
 constexpr int AT_BM = 128;  // queries per CTA
-constexpr int AT_BN = 128;  // keys per block
-constexpr int AT_HD = 64;
 constexpr int AT_THREADS = 320;
 constexpr int AT_SOFT_WARPS = 8;
-constexpr int AT_Q_BYTES = AT_BM * AT_HD * 2;         // 16 KB
-constexpr int AT_K_BYTES = AT_BN * AT_HD * 2;         // 16 KB
-constexpr int AT_V_BYTES = AT_HD * AT_BN * 2;         // 16 KB: two 64-key chunks of [64 d x 64 keys]
-constexpr int AT_P_BYTES = AT_BM * AT_BN * 2;         // 32 KB: two 64-key chunks of [128 q x 64 keys]
 constexpr int AT_STAGES = 3;  // K/V^T stages: V stays until MMA2, after the softmax
-// Q[2] | K[2] | V^T[2] | P_hi | P_lo | barriers | row-max exchange [2][2][128] |
-// row-sum exchange [2][128]; +1 KB to align to the 1024 B swizzle atom
-constexpr size_t AT_SMEM = 2 * AT_Q_BYTES + AT_STAGES * (AT_K_BYTES + AT_V_BYTES) + 2 * AT_P_BYTES + 256 +
-                           6 * AT_BM * 4 + 1024;
-constexpr uint32_t AT_TMEM_COLS = 512;  // S[2] (2 x 128) + O[2] (2 x 64), rounded to a power of two
+constexpr uint32_t AT_TMEM_COLS = 512;  // S[2] (2 x BN) + O[2] (2 x HD), rounded to a power of two
+
+// Tile geometry per head size.  Operands are stored as 64-element-wide
+// (128-byte) swizzled chunks: Q [128 q x HD] and K [BN x HD] as HD/64 chunks
+// over the head dims, V^T [HD x BN] and P [128 q x BN] as BN/64 chunks over
+// the keys.
+template <int HD>
+struct AtCfg {
+  static constexpr int BN = HD == 64 ? 128 : 64;  // keys per block
+  static constexpr int Q_BYTES = AT_BM * HD * 2;
+  static constexpr int K_BYTES = BN * HD * 2;
+  static constexpr int V_BYTES = HD * BN * 2;
+  static constexpr int P_BYTES = AT_BM * BN * 2;
+  // Q[2] | K[STAGES] | V^T[STAGES] | P_hi | P_lo | barriers | row-max exchange
+  // [2][2][128] | row-sum exchange [2][128]; +1 KB to align to the swizzle atom
+  static constexpr size_t SMEM = 2 * Q_BYTES + AT_STAGES * (K_BYTES + V_BYTES) + 2 * P_BYTES + 256 +
+                                 6 * AT_BM * 4 + 1024;
+  static constexpr int O_COL = 2 * BN;  // TMEM column of O[0]
+};
+static_assert(AtCfg<64>::SMEM <= 227 * 1024 && AtCfg<128>::SMEM <= 227 * 1024, "shared memory");
+static_assert(2 * AtCfg<64>::BN + 2 * 64 <= 512 && 2 * AtCfg<128>::BN + 2 * 128 <= 512, "TMEM columns");
 
 struct AtArgs {
   float* lse2;  // [B, Hq, N]
-  bf16* out;    // [B*N, Hq*64]
+  bf16* out;    // [B*N, Hq*HD]
   int B, N, Hq, Hkv, n_qb, causal;  // grid: persistent, one CTA per SM
   float scale_log2;
   int* status;
@@ -72,6 +83,7 @@ __device__ __forceinline__ uint32_t swz128(int row, int chunk) {
 struct AtItem {
   int qb, h, b, n_kb;
 };
+template <int BN>
 __device__ __forceinline__ AtItem at_item(int t, const AtArgs& a) {
   AtItem it;
   const int per_qb = a.Hq * a.B;
@@ -79,13 +91,20 @@ __device__ __forceinline__ AtItem at_item(int t, const AtArgs& a) {
   const int r = t % per_qb;
   it.h = r % a.Hq;
   it.b = r / a.Hq;
-  it.n_kb = a.causal ? it.qb + 1 : (a.N + AT_BN - 1) / AT_BN;
+  // causal: the key blocks up to the last query of the block (or the sequence)
+  const int keys = a.causal ? min(a.N, (it.qb + 1) * AT_BM) : a.N;
+  it.n_kb = (keys + BN - 1) / BN;
   return it;
 }
 
+template <int HD>
 __global__ void __launch_bounds__(AT_THREADS, 1)
-    attn_tc_kernel(const __grid_constant__ CUtensorMap tm_qk, const __grid_constant__ CUtensorMap tm_vt,
-                   const AtArgs a) {
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                   const __grid_constant__ CUtensorMap tm_vt, const AtArgs a) {
+  using C = AtCfg<HD>;
+  constexpr int AT_BN = C::BN, AT_HD = HD;
+  constexpr int AT_Q_BYTES = C::Q_BYTES, AT_K_BYTES = C::K_BYTES, AT_V_BYTES = C::V_BYTES,
+                AT_P_BYTES = C::P_BYTES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -131,7 +150,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     fence_barrier_init();
   }
   if (warp == 0 && lane == 0) {
-    prefetch_tmap(&tm_qk);
+    prefetch_tmap(&tm_q);
+    prefetch_tmap(&tm_k);
     prefetch_tmap(&tm_vt);
   }
   if (warp == 1) tmem_alloc(tmem_slot, AT_TMEM_COLS);
@@ -148,7 +168,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       bool ok = true;
       uint32_t J = 0, items = 0, q_issued = 0;
       for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++items) {
-        const AtItem it = at_item(t, a);
+        const AtItem it = at_item<AT_BN>(t, a);
         const int g = it.h / (a.Hq / a.Hkv);
         const int row0 = it.b * a.N;
         const int qs = items & 1;
@@ -158,7 +178,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         }
         ++q_issued;
         mbar_arrive_expect_tx(&q_full[qs], AT_Q_BYTES);
-        tma_load_2d(sQ + qs * AT_Q_BYTES, &tm_qk, it.h * AT_HD, row0 + it.qb * AT_BM, &q_full[qs]);
+        for (int c = 0; c < AT_HD / 64; ++c)
+          tma_load_2d(sQ + qs * AT_Q_BYTES + c * (AT_BM * 128), &tm_q, it.h * AT_HD + c * 64,
+                      row0 + it.qb * AT_BM, &q_full[qs]);
         for (int j = 0; j < it.n_kb; ++j, ++J) {
           const int st = J % AT_STAGES;
           if (!mbar_wait_ab(&kv_empty[st], ((J / AT_STAGES) & 1) ^ 1, a.status, abort_flag)) {
@@ -166,9 +188,11 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
             break;
           }
           mbar_arrive_expect_tx(&kv_full[st], AT_K_BYTES + AT_V_BYTES);
-          tma_load_2d(sK + st * AT_K_BYTES, &tm_qk, (a.Hq + g) * AT_HD, row0 + j * AT_BN, &kv_full[st]);
-          for (int c = 0; c < 2; ++c)
-            tma_load_2d(sV + st * AT_V_BYTES + c * (AT_V_BYTES / 2), &tm_vt, j * AT_BN + c * 64,
+          for (int c = 0; c < AT_HD / 64; ++c)
+            tma_load_2d(sK + st * AT_K_BYTES + c * (AT_BN * 128), &tm_k, (a.Hq + g) * AT_HD + c * 64,
+                        row0 + j * AT_BN, &kv_full[st]);
+          for (int c = 0; c < AT_BN / 64; ++c)
+            tma_load_2d(sV + st * AT_V_BYTES + c * (AT_HD * 128), &tm_vt, j * AT_BN + c * 64,
                         (it.b * a.Hkv + g) * AT_HD, &kv_full[st]);
         }
       }
@@ -191,14 +215,14 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         if (!mbar_wait_ab(&o_empty[ob], ((J >> 1) & 1) ^ 1, a.status, abort_flag)) return false;
         tc_fence_after();
         const uint32_t v_base = smem_u32(sV + (J % AT_STAGES) * AT_V_BYTES);
-        const uint32_t d_tmem = tmem + 2 * AT_BN + ob * AT_HD;
+        const uint32_t d_tmem = tmem + C::O_COL + ob * AT_HD;
 #pragma unroll
         for (int part = 0; part < 2; ++part) {
           const uint32_t p_base = smem_u32(part ? sPl : sPh);
 #pragma unroll
-          for (int kk = 0; kk < AT_BN / 16; ++kk) {
-            const uint32_t pa = p_base + (kk / 4) * (AT_P_BYTES / 2) + (kk % 4) * 32;
-            const uint32_t va = v_base + (kk / 4) * (AT_V_BYTES / 2) + (kk % 4) * 32;
+          for (int kk = 0; kk < AT_BN / 16; ++kk) {  // 64-key chunk kk/4 of P and of V^T
+            const uint32_t pa = p_base + (kk / 4) * (AT_BM * 128) + (kk % 4) * 32;
+            const uint32_t va = v_base + (kk / 4) * (AT_HD * 128) + (kk % 4) * 32;
             tc_mma_bf16(d_tmem, sdesc_sw128(pa), sdesc_sw128(va), idesc_o, (part | kk) ? 1u : 0u);
           }
         }
@@ -209,7 +233,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
       };
       uint32_t J = 0, items = 0;
       for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++items) {
-        const AtItem it = at_item(t, a);
+        const AtItem it = at_item<AT_BN>(t, a);
         const int qs = items & 1;
         if (!mbar_wait_ab(&q_full[qs], (items >> 1) & 1, a.status, abort_flag)) {
           ok = false;
@@ -227,8 +251,9 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
           const uint32_t k_base = smem_u32(sK + kst * AT_K_BYTES);
           const uint32_t d_tmem = tmem + sb * AT_BN;
 #pragma unroll
-          for (int kk = 0; kk < AT_HD / 16; ++kk)
-            tc_mma_bf16(d_tmem, sdesc_sw128(q_base + kk * 32), sdesc_sw128(k_base + kk * 32), idesc_s,
+          for (int kk = 0; kk < AT_HD / 16; ++kk)  // 64-dim chunk kk/4 of Q and of K
+            tc_mma_bf16(d_tmem, sdesc_sw128(q_base + (kk / 4) * (AT_BM * 128) + (kk % 4) * 32),
+                        sdesc_sw128(k_base + (kk / 4) * (AT_BN * 128) + (kk % 4) * 32), idesc_s,
                         kk > 0 ? 1u : 0u);
           tc_commit(&s_full[sb]);
           if (j + 1 == it.n_kb) tc_commit(&q_empty[qs]);  // this item's Q is read for the last time
@@ -257,7 +282,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
     };
     uint32_t J = 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
-      const AtItem it = at_item(t, a);
+      const AtItem it = at_item<AT_BN>(t, a);
       const int q0 = it.qb * AT_BM, q = q0 + row;
       float m = -INFINITY, l = 0.f;
       float o[OH];
@@ -269,14 +294,17 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         tc_fence_after();
         if (ok) {
           const float cj = corr_ring[Jm & 1];
-          uint32_t r[32];
-          __syncwarp();
-          const uint32_t oaddr = tmem + lane_off + 2 * AT_BN + ob * AT_HD + half * OH;
-          tmem_ld16(oaddr, *reinterpret_cast<uint32_t(*)[16]>(r));
-          tmem_ld16(oaddr + 16, *reinterpret_cast<uint32_t(*)[16]>(r + 16));
-          tmem_ld_wait();
+          const uint32_t oaddr = tmem + lane_off + C::O_COL + ob * AT_HD + half * OH;
 #pragma unroll
-          for (int e = 0; e < OH; ++e) o[e] = fmaf(o[e], cj, __uint_as_float(r[e]));
+          for (int c = 0; c < OH; c += 32) {
+            uint32_t r[32];
+            __syncwarp();
+            tmem_ld16(oaddr + c, *reinterpret_cast<uint32_t(*)[16]>(r));
+            tmem_ld16(oaddr + c + 16, *reinterpret_cast<uint32_t(*)[16]>(r + 16));
+            tmem_ld_wait();
+#pragma unroll
+            for (int e = 0; e < 32; ++e) o[c + e] = fmaf(o[c + e], cj, __uint_as_float(r[e]));
+          }
         }
         tc_fence_before();
         arrive(&o_empty[ob]);
@@ -325,7 +353,7 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
         ok = ok && __all_sync(0xffffffffu, mbar_wait_ab(p_empty, (J & 1) ^ 1, a.status, abort_flag));
         if (ok) {
 #pragma unroll
-          for (int c = 0; c < KH / 8; ++c) {  // 16-byte chunk c: keys 8c .. 8c+7 of this half
+          for (int c = 0; c < KH / 8; ++c) {  // 16-byte chunk c: keys half*KH + 8c .. +7
             uint32_t hi[4], lo[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
@@ -335,7 +363,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
               hi[e] = pack_bf16x2(p0, p1);
               lo[e] = pack_bf16x2(p0 - bf16lo(hi[e]), p1 - bf16hi(hi[e]));
             }
-            const uint32_t off = half * (AT_P_BYTES / 2) + swz128(row, c);
+            const int key = half * KH + 8 * c;  // in 64-key chunk key/64, 16-byte unit (key%64)/8
+            const uint32_t off = (key / 64) * (AT_BM * 128) + swz128(row, (key % 64) / 8);
             *reinterpret_cast<uint4*>(sPh + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
             *reinterpret_cast<uint4*>(sPl + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
           }
@@ -375,7 +404,8 @@ __global__ void __launch_bounds__(AT_THREADS, 1)
   }
 }
 
-// vt[(b*Hkv + g)*64 + d][j] = v of key j, group g, dim d (keys past N: zero up to ldt).
+// vt[(b*Hkv + g)*HD + d][j] = v of key j, group g, dim d (keys past N: zero up to ldt).
+template <int AT_HD>
 __global__ void v_transpose_kernel(const bf16* __restrict__ qkv, int B, int N, int Hq, int Hkv,
                                    int ldt, bf16* __restrict__ vt) {
   pdl_trigger();
@@ -423,13 +453,13 @@ bool encode(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uin
 
 }  // namespace
 
-size_t attention_tc_vt_elems(int B, int N, int Hkv) {
-  return static_cast<size_t>(B) * Hkv * AT_HD * ((N + 7) & ~7);
+size_t attention_tc_vt_elems(int B, int N, int Hkv, int hd) {
+  return static_cast<size_t>(B) * Hkv * hd * ((N + 7) & ~7);
 }
 
 bool attention_tc_supported(int dtype, int hd, const int* cu, const uint8_t* key_alive, int* status,
                             void* vt) {
-  return dtype == ZSAA_BF16 && hd == AT_HD && cu == nullptr && key_alive == nullptr &&
+  return dtype == ZSAA_BF16 && (hd == 64 || hd == 128) && cu == nullptr && key_alive == nullptr &&
          status != nullptr && vt != nullptr;
 }
 
@@ -438,25 +468,31 @@ bool attention_tc_supported(int dtype, int hd, const int* cu, const uint8_t* key
 // extra launch and 128-row tiles on short sequences cost more than they save.
 bool attention_tc_preferred(int N) { return N >= kAttentionTcMinN; }
 
-cudaError_t launch_attention_tc(const void* qkv, void* vt, int B, int N, int Hq, int Hkv, void* out,
-                                float* lse, int causal, int* status, cudaStream_t s) {
+namespace {
+
+template <int HD>
+cudaError_t run_attention_tc(const void* qkv, void* vt, int B, int N, int Hq, int Hkv, void* out,
+                             float* lse, int causal, int* status, cudaStream_t s) {
+  using C = AtCfg<HD>;
   const int ldt = (N + 7) & ~7;
-  const int ld = (Hq + 2 * Hkv) * AT_HD;
+  const int ld = (Hq + 2 * Hkv) * HD;
   {
-    dim3 grid((ldt + 31) / 32, AT_HD / 32, B * Hkv);
-    ZSAA_LAUNCH(v_transpose_kernel, grid, dim3(256), 0, s, static_cast<const bf16*>(qkv), B, N, Hq, Hkv,
+    dim3 grid((ldt + 31) / 32, HD / 32, B * Hkv);
+    ZSAA_LAUNCH(v_transpose_kernel<HD>, grid, dim3(256), 0, s, static_cast<const bf16*>(qkv), B, N, Hq, Hkv,
                 ldt, static_cast<bf16*>(vt));
   }
-  CUtensorMap tm_qk, tm_vt;
-  if (!encode(&tm_qk, qkv, static_cast<uint64_t>(ld), static_cast<uint64_t>(B) * N, ld, 64, AT_BM))
+  CUtensorMap tm_q, tm_k, tm_vt;
+  if (!encode(&tm_q, qkv, static_cast<uint64_t>(ld), static_cast<uint64_t>(B) * N, ld, 64, AT_BM))
     return cudaErrorInvalidValue;
-  if (!encode(&tm_vt, vt, static_cast<uint64_t>(ldt), static_cast<uint64_t>(B) * Hkv * AT_HD, ldt, 64, AT_HD))
+  if (!encode(&tm_k, qkv, static_cast<uint64_t>(ld), static_cast<uint64_t>(B) * N, ld, 64, C::BN))
+    return cudaErrorInvalidValue;
+  if (!encode(&tm_vt, vt, static_cast<uint64_t>(ldt), static_cast<uint64_t>(B) * Hkv * HD, ldt, 64, HD))
     return cudaErrorInvalidValue;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, [] {
-    attr_err = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    static_cast<int>(AT_SMEM));
+    attr_err = cudaFuncSetAttribute(attn_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    static_cast<int>(C::SMEM));
   });
   if (attr_err != cudaSuccess) return attr_err;
   AtArgs a;
@@ -468,12 +504,21 @@ cudaError_t launch_attention_tc(const void* qkv, void* vt, int B, int N, int Hq,
   a.Hkv = Hkv;
   a.n_qb = (N + AT_BM - 1) / AT_BM;
   a.causal = causal;
-  a.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(AT_HD));
+  a.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(HD));
   a.status = status;
   const int total = a.n_qb * Hq * B;
   const int grid = total < attn_sms() ? total : attn_sms();
-  ZSAA_LAUNCH(attn_tc_kernel, dim3(grid), dim3(AT_THREADS), AT_SMEM, s, tm_qk, tm_vt, a);
+  ZSAA_LAUNCH(attn_tc_kernel<HD>, dim3(grid), dim3(AT_THREADS), C::SMEM, s, tm_q, tm_k, tm_vt, a);
   return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_attention_tc(const void* qkv, void* vt, int B, int N, int Hq, int Hkv, int hd,
+                                void* out, float* lse, int causal, int* status, cudaStream_t s) {
+  if (hd == 64) return run_attention_tc<64>(qkv, vt, B, N, Hq, Hkv, out, lse, causal, status, s);
+  if (hd == 128) return run_attention_tc<128>(qkv, vt, B, N, Hq, Hkv, out, lse, causal, status, s);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace zsaa

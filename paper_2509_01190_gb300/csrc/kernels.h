@@ -125,16 +125,16 @@ cudaError_t launch_gemm_f32(const float* A, int lda, const float* W, const float
                             const GemmParams& p, cudaStream_t s);
 
 // ---- attention (k_attn.cu)
-// tcgen05 attention (k_attn_tc.cu) for bf16 heads of 64 dims, fixed lengths:
-// a transpose kernel writes V^T into vt (attention_tc_vt_elems bf16 elements),
-// then one CTA per (128 queries, head, sequence).  Same outputs as
-// launch_attention; bounded waits report through status.
+// tcgen05 attention (k_attn_tc.cu) for bf16 heads of 64 or 128 dims, fixed
+// lengths: a transpose kernel writes V^T into vt (attention_tc_vt_elems bf16
+// elements), then persistent CTAs walk (128 queries, head, sequence) items.
+// Same outputs as launch_attention; bounded waits report through status.
 bool attention_tc_supported(int dtype, int hd, const int* cu, const uint8_t* key_alive, int* status,
                             void* vt);
-size_t attention_tc_vt_elems(int B, int N, int Hkv);
+size_t attention_tc_vt_elems(int B, int N, int Hkv, int hd);
 constexpr int kAttentionTcMinN = 256;
 bool attention_tc_preferred(int N);
-cudaError_t launch_attention_tc(const void* qkv, void* vt, int B, int N, int Hq, int Hkv, void* out,
+cudaError_t launch_attention_tc(const void* qkv, void* vt, int B, int N, int Hq, int Hkv, int hd, void* out,
                                 float* lse, int causal, int* status, cudaStream_t s);
 // causal = 0: bidirectional (Eq. 1 with M = 0); the column-mass kernels below
 // take the same flag.

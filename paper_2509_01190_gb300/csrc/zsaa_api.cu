@@ -605,7 +605,7 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
       TRACE("attention", 4.0 * pairs * hd, Md * (m->ld_qkv + m->dq) * es + static_cast<double>(B) * Hq * N * 4.0);
       if (attention_tc_supported(dt, hd, nullptr, nullptr, m->status, m->vt) && attention_tc_preferred(N)) {
         trace_scope_.kernels = 2;  // V transpose + attention
-        ZCK(launch_attention_tc(m->qkv, m->vt, B, N, Hq, Hkv, m->attn, m->lse, causal, m->status, s));
+        ZCK(launch_attention_tc(m->qkv, m->vt, B, N, Hq, Hkv, hd, m->attn, m->lse, causal, m->status, s));
       } else {
         ZCK(launch_attention(dt, m->qkv, B, N, Hq, Hkv, hd, m->attn, m->lse, causal, s));
       }
@@ -1585,8 +1585,8 @@ zsaa_status zsaa_model_create(const zsaa_config* cfg, const zsaa_weights* w, int
   alloc(&m->attn, rows * m->dq * esz);
   alloc(&m->act, rows * F * esz);
   alloc(reinterpret_cast<void**>(&m->lse), rows * cfg->n_heads * sizeof(float));
-  if (cfg->dtype == ZSAA_BF16 && cfg->head_dim == 64)
-    alloc(&m->vt, attention_tc_vt_elems(max_B, max_L, cfg->n_kv_heads) * 2);
+  if (cfg->dtype == ZSAA_BF16 && (cfg->head_dim == 64 || cfg->head_dim == 128))
+    alloc(&m->vt, attention_tc_vt_elems(max_B, max_L, cfg->n_kv_heads, cfg->head_dim) * 2);
   alloc(reinterpret_cast<void**>(&m->colmass),
         colmass_parts_elems(max_B, max_L, cfg->n_heads, cfg->n_kv_heads) * sizeof(float));
   alloc(reinterpret_cast<void**>(&m->vnorm), rows * cfg->n_kv_heads * sizeof(float));
@@ -1773,10 +1773,10 @@ zsaa_status zsaa_op_attention_ex(const void* qkv, int B, int N, int Hq, int Hkv,
   if (dtype == ZSAA_F32 && (hd < 1 || hd > 128)) return fail(ZSAA_ERR_UNSUPPORTED, "f32 attention needs hd <= 128");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   int* status = shared_status();
-  if (dtype == ZSAA_BF16 && hd == 64 && status != nullptr) {  // the tcgen05 kernel, V^T scratch
+  if (dtype == ZSAA_BF16 && status != nullptr) {  // the tcgen05 kernel, V^T scratch
     void* vt = nullptr;
-    ZCK(cudaMallocAsync(&vt, attention_tc_vt_elems(B, N, Hkv) * 2, s));
-    cudaError_t e = launch_attention_tc(qkv, vt, B, N, Hq, Hkv, out, lse, causal ? 1 : 0, status, s);
+    ZCK(cudaMallocAsync(&vt, attention_tc_vt_elems(B, N, Hkv, hd) * 2, s));
+    cudaError_t e = launch_attention_tc(qkv, vt, B, N, Hq, Hkv, hd, out, lse, causal ? 1 : 0, status, s);
     cudaError_t e2 = cudaFreeAsync(vt, s);
     ZCK(e);
     ZCK(e2);

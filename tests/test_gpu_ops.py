@@ -267,7 +267,8 @@ def _oracle_attention(qkv, B, N, Hq, Hkv, hd, causal=True):
 
 @pytest.mark.parametrize("B,N,Hq,Hkv,hd", [(2, 1, 4, 2, 64), (2, 65, 4, 2, 64), (1, 200, 4, 1, 128),
                                            (2, 130, 8, 2, 128), (1, 64, 2, 2, 64), (2, 300, 4, 2, 64),
-                                           (1, 517, 8, 2, 64), (1, 1024, 4, 4, 64)])
+                                           (1, 517, 8, 2, 64), (1, 1024, 4, 4, 64), (2, 300, 4, 2, 128),
+                                           (1, 517, 8, 2, 128), (1, 1024, 4, 4, 128), (3, 63, 2, 1, 128)])
 def test_attention_and_colmass_bf16(z, B, N, Hq, Hkv, hd):
     qkv = _qkv(B, N, Hq, Hkv, hd, 20 + N, torch.bfloat16)
     out = torch.empty(B * N, Hq * hd, device="cuda", dtype=torch.bfloat16)
