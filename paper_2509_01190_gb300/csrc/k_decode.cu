@@ -116,6 +116,21 @@ __global__ void __launch_bounds__(decode_warps<HD, PER>() * 32)
   }
   for (int j0 = warp * 32; j0 < n_keys; j0 += W * 32) {
     const int j = j0 + lane;
+    const int nb = min(32, n_keys - j0);
+    // this lane's head-dim slice of the block's 32 value rows, requested with
+    // the key row below so that both memory latencies overlap
+    uint32_t vw[32][DPL / 2];
+#pragma unroll
+    for (int jj = 0; jj < 32; ++jj) {
+      const bf16* vr = Vc + static_cast<size_t>(j0 + (jj < nb ? jj : 0)) * HD + lane * DPL;
+      if constexpr (DPL == 2) {
+        vw[jj][0] = *reinterpret_cast<const uint32_t*>(vr);
+      } else {
+        const uint2 w = *reinterpret_cast<const uint2*>(vr);
+        vw[jj][0] = w.x;
+        vw[jj][1] = w.y;
+      }
+    }
     float sc[PER];
     if (j < n_keys) {
       float dot[PER];
@@ -157,27 +172,21 @@ __global__ void __launch_bounds__(decode_warps<HD, PER>() * 32)
       for (int e = 0; e < DPL; ++e) acc[h][e] *= corr;
       m[h] = mn;
     }
-    const int nb = min(32, n_keys - j0);
-#pragma unroll 4
-    for (int jj = 0; jj < nb; ++jj) {
-      const bf16* vr = Vc + static_cast<size_t>(j0 + jj) * HD + lane * DPL;
-      float vv[DPL];
-      if constexpr (DPL == 2) {
-        const uint32_t w = *reinterpret_cast<const uint32_t*>(vr);
-        vv[0] = __uint_as_float(w << 16);
-        vv[1] = __uint_as_float(w & 0xffff0000u);
-      } else {
-        const uint2 w = *reinterpret_cast<const uint2*>(vr);
-        vv[0] = __uint_as_float(w.x << 16);
-        vv[1] = __uint_as_float(w.x & 0xffff0000u);
-        vv[2] = __uint_as_float(w.y << 16);
-        vv[3] = __uint_as_float(w.y & 0xffff0000u);
-      }
 #pragma unroll
-      for (int h = 0; h < PER; ++h) {
-        const float pk = __shfl_sync(0xffffffffu, pj[h], jj);
+    for (int jj = 0; jj < 32; ++jj) {
+      if (jj < nb) {  // warp-uniform
+        float vv[DPL];
 #pragma unroll
-        for (int e = 0; e < DPL; ++e) acc[h][e] = fmaf(pk, vv[e], acc[h][e]);
+        for (int e2 = 0; e2 < DPL / 2; ++e2) {
+          vv[2 * e2] = __uint_as_float(vw[jj][e2] << 16);
+          vv[2 * e2 + 1] = __uint_as_float(vw[jj][e2] & 0xffff0000u);
+        }
+#pragma unroll
+        for (int h = 0; h < PER; ++h) {
+          const float pk = __shfl_sync(0xffffffffu, pj[h], jj);
+#pragma unroll
+          for (int e = 0; e < DPL; ++e) acc[h][e] = fmaf(pk, vv[e], acc[h][e]);
+        }
       }
     }
   }
