@@ -350,6 +350,9 @@ struct zsaa_model {
   // joined before the gather), created on first use
   cudaStream_t side = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  // zsaa_forward_host with a pinned logits buffer: the LM head runs in column
+  // slabs and each slab is copied to this host buffer while the next computes
+  float* host_logits = nullptr;
 };
 
 // Pruned KV cache for generation (zsaa_cache_create).
@@ -376,6 +379,16 @@ struct zsaa_cache {
 };
 
 namespace {
+
+// Column slabs of the LM head when its logits stream to a pinned host buffer
+// (zsaa_forward_host): slab i covers columns [slab_col(V, i), slab_col(V, i+1)),
+// boundaries on 128-column multiples.
+constexpr int kHeadSlabs = 4;
+int slab_col(int V, int i, int n) {
+  if (i >= n) return V;
+  const long long c = (static_cast<long long>(V) * i / n + 127) / 128 * 128;
+  return static_cast<int>(c < V ? c : V);
+}
 
 // Make the model's side stream wait for the work enqueued on s so far
 // (creating the stream and its events on first use).
@@ -781,18 +794,38 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
       TRACE("rmsnorm", 0.0, 2.0 * static_cast<double>(M) * d * es);
       ZCK(launch_rmsnorm(dt, m->h[cur], m->final_norm, M, d, c.rms_eps, m->x, s));
     }
-    GemmParams q{};
-    q.M = M;
-    q.N = c.vocab;
-    q.K = d;
-    q.out = logits;
-    q.ldo = c.vocab;
-    TcWeights W{m->head, nullptr, nullptr, c.vocab, c.vocab};
+    // With a pinned host destination (and not tracing) the head runs as
+    // kHeadSlabs column slabs; the side stream copies each slab to the host
+    // while the next one computes, and s joins the copies.
+    const bool slabs = m->host_logits != nullptr && !m->tracing && dt == ZSAA_BF16;
+    const int n_slabs = slabs ? kHeadSlabs : 1;
     const double V = c.vocab, Mh = M;
-    TRACE("gemm_lm_head", 2.0 * Mh * V * d, (Mh * d + V * d) * es + Mh * V * 4.0);
-    trace_scope_.kernels = 0;
-    st = linear(m, m->x, d, W, dt == ZSAA_BF16 ? kEpiStoreF32 : kEpiStore, q, s, &trace_scope_.kernels);
-    if (st != ZSAA_OK) return st;
+    for (int sl = 0; sl < n_slabs; ++sl) {
+      const int c0 = slab_col(c.vocab, sl, n_slabs), c1 = slab_col(c.vocab, sl + 1, n_slabs);
+      if (c1 <= c0) continue;  // a small vocabulary leaves some slabs empty
+      GemmParams q{};
+      q.M = M;
+      q.N = c1 - c0;
+      q.K = d;
+      q.out = logits + c0;
+      q.ldo = c.vocab;
+      const void* w0 = static_cast<const uint8_t*>(m->head) + static_cast<size_t>(c0) * d * m->esz;
+      TcWeights W{w0, nullptr, nullptr, c1 - c0, c1 - c0};
+      TRACE("gemm_lm_head", 2.0 * Mh * (c1 - c0) * d, (Mh * d + (c1 - c0) * static_cast<double>(d)) * es + Mh * (c1 - c0) * 4.0);
+      trace_scope_.kernels = 0;
+      st = linear(m, m->x, d, W, dt == ZSAA_BF16 ? kEpiStoreF32 : kEpiStore, q, s, &trace_scope_.kernels);
+      if (st != ZSAA_OK) return st;
+      if (slabs) {
+        ZCK(fork_side(m, s));
+        ZCK(cudaMemcpy2DAsync(m->host_logits + c0, sizeof(float) * c.vocab, logits + c0,
+                              sizeof(float) * c.vocab, sizeof(float) * (c1 - c0), M,
+                              cudaMemcpyDeviceToHost, m->side));
+      }
+    }
+    if (slabs) {
+      ZCK(cudaEventRecord(m->ev_join, m->side));
+      ZCK(cudaStreamWaitEvent(s, m->ev_join, 0));
+    }
   }
   if (kept_pos)
     ZCK(cudaMemcpyAsync(kept_pos, m->pos[cur], sizeof(int32_t) * M, cudaMemcpyDeviceToDevice, s));
@@ -1241,8 +1274,9 @@ zsaa_status forward_cached(zsaa_model* m, const int32_t* tok, int B, int L, doub
   if (!m->use_graphs || m->tracing)
     return run_forward(m, tok, B, L, accel, logits, kept_pos, nullptr, s, kc);
   char key[200];
-  snprintf(key, sizeof(key), "%p/%d/%d/%.17g/%p/%p/%p", static_cast<const void*>(tok), B, L, accel,
-           static_cast<void*>(logits), static_cast<void*>(kept_pos), static_cast<void*>(kc));
+  snprintf(key, sizeof(key), "%p/%d/%d/%.17g/%p/%p/%p/%p", static_cast<const void*>(tok), B, L, accel,
+           static_cast<void*>(logits), static_cast<void*>(kept_pos), static_cast<void*>(kc),
+           static_cast<void*>(m->host_logits));
   auto it = m->graphs.begin();
   for (; it != m->graphs.end(); ++it)
     if (it->key == key) break;
@@ -1690,10 +1724,23 @@ zsaa_status zsaa_forward_host(zsaa_model* m, const int32_t* token_ids, int B, in
     ZCK(cudaMalloc(&m->stage_logits, n_logits * sizeof(float)));
     m->stage_logits_cap = n_logits;
   }
+  // A pinned (page-locked) logits buffer lets the LM head's column slabs be
+  // copied while later slabs compute; other buffers get one copy at the end.
+  bool stream_logits = false;
+  if (m->cfg.n_classes == 0 && m->cfg.dtype == ZSAA_BF16) {
+    cudaPointerAttributes pa{};
+    if (cudaPointerGetAttributes(&pa, logits_out) == cudaSuccess)
+      stream_logits = pa.type == cudaMemoryTypeHost;
+    else
+      cudaGetLastError();
+  }
   ZCK(cudaMemcpyAsync(m->stage_tok, token_ids, sizeof(int32_t) * B * L, cudaMemcpyHostToDevice, s));
+  m->host_logits = stream_logits ? logits_out : nullptr;
   st = forward_cached(m, m->stage_tok, B, L, accel, m->stage_logits, m->stage_pos, s);
+  m->host_logits = nullptr;
   if (st != ZSAA_OK) return st;
-  ZCK(cudaMemcpyAsync(logits_out, m->stage_logits, n_logits * sizeof(float), cudaMemcpyDeviceToHost, s));
+  if (!stream_logits)
+    ZCK(cudaMemcpyAsync(logits_out, m->stage_logits, n_logits * sizeof(float), cudaMemcpyDeviceToHost, s));
   if (kept_pos_out)
     ZCK(cudaMemcpyAsync(kept_pos_out, m->stage_pos, sizeof(int32_t) * B * n_final,
                         cudaMemcpyDeviceToHost, s));

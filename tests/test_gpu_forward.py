@@ -301,3 +301,23 @@ def test_full_size_8b_layerwise_and_head(z):
     shape = wl["shape"]
     model, _, tokens, sched, ores = layerwise_case(z, shape, wl["B"], wl["L"], 11.0, [1, 2, 16, 32])
     chained_check(z, model, shape, tokens, sched, ores, 11.0)
+
+
+@pytest.mark.parametrize("vocab", [None, 256])
+def test_forward_host_pinned_streams_head(z, vocab):
+    # A pinned logits buffer: the LM head runs as column slabs copied to the
+    # host while later slabs compute.  Eager, captured and replayed calls (the
+    # forward is graph-cached) must all equal the device forward bit for bit;
+    # with 256 columns, some of the four slabs are empty.
+    shape = SMALL_BF16 if vocab is None else dataclasses.replace(SMALL_BF16, name="small-v256", vocab=vocab)
+    res = run_case(z, shape, 2, 96, 2.0, seqs=[0])
+    model, sched = res["model"], res["sched"]
+    B, L = 2, 96
+    tok = torch.from_numpy(np.ascontiguousarray(res["tokens"])).pin_memory()
+    logits_h = torch.zeros(B, sched[-1], shape.vocab, dtype=torch.float32).pin_memory()
+    kept_h = torch.zeros(B, sched[-1], dtype=torch.int32).pin_memory()
+    for _ in range(3):
+        logits_h.zero_()
+        z.zsaa_forward_host(model, tok, B, L, 2.0, logits_h, kept_h)
+        np.testing.assert_array_equal(logits_h.numpy(), res["nat_logits"])
+        np.testing.assert_array_equal(kept_h.numpy(), res["kept_nat"])
