@@ -177,7 +177,10 @@ zsaa_status zsaa_forward_ex(zsaa_model* m, const int32_t* token_ids, int B, int 
 /* zsaa_forward on HOST buffers: copies token_ids (host [B, L]) in, runs, copies
  * logits (host float32, same shape as zsaa_forward) and kept positions (host or
  * NULL) out, and returns after the stream has finished.  Device staging is
- * owned by the model (allocated on first use). */
+ * owned by the model (allocated on first use).  When logits_out is page-locked
+ * host memory (cudaHostAlloc / cudaHostRegister) and the model is a bf16 LM,
+ * the LM head runs in column slabs and each slab is copied while the next one
+ * computes; the values are the same either way. */
 zsaa_status zsaa_forward_host(zsaa_model* m, const int32_t* token_ids, int B, int L,
                               double accel, float* logits_out, int32_t* kept_pos_out,
                               zsaa_stream stream);
