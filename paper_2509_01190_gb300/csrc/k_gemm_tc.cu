@@ -574,6 +574,212 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// ---------------------------------------------------------------------------
+// CTA-pair kernel for many rows: tcgen05.mma.cta_group::2.
+// A cluster of two CTAs (the two SMs of a TPC) computes 256 x 256 tiles.  CTA
+// r of the pair stages A rows [m0 + 128 r, +128) and 128 of the tile's 256
+// weight rows (rows n0 + 128 r; SwiGLU: CTA 0 the 128 gate rows of W, CTA 1 the
+// same 128 up rows of W2) for each 64-deep k-block; the leader (rank 0) issues
+// M=256, N=256 MMAs that read both CTAs' shared memory, and each CTA's TMEM
+// receives its own 128 rows x 256 columns of the tile.  Per SM that is 32 KB of
+// operands per 128 x 256 x 64 step instead of the one-CTA kernel's 48 KB, the
+// stream that limits the one-CTA kernel at large M.
+//   warp 0 (both CTAs)  TMA producer: this CTA's halves into a P_STAGES ring;
+//                       the copies of both CTAs complete on the leader's
+//                       "full" barrier, which the leader arms for both;
+//   warp 1 (leader)     MMA issuer; tcgen05.commit multicasts each stage's
+//                       release to both CTAs' "empty" barriers and each finished
+//                       accumulator to both CTAs' "acc_full" barriers;
+//   warps 2..5 (both)   epilogue of this CTA's 128 rows (the one-CTA kernel's),
+//                       then release the accumulator on the leader's barrier.
+// Whole tiles only, round robin over the pairs; tile t -> (row pair t % mp_tiles,
+// column tile t / mp_tiles), so concurrent pairs share weight tiles in L2.
+// Every wait is bounded; a CTA that gives up waits briefly for its own copies
+// in flight and still reaches the closing cluster barrier.
+constexpr int P_BN = 256;
+constexpr int P_STAGES = 6;
+constexpr int P_A_BYTES = BM * BK * 2;          // this CTA's 128 rows of A
+constexpr int P_B_BYTES = (P_BN / 2) * BK * 2;  // this CTA's 128 weight rows
+constexpr int P_STAGE_BYTES = P_A_BYTES + P_B_BYTES;
+constexpr size_t P_SMEM = static_cast<size_t>(P_STAGES) * P_STAGE_BYTES + 1024 + 256;
+constexpr uint32_t P_TMEM_COLS = 2 * P_BN;  // two accumulators
+constexpr double kPairTileCost = 0.9;
+
+struct PairSched {
+  int mp_tiles, n_tiles, num_kb, total;
+};
+
+template <int EPI>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_pair_kernel(const __grid_constant__ TcMaps maps, const int n1, const int n2,
+                     const GemmParams p, const PairSched ps) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + P_STAGES * P_A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + P_STAGES * P_STAGE_BYTES);
+  uint64_t* empty = full + P_STAGES;
+  uint64_t* acc_full = empty + P_STAGES;  // [2]
+  uint64_t* acc_empty = acc_full + 2;     // [2], used in the leader
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int rank = static_cast<int>(cluster_rank());
+  const int pair = static_cast<int>(blockIdx.x >> 1), npairs = static_cast<int>(gridDim.x >> 1);
+  pdl_trigger();
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < P_STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 8);  // four epilogue warps in each CTA
+    }
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    prefetch_tmap(&maps.a);
+    prefetch_tmap(&maps.b0);
+    if (EPI == kEpiSwiGLU || n1 < p.N) prefetch_tmap(&maps.b1);
+    if (n2 < p.N) prefetch_tmap(&maps.b2);
+  }
+  if (warp == 1) tmem_alloc_pair(tmem_slot, P_TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // both CTAs' barriers initialised before any copy or arrival crosses
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      const uint32_t full_leader = map_rank(smem_u32(full), 0);
+      // this CTA's 128 weight rows of column tile nt: (map, first row)
+      auto w_rows = [&](int nt, const CUtensorMap*& mb, int& wy) {
+        const int n0 = nt * P_BN;
+        if (EPI == kEpiSwiGLU) {
+          mb = rank == 0 ? &maps.b0 : &maps.b1;
+          wy = n0 / 2;
+        } else {
+          mb = n0 >= n2 ? &maps.b2 : (n0 >= n1 ? &maps.b1 : &maps.b0);
+          wy = (n0 >= n2 ? n0 - n2 : (n0 >= n1 ? n0 - n1 : n0)) + rank * (P_BN / 2);
+        }
+      };
+      uint32_t it = 0, issued = 0;
+      bool ok = true;
+      // weights are never written by another kernel: request the first tile's
+      // first stages before waiting for the previous kernel
+      int npre = 0;
+      if (pair < ps.total) {
+        const CUtensorMap* mb;
+        int wy;
+        w_rows(pair / ps.mp_tiles, mb, wy);
+        npre = min(P_STAGES, ps.num_kb);
+        for (int j = 0; j < npre; ++j) {
+          if (rank == 0) mbar_arrive_expect_tx(&full[j], 2 * P_STAGE_BYTES);
+          tma_load_2d_pair(sB + j * P_B_BYTES, mb, j * BK, wy, full_leader + 8u * j);
+        }
+      }
+      pdl_wait();
+      for (int t = pair; ok && t < ps.total; t += npairs) {
+        const int mp = t % ps.mp_tiles, nt = t / ps.mp_tiles;
+        const int m0 = mp * (2 * BM) + rank * BM;
+        const CUtensorMap* mb;
+        int wy;
+        w_rows(nt, mb, wy);
+        for (int kb = 0; kb < ps.num_kb; ++kb, ++it) {
+          const int s = it % P_STAGES;
+          const uint32_t ph = (it / P_STAGES) & 1;
+          if (static_cast<int>(it) >= npre) {
+            if (!mbar_wait_ab(&empty[s], ph ^ 1, p.status, abort_flag)) {
+              ok = false;
+              break;
+            }
+            if (rank == 0) mbar_arrive_expect_tx(&full[s], 2 * P_STAGE_BYTES);
+            tma_load_2d_pair(sB + s * P_B_BYTES, mb, kb * BK, wy, full_leader + 8u * s);
+          }
+          tma_load_2d_pair(sA + s * P_A_BYTES, &maps.a, kb * BK, m0, full_leader + 8u * s);
+          issued = it + 1;
+        }
+      }
+      // The copies land on the leader's barrier, which this thread cannot always
+      // watch: after a stop, give copies still in flight time to land (a TMA
+      // copy takes microseconds) before the CTA can exit.
+      if ((!ok || *abort_flag) && issued > 0) {
+        const unsigned long long t0 = globaltimer_ns();
+        while (globaltimer_ns() - t0 < 200000ull) __nanosleep(1000);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(2 * BM, P_BN);
+      uint32_t it = 0;
+      bool ok = true;
+      int i = 0;
+      for (int t = pair; ok && t < ps.total; t += npairs) {
+        const int ab = i & 1;
+        const uint32_t use = static_cast<uint32_t>(i >> 1);
+        ++i;
+        if (!mbar_wait_cluster_ab(&acc_empty[ab], (use & 1) ^ 1, p.status, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem + static_cast<uint32_t>(ab * P_BN);
+        for (int kb = 0; kb < ps.num_kb; ++kb, ++it) {
+          const int s = it % P_STAGES;
+          const uint32_t ph = (it / P_STAGES) & 1;
+          if (!mbar_wait_ab(&full[s], ph, p.status, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_base = smem_u32(sA + s * P_A_BYTES);
+          const uint32_t b_base = smem_u32(sB + s * P_B_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            tc_mma_bf16_pair(d_tmem, sdesc_sw128(a_base + k * 32), sdesc_sw128(b_base + k * 32), idesc,
+                             (kb > 0 || k > 0) ? 1u : 0u);
+          tc_commit_pair(&empty[s]);
+        }
+        if (ok) tc_commit_pair(&acc_full[ab]);
+      }
+    }
+    __syncwarp();
+  } else {
+    // Epilogue: warp w reads TMEM lanes 32*(w%4) .. +32 -- this CTA's tile rows.
+    pdl_wait();
+    const int quad = warp & 3;
+    const int rit = quad * 32 + lane;
+    const uint32_t acc_empty_leader = map_rank(smem_u32(acc_empty), 0);
+    int i = 0;
+    for (int t = pair; t < ps.total; t += npairs) {
+      const int mp = t % ps.mp_tiles, nt = t / ps.mp_tiles;
+      const int row = mp * (2 * BM) + rank * BM + rit;
+      const int ab = i & 1;
+      const uint32_t use = static_cast<uint32_t>(i >> 1);
+      ++i;
+      const bool ok = __all_sync(0xffffffffu, mbar_wait_ab(&acc_full[ab], use & 1, p.status, abort_flag));
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t tbase = tmem + static_cast<uint32_t>(ab * P_BN) + (static_cast<uint32_t>(quad * 32) << 16);
+      tile_epilogue<P_BN, EPI>(tbase, row, row < p.M, nt * P_BN, p, nullptr, 1, 0, rit);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(acc_empty_leader + 8u * ab);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // no copy, commit or arrival of this tile loop still targets the other CTA
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, P_TMEM_COLS);
+  }
+}
+
 bool encode_2d(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t rows, uint64_t row_elems,
                uint32_t box_rows) {
   EncodeTiledFn enc = get_encode_tiled();
@@ -626,6 +832,91 @@ cudaError_t dispatch_epi(int epi, const TcMaps& maps, int n1, int n2, const Gemm
     case kEpiSwiGLU: return run_tc<BN, kEpiSwiGLU>(maps, n1, n2, p, ts, grid, s);
     case kEpiStoreF32: return run_tc<BN, kEpiStoreF32>(maps, n1, n2, p, ts, grid, s);
     case kEpiRope: return run_tc<BN, kEpiRope>(maps, n1, n2, p, ts, grid, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+template <int EPI>
+cudaError_t pair_attr() {
+  static std::once_flag once;
+  static cudaError_t err = cudaSuccess;
+  std::call_once(once, [] {
+    err = cudaFuncSetAttribute(gemm_pair_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(P_SMEM));
+  });
+  return err;
+}
+
+cudaLaunchConfig_t pair_cfg(int pairs, cudaStream_t s, cudaLaunchAttribute (&attr)[2]) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * pairs);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = P_SMEM;
+  cfg.stream = s;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cfg;
+}
+
+// CTA pairs of the pair kernel resident at once (0 if the query fails), per device.
+template <int EPI>
+int pair_slots() {
+  static std::mutex mu;
+  static int cached[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  std::lock_guard<std::mutex> lk(mu);
+  if (cached[dev] != 0) return cached[dev] > 0 ? cached[dev] : 0;
+  int n = 0;
+  if (pair_attr<EPI>() == cudaSuccess) {
+    cudaLaunchAttribute attr[2];
+    cudaLaunchConfig_t cfg = pair_cfg(1, nullptr, attr);
+    cfg.numAttrs = 1;  // the cluster dimension only
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_pair_kernel<EPI>, &cfg) != cudaSuccess) n = 0;
+  }
+  cudaGetLastError();
+  cached[dev] = n > 0 ? n : -1;
+  return n > 0 ? n : 0;
+}
+
+int pair_slots_for(int epi) {
+  switch (epi) {
+    case kEpiStore: return pair_slots<kEpiStore>();
+    case kEpiResid: return pair_slots<kEpiResid>();
+    case kEpiSwiGLU: return pair_slots<kEpiSwiGLU>();
+    case kEpiStoreF32: return pair_slots<kEpiStoreF32>();
+    case kEpiRope: return pair_slots<kEpiRope>();
+    default: return 0;
+  }
+}
+
+template <int EPI>
+cudaError_t run_pair(const TcMaps& maps, int n1, int n2, const GemmParams& p, const PairSched& ps,
+                     int pairs, cudaStream_t s) {
+  cudaError_t e = pair_attr<EPI>();
+  if (e != cudaSuccess) return e;
+  cudaLaunchAttribute attr[2];
+  cudaLaunchConfig_t cfg = pair_cfg(pairs, s, attr);
+  e = cudaLaunchKernelEx(&cfg, gemm_pair_kernel<EPI>, maps, n1, n2, p, ps);
+  if (e != cudaSuccess) return e;
+  if (p.launches) *p.launches += 1;
+  return cudaSuccess;
+}
+
+cudaError_t dispatch_pair(int epi, const TcMaps& maps, int n1, int n2, const GemmParams& p,
+                          const PairSched& ps, int pairs, cudaStream_t s) {
+  switch (epi) {
+    case kEpiStore: return run_pair<kEpiStore>(maps, n1, n2, p, ps, pairs, s);
+    case kEpiResid: return run_pair<kEpiResid>(maps, n1, n2, p, ps, pairs, s);
+    case kEpiSwiGLU: return run_pair<kEpiSwiGLU>(maps, n1, n2, p, ps, pairs, s);
+    case kEpiStoreF32: return run_pair<kEpiStoreF32>(maps, n1, n2, p, ps, pairs, s);
+    case kEpiRope: return run_pair<kEpiRope>(maps, n1, n2, p, ps, pairs, s);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -695,9 +986,32 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
       grid = static_cast<int>(g < 1 ? 1 : (g < sms ? g : sms));
     }
   }
+  // CTA pairs (256 x 256 tiles on the 2-SM MMA) for whole-tile problems of
+  // several waves: per MMA step each SM streams 32 KB of operands instead of
+  // 48 KB, the stream that limits the one-CTA kernel at many rows.  Measured on
+  // GB300 (Llama-3.2-1B and -8B projections, 288..8192 rows, graph-timed): a
+  // pair wave takes 0.84..0.96 of a one-CTA wave, but pairing 128-row tiles
+  // can leave half a pair empty and add a wave, and in a single short-K wave
+  // the pair's extra synchronisation costs 1..4%, so pairs are taken when they
+  // save waves at kPairTileCost each, and in one wave only for deep K.
+  PairSched ps{};
+  int pairs = 0;
+  if (BN == P_BN && ts.sk_iters == 0) {
+    const int slots = pair_slots_for(epi);
+    ps.mp_tiles = (m_tiles + 1) / 2;
+    ps.n_tiles = ts.n_tiles;
+    ps.num_kb = ts.num_kb;
+    ps.total = ps.mp_tiles * ps.n_tiles;
+    if (slots > 0) {
+      const int waves_pair = (ps.total + slots - 1) / slots;
+      const int waves_one = (ts.total + sms - 1) / sms;
+      if (waves_pair * kPairTileCost < waves_one && (waves_one >= 2 || ps.num_kb >= 64))
+        pairs = ps.total < slots ? ps.total : slots;
+    }
+  }
   TcMaps maps;
   memset(&maps, 0, sizeof(maps));
-  const uint32_t brows = epi == kEpiSwiGLU ? BN / 2 : BN;
+  const uint32_t brows = (pairs > 0 || epi == kEpiSwiGLU) ? BN / 2 : BN;
   if (!encode_2d(&maps.a, A, static_cast<uint64_t>(p.K), static_cast<uint64_t>(p.M),
                  static_cast<uint64_t>(lda), BM))
     return cudaErrorInvalidValue;
@@ -717,6 +1031,7 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
       if (!encode_2d(&maps.b2, W.w2, p.K, p.N - n2, p.K, brows)) return cudaErrorInvalidValue;
     }
   }
+  if (pairs > 0) return dispatch_pair(epi, maps, n1, n2, p, ps, pairs, s);
   switch (BN) {
     case 256: return dispatch_epi<256>(epi, maps, n1, n2, p, ts, grid, s);
     case 128: return dispatch_epi<128>(epi, maps, n1, n2, p, ts, grid, s);

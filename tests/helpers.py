@@ -52,3 +52,66 @@ def accum_bound(A, W):
 def logits_report(got, ref):
     d = np.abs(np.asarray(got, np.float64) - np.asarray(ref, np.float64))
     return float(d.max()), float(d.mean())
+
+
+def rand_bf16(shape, seed, scale=1.0):
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+    return (torch.randn(*shape, generator=g, device="cuda") * scale).to(torch.bfloat16)
+
+
+def np64(t):
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+def linear_case(z, epi, M, N, K, seed, hd=64, rope_cols=0):
+    """One zsaa_op_linear call on seeded bf16 operands; returns (output, float64
+    reference of the same operands and epilogue, per-element tolerance)."""
+    A = rand_bf16((M, K), seed)
+    W = rand_bf16((N, K), seed + 1, 0.05)
+    An, Wn = np64(A), np64(W)
+    tol = accum_bound(An, Wn)
+    if epi == "swiglu":
+        W2 = rand_bf16((N, K), seed + 2, 0.05)
+        out = torch.empty(M, N, device="cuda", dtype=torch.bfloat16)
+        z.zsaa_op_linear(A, W, W2, None, out, M, N, K, z.ZSAA_BF16, z.EPI_SWIGLU)
+        g, u = An @ Wn.T, An @ np64(W2).T
+        ref = O.bf16_round(O.silu(g) * u)
+        tol = 1.1 * np.abs(u) * tol + np.abs(O.silu(g)) * accum_bound(An, np64(W2))
+    elif epi == "rope":
+        pos = torch.randint(0, 4096, (M,), generator=torch.Generator().manual_seed(seed)).to(torch.int32).cuda()
+        out = torch.empty(M, N, device="cuda", dtype=torch.bfloat16)
+        z.zsaa_op_linear(A, W, None, None, out, M, N, K, z.ZSAA_BF16, z.EPI_ROPE, pos=pos,
+                         rope_cols=rope_cols, rope_hd=hd, rope_theta=500000.0)
+        acc = An @ Wn.T
+        cos, sin = O.rope_angles(pos.cpu().numpy(), hd, 500000.0)
+        qk = O.apply_rope(acc[:, :rope_cols].reshape(M, -1, hd), cos, sin).reshape(M, rope_cols)
+        ref = O.bf16_round(np.concatenate([qk, acc[:, rope_cols:]], axis=1))
+        tol = 2 * tol.max(axis=1, keepdims=True) + 1e-6 * np.abs(acc)
+    elif epi == "resid":
+        H = rand_bf16((M, N), seed + 3)
+        h0 = np64(H)
+        z.zsaa_op_linear(A, W, None, H, H, M, N, K, z.ZSAA_BF16, z.EPI_RESID)
+        out, ref = H, O.bf16_round(h0 + An @ Wn.T)
+    elif epi == "store_f32":
+        out = torch.empty(M, N, device="cuda", dtype=torch.float32)
+        z.zsaa_op_linear(A, W, None, None, out, M, N, K, z.ZSAA_BF16, z.EPI_STORE_F32)
+        ref = An @ Wn.T
+    else:
+        out = torch.empty(M, N, device="cuda", dtype=torch.bfloat16)
+        z.zsaa_op_linear(A, W, None, None, out, M, N, K, z.ZSAA_BF16, z.EPI_STORE)
+        ref = O.bf16_round(An @ Wn.T)
+    torch.cuda.synchronize()
+    z.zsaa_device_status()
+    return out, ref, tol
+
+
+def check_linear(out, ref, tol, epi, what):
+    """float32 outputs within the accumulation bound; bf16 within 2 ulps plus the
+    bound, 99.5% within 1 ulp."""
+    got = np64(out)
+    if epi == "store_f32":
+        assert np.all(np.abs(got - ref) <= tol + 1e-6 * np.abs(ref)), what
+    else:
+        assert np.all(bf16_ulp_close(got, ref, 2, tol)), what
+        assert np.mean(bf16_ulp_close(got, ref, 1)) > 0.995, what

@@ -1,0 +1,78 @@
+"""Parity of the CTA-pair tensor-core GEMM (many rows: 256 x 256 tiles on the
+2-SM tcgen05 MMA, each CTA of a cluster pair staging half of the A rows and
+half of the weight rows) against a float64 matmul of the same bf16 operands,
+for every epilogue.  The shapes are ones the routing sends to the pair kernel
+on a 152-SM GB300 (two or more waves of whole tiles, pairs saving a wave or
+more; the launch list of the forward shows the kernel): odd numbers of 128-row
+tiles, so the last pair's second CTA has no rows; ragged columns, so the last
+tile's second weight half lies wholly past N; and the large-row projections
+of the Llama-3.2-1B forward."""
+
+import pytest
+import torch
+
+from tests.helpers import check_linear, linear_case, need_gpu, rand_bf16
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def z(zlib):
+    need_gpu()
+    return zlib
+
+
+# N = 2064: eight 256-column tiles and 16 columns; 2056 rows: 17 tiles of 128
+# (the last pair half empty, its first half 8 rows), 2300: 18 (ragged).
+@pytest.mark.parametrize("M", [2056, 2300])
+@pytest.mark.parametrize("epi", ["store", "store_f32", "resid"])
+def test_pair_plain_epilogues(z, epi, M):
+    out, ref, tol = linear_case(z, epi, M, 2064, 512, 600 + M)
+    check_linear(out, ref, tol, epi, f"{epi} M={M}")
+
+
+@pytest.mark.parametrize("M", [2056, 2300])
+def test_pair_swiglu(z, M):
+    # 1088 outputs: eight tiles of 128 gate + 128 up rows, the ninth 64 + 64
+    out, ref, tol = linear_case(z, "swiglu", M, 1088, 512, 700 + M)
+    check_linear(out, ref, tol, "swiglu", f"M={M}")
+
+
+@pytest.mark.parametrize("hd,Hq,Hkv", [(64, 32, 8), (128, 16, 4), (64, 30, 9)])
+def test_pair_rope(z, hd, Hq, Hkv):
+    # 3072 columns (12 tiles); each CTA's 128 tile columns are whole heads;
+    # (64, 30, 9): 2496 rotated columns, so one CTA half holds a rotated key
+    # head and a value head
+    M = 2300
+    N = (Hq + 2 * Hkv) * hd
+    out, ref, tol = linear_case(z, "rope", M, N, 512, 800 + hd + Hq, hd=hd, rope_cols=(Hq + Hkv) * hd)
+    check_linear(out, ref, tol, "rope", f"hd={hd} Hq={Hq}")
+
+
+# Layers of the pruned 1B forward on the pair kernel: QKV with RoPE, O and
+# down with the residual, gate/up SwiGLU, at kept-row counts of accel 1 and 4
+# (288 rows: three 128-row tiles, two pairs).
+LARGE_1B = [("qkv", 3296, 3072, 2048), ("o", 4096, 2048, 2048), ("gate_up", 288, 8192, 2048),
+            ("gate_up", 3296, 8192, 2048), ("down", 4096, 2048, 8192)]
+
+
+@pytest.mark.parametrize("name,M,N,K", LARGE_1B)
+def test_pair_large_1b_shapes(z, name, M, N, K):
+    epi = {"qkv": "rope", "o": "resid", "gate_up": "swiglu", "down": "resid"}[name]
+    out, ref, tol = linear_case(z, epi, M, N, K, 900 + M, hd=64, rope_cols=2560)
+    check_linear(out, ref, tol, epi, f"{name} M={M}")
+
+
+def test_pair_deterministic(z):
+    M, N, K = 2048, 2048, 2048
+    A = rand_bf16((M, K), 17)
+    W = rand_bf16((N, K), 18, 0.05)
+    outs = []
+    for _ in range(3):
+        out = torch.empty(M, N, device="cuda", dtype=torch.float32)
+        z.zsaa_op_linear(A, W, None, None, out, M, N, K, z.ZSAA_BF16, z.EPI_STORE_F32)
+        outs.append(out)
+    torch.cuda.synchronize()
+    z.zsaa_device_status()
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
+
