@@ -1,7 +1,8 @@
 // bf16 GEMM on the sm_103a tensor cores: out = epi(A[M,K] W[N,K]^T), fp32
 // accumulation in tensor memory.
 //
-// Persistent stream-K kernel: one CTA per SM.  Tiles are 128 x BN (tiles
+// Persistent stream-K kernels: one CTA per SM, or (gemm_pair_kernel, for
+// many rows) one CTA pair per TPC on the 2-SM MMA.  Tiles are 128 x BN (tiles
 // sharing a weight tile are adjacent, so weights stream from HBM once and are
 // re-read from L2).  All but the last one-to-two waves of tiles are handed out
 // whole, round robin; the k-iterations of the remaining tiles are split evenly
@@ -52,13 +53,14 @@ struct TcMaps {
   CUtensorMap a, b0, b1, b2;
 };
 
-// Work split: tiles [0, dp_tiles) go whole to CTA t % grid; the k-iterations
+// Work split: tiles [0, dp_tiles) go whole to unit t % units; the k-iterations
 // of tiles [dp_tiles, total) (sk_iters of them, num_kb per tile) are cut into
-// grid equal contiguous ranges.  Tile t -> (m tile t % m_tiles, n tile t / m_tiles).
+// `units` equal contiguous ranges.  Tile t -> (m tile t % m_tiles, n tile
+// t / m_tiles); the pair kernel's m tiles are 256 rows.
 struct TileSched {
   int m_tiles, n_tiles, num_kb, total, dp_tiles;
   long long sk_iters;
-  float* ws;   // fp32 partial tiles, one BM x BN slot per CTA
+  float* ws;   // fp32 partial tiles, one BM x BN slot per CTA (slot = blockIdx.x)
   int* flags;  // per CTA and epilogue warp: 1 while its partial is ready (reset by the reader)
 };
 
@@ -71,14 +73,17 @@ struct Item {
   int tile, kb0, kb1, kind, c_hi;
 };
 
+// Work of unit `unit` of `units` (a CTA of the one-CTA kernel, a CTA pair of
+// the pair kernel; both CTAs of a pair walk the same items).
 struct WorkIter {
-  int t_dp;
+  int t_dp, units;
   long long it, end;
-  __device__ __forceinline__ void init(const TileSched& ts) {
-    t_dp = blockIdx.x;
-    const long long G = gridDim.x;
-    it = static_cast<long long>(blockIdx.x) * ts.sk_iters / G;
-    end = static_cast<long long>(blockIdx.x + 1) * ts.sk_iters / G;
+  __device__ __forceinline__ void init(const TileSched& ts, int unit, int nunits) {
+    t_dp = unit;
+    units = nunits;
+    const long long G = nunits;
+    it = static_cast<long long>(unit) * ts.sk_iters / G;
+    end = static_cast<long long>(unit + 1) * ts.sk_iters / G;
   }
   __device__ __forceinline__ bool next(const TileSched& ts, Item& w) {
     if (t_dp < ts.dp_tiles) {
@@ -87,7 +92,7 @@ struct WorkIter {
       w.kb1 = ts.num_kb;
       w.kind = 0;
       w.c_hi = 0;
-      t_dp += gridDim.x;
+      t_dp += units;
       return true;
     }
     if (it >= end) return false;
@@ -102,9 +107,9 @@ struct WorkIter {
     if (a == 0 && b == KB) {
       w.kind = 0;
     } else if (a == 0) {
-      // the CTA holding iteration x is floor(((x + 1) * grid - 1) / sk_iters)
+      // the unit holding iteration x is floor(((x + 1) * units - 1) / sk_iters)
       w.kind = 2;
-      const long long G = gridDim.x;
+      const long long G = units;
       w.c_hi = static_cast<int>(((u + 1) * KB * G - 1) / ts.sk_iters);
     } else {
       w.kind = 1;
@@ -145,19 +150,20 @@ __device__ __forceinline__ void store_bf16x16(bf16* dst, const float (&v)[16]) {
   d[1] = make_uint4(o[4], o[5], o[6], o[7]);
 }
 
-// Sum of the partial tiles of CTAs c0..c1 (inclusive; none if c0 > c1) at
-// this thread's row, tile columns [col, col + 16), added to v.  Partials are
-// stored column-major ([BN][BM] per CTA slot) so a warp's loads are coalesced;
-// up to four contributors' loads are in flight together, then added in order.
+// Sum of the partial tiles of contributors c0..c1 (inclusive; none if
+// c0 > c1) at this thread's row, tile columns [col, col + 16), added to v.
+// Contributor c's slot starts at ws + c * cstride.  Partials are stored
+// column-major ([BN][BM] per slot) so a warp's loads are coalesced; up to four
+// contributors' loads are in flight together, then added in order.
 template <int BN>
-__device__ __forceinline__ void add_partials(float (&v)[16], const float* ws, int c0, int c1,
-                                             int rit, int col) {
+__device__ __forceinline__ void add_partials(float (&v)[16], const float* ws, size_t cstride, int c0,
+                                             int c1, int rit, int col) {
   for (int c = c0; c <= c1; c += 4) {
     float t[4][16];
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
       if (c + k <= c1) {
-        const float* q = ws + static_cast<size_t>(c + k) * BM * BN + static_cast<size_t>(col) * BM + rit;
+        const float* q = ws + static_cast<size_t>(c + k) * cstride + static_cast<size_t>(col) * BM + rit;
 #pragma unroll
         for (int e = 0; e < 16; ++e) t[k][e] = __ldcg(q + e * BM);
       }
@@ -173,11 +179,12 @@ __device__ __forceinline__ void add_partials(float (&v)[16], const float* ws, in
 }
 
 // Epilogue of one finished accumulator tile for this thread's row; the
-// partials of CTAs c0..c1 (if any) are added to the accumulator first.
+// partials of contributors c0..c1 (slots ws + c * cstride, if any) are added
+// to the accumulator first.
 template <int BN, int EPI>
 __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_ok, int n0,
-                                              const GemmParams& p, const float* ws, int c0, int c1,
-                                              int rit) {
+                                              const GemmParams& p, const float* ws, size_t cstride,
+                                              int c0, int c1, int rit) {
   if (EPI == kEpiSwiGLU) {
     bf16* out = static_cast<bf16*>(p.out);
     const int oc0 = n0 / 2;
@@ -195,8 +202,8 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
           gv[e] = __uint_as_float(g[e]);
           uv[e] = __uint_as_float(u[e]);
         }
-        add_partials<BN>(gv, ws, c0, c1, rit, c);
-        add_partials<BN>(uv, ws, c0, c1, rit, BN / 2 + c);
+        add_partials<BN>(gv, ws, cstride, c0, c1, rit, c);
+        add_partials<BN>(uv, ws, cstride, c0, c1, rit, BN / 2 + c);
 #pragma unroll
         for (int e = 0; e < 16; ++e) v[e] = silu_f(gv[e]) * uv[e];
         store_bf16x16(out + static_cast<size_t>(row) * p.ldo + oc0 + c, v);
@@ -217,7 +224,7 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
           float v[16];
 #pragma unroll
           for (int e = 0; e < 16; ++e) v[e] = __uint_as_float(r[16 * h + e]);
-          add_partials<BN>(v, ws, c0, c1, rit, c + 16 * h);
+          add_partials<BN>(v, ws, cstride, c0, c1, rit, c + 16 * h);
           float4* dst = reinterpret_cast<float4*>(out + static_cast<size_t>(row) * p.ldo + n0 + c + 16 * h);
 #pragma unroll
           for (int q = 0; q < 4; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
@@ -256,8 +263,8 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
             a1[e] = __uint_as_float(x1[e]);
             a2[e] = __uint_as_float(x2[e]);
           }
-          add_partials<BN>(a1, ws, c0, c1, rit, hs + c);
-          add_partials<BN>(a2, ws, c0, c1, rit, hs + half + c);
+          add_partials<BN>(a1, ws, cstride, c0, c1, rit, hs + c);
+          add_partials<BN>(a2, ws, cstride, c0, c1, rit, hs + half + c);
           if (rot) {
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -327,7 +334,7 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
           float v[16];
 #pragma unroll
           for (int e = 0; e < 16; ++e) v[e] = __uint_as_float(r[16 * h + e]);
-          add_partials<BN>(v, ws, c0, c1, rit, c + 16 * h);
+          add_partials<BN>(v, ws, cstride, c0, c1, rit, c + 16 * h);
           if (EPI == kEpiResid) {
             const uint32_t rr[8] = {rc[2 * h].x, rc[2 * h].y, rc[2 * h].z, rc[2 * h].w,
                                     rc[2 * h + 1].x, rc[2 * h + 1].y, rc[2 * h + 1].z, rc[2 * h + 1].w};
@@ -411,7 +418,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t it = 0, issued_last = 0;
       bool ok = true;
       WorkIter wi;
-      wi.init(ts);
+      wi.init(ts, blockIdx.x, gridDim.x);
       // The weights are never written by another kernel: start streaming the
       // first stages' weight tiles before waiting for the previous kernel.
       int npre = 0;
@@ -487,7 +494,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       int i = 0;
       WorkIter wi;
-      wi.init(ts);
+      wi.init(ts, blockIdx.x, gridDim.x);
       Item w;
       while (ok && wi.next(ts, w)) {
         const int ab = i & 1;
@@ -523,7 +530,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int rit = quad * 32 + lane;  // row within the tile
     int i = 0;
     WorkIter wi;
-    wi.init(ts);
+    wi.init(ts, blockIdx.x, gridDim.x);
     Item w;
     while (wi.next(ts, w)) {
       const int mt = w.tile % ts.m_tiles, nt = w.tile / ts.m_tiles;
@@ -554,7 +561,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             got = got && wait_flag(ts.flags + c * 4 + quad, p.status, abort_flag);
           if (!__all_sync(0xffffffffu, got)) c1 = c0 - 1;  // gave up: status already set
         }
-        tile_epilogue<BN, EPI>(tbase, row, row < p.M, nt * BN, p, ts.ws, c0, c1, rit);
+        tile_epilogue<BN, EPI>(tbase, row, row < p.M, nt * BN, p, ts.ws, static_cast<size_t>(BM) * BN, c0, c1, rit);
         if (w.kind == 2) {
           __syncwarp();
           if (lane == 0)
@@ -592,8 +599,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 //                       accumulator to both CTAs' "acc_full" barriers;
 //   warps 2..5 (both)   epilogue of this CTA's 128 rows (the one-CTA kernel's),
 //                       then release the accumulator on the leader's barrier.
-// Whole tiles only, round robin over the pairs; tile t -> (row pair t % mp_tiles,
-// column tile t / mp_tiles), so concurrent pairs share weight tiles in L2.
+// Work is split as in the one-CTA kernel, with the pair as the unit: whole
+// tiles round robin (tile t -> row pair t % m_tiles, column tile t / m_tiles,
+// so concurrent pairs share weight tiles in L2), then, for deep K, the
+// k-iterations of the last tiles in equal ranges; CTA r of a pair that holds
+// a later part of a split tile writes its 128 rows of the partial to slot
+// blockIdx.x, and CTA r of the tile's first pair P adds the slots 2c + r of the
+// contributing pairs c, in pair order.
 // Every wait is bounded; a CTA that gives up waits briefly for its own copies
 // in flight and still reaches the closing cluster barrier.
 constexpr int P_BN = 256;
@@ -605,14 +617,10 @@ constexpr size_t P_SMEM = static_cast<size_t>(P_STAGES) * P_STAGE_BYTES + 1024 +
 constexpr uint32_t P_TMEM_COLS = 2 * P_BN;  // two accumulators
 constexpr double kPairTileCost = 0.9;
 
-struct PairSched {
-  int mp_tiles, n_tiles, num_kb, total;
-};
-
 template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_pair_kernel(const __grid_constant__ TcMaps maps, const int n1, const int n2,
-                     const GemmParams p, const PairSched ps) {
+                     const GemmParams p, const TileSched ts) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -671,27 +679,34 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       uint32_t it = 0, issued = 0;
       bool ok = true;
-      // weights are never written by another kernel: request the first tile's
+      WorkIter wi;
+      wi.init(ts, pair, npairs);
+      // weights are never written by another kernel: request the first item's
       // first stages before waiting for the previous kernel
       int npre = 0;
-      if (pair < ps.total) {
-        const CUtensorMap* mb;
-        int wy;
-        w_rows(pair / ps.mp_tiles, mb, wy);
-        npre = min(P_STAGES, ps.num_kb);
-        for (int j = 0; j < npre; ++j) {
-          if (rank == 0) mbar_arrive_expect_tx(&full[j], 2 * P_STAGE_BYTES);
-          tma_load_2d_pair(sB + j * P_B_BYTES, mb, j * BK, wy, full_leader + 8u * j);
+      {
+        WorkIter peek = wi;
+        Item w0;
+        if (peek.next(ts, w0)) {
+          const CUtensorMap* mb;
+          int wy;
+          w_rows(w0.tile / ts.m_tiles, mb, wy);
+          npre = min(P_STAGES, w0.kb1 - w0.kb0);
+          for (int j = 0; j < npre; ++j) {
+            if (rank == 0) mbar_arrive_expect_tx(&full[j], 2 * P_STAGE_BYTES);
+            tma_load_2d_pair(sB + j * P_B_BYTES, mb, (w0.kb0 + j) * BK, wy, full_leader + 8u * j);
+          }
         }
       }
       pdl_wait();
-      for (int t = pair; ok && t < ps.total; t += npairs) {
-        const int mp = t % ps.mp_tiles, nt = t / ps.mp_tiles;
+      Item w;
+      while (ok && wi.next(ts, w)) {
+        const int mp = w.tile % ts.m_tiles, nt = w.tile / ts.m_tiles;
         const int m0 = mp * (2 * BM) + rank * BM;
         const CUtensorMap* mb;
         int wy;
         w_rows(nt, mb, wy);
-        for (int kb = 0; kb < ps.num_kb; ++kb, ++it) {
+        for (int kb = w.kb0; kb < w.kb1; ++kb, ++it) {
           const int s = it % P_STAGES;
           const uint32_t ph = (it / P_STAGES) & 1;
           if (static_cast<int>(it) >= npre) {
@@ -721,14 +736,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t it = 0;
       bool ok = true;
       int i = 0;
-      for (int t = pair; ok && t < ps.total; t += npairs) {
+      WorkIter wi;
+      wi.init(ts, pair, npairs);
+      Item w;
+      while (ok && wi.next(ts, w)) {
         const int ab = i & 1;
         const uint32_t use = static_cast<uint32_t>(i >> 1);
         ++i;
         if (!mbar_wait_cluster_ab(&acc_empty[ab], (use & 1) ^ 1, p.status, abort_flag)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem + static_cast<uint32_t>(ab * P_BN);
-        for (int kb = 0; kb < ps.num_kb; ++kb, ++it) {
+        for (int kb = w.kb0; kb < w.kb1; ++kb, ++it) {
           const int s = it % P_STAGES;
           const uint32_t ph = (it / P_STAGES) & 1;
           if (!mbar_wait_ab(&full[s], ph, p.status, abort_flag)) {
@@ -741,7 +759,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
             tc_mma_bf16_pair(d_tmem, sdesc_sw128(a_base + k * 32), sdesc_sw128(b_base + k * 32), idesc,
-                             (kb > 0 || k > 0) ? 1u : 0u);
+                             (kb > w.kb0 || k > 0) ? 1u : 0u);
           tc_commit_pair(&empty[s]);
         }
         if (ok) tc_commit_pair(&acc_full[ab]);
@@ -754,9 +772,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int quad = warp & 3;
     const int rit = quad * 32 + lane;
     const uint32_t acc_empty_leader = map_rank(smem_u32(acc_empty), 0);
+    constexpr size_t kSlot = static_cast<size_t>(BM) * P_BN;  // one CTA's partial
     int i = 0;
-    for (int t = pair; t < ps.total; t += npairs) {
-      const int mp = t % ps.mp_tiles, nt = t / ps.mp_tiles;
+    WorkIter wi;
+    wi.init(ts, pair, npairs);
+    Item w;
+    while (wi.next(ts, w)) {
+      const int mp = w.tile % ts.m_tiles, nt = w.tile / ts.m_tiles;
       const int row = mp * (2 * BM) + rank * BM + rit;
       const int ab = i & 1;
       const uint32_t use = static_cast<uint32_t>(i >> 1);
@@ -765,7 +787,34 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       tc_fence_after();
       const uint32_t tbase = tmem + static_cast<uint32_t>(ab * P_BN) + (static_cast<uint32_t>(quad * 32) << 16);
-      tile_epilogue<P_BN, EPI>(tbase, row, row < p.M, nt * P_BN, p, nullptr, 1, 0, rit);
+      if (w.kind == 1) {
+        // a later part of a split tile: hand this CTA's rows to the tile's first pair
+        write_partial<P_BN>(tbase, ts.ws + static_cast<size_t>(blockIdx.x) * kSlot, rit);
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) {
+          int* f = ts.flags + blockIdx.x * 4 + quad;
+          asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(f), "r"(1) : "memory");
+        }
+      } else {
+        int c0 = 1, c1 = 0;  // no partials
+        if (w.kind == 2) {
+          c0 = pair + 1;
+          c1 = w.c_hi;
+          bool got = true;
+          for (int c = c0; c <= c1; ++c)
+            got = got && wait_flag(ts.flags + (2 * c + rank) * 4 + quad, p.status, abort_flag);
+          if (!__all_sync(0xffffffffu, got)) c1 = c0 - 1;  // gave up: status already set
+        }
+        // contributor pair c's rows of this CTA are in slot 2c + rank
+        const float* ws = c0 <= c1 ? ts.ws + rank * kSlot : nullptr;
+        tile_epilogue<P_BN, EPI>(tbase, row, row < p.M, nt * P_BN, p, ws, 2 * kSlot, c0, c1, rit);
+        if (w.kind == 2) {
+          __syncwarp();
+          if (lane == 0)
+            for (int c = c0; c <= c1; ++c) ts.flags[(2 * c + rank) * 4 + quad] = 0;
+        }
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(acc_empty_leader + 8u * ab);
@@ -897,7 +946,7 @@ int pair_slots_for(int epi) {
 }
 
 template <int EPI>
-cudaError_t run_pair(const TcMaps& maps, int n1, int n2, const GemmParams& p, const PairSched& ps,
+cudaError_t run_pair(const TcMaps& maps, int n1, int n2, const GemmParams& p, const TileSched& ps,
                      int pairs, cudaStream_t s) {
   cudaError_t e = pair_attr<EPI>();
   if (e != cudaSuccess) return e;
@@ -910,7 +959,7 @@ cudaError_t run_pair(const TcMaps& maps, int n1, int n2, const GemmParams& p, co
 }
 
 cudaError_t dispatch_pair(int epi, const TcMaps& maps, int n1, int n2, const GemmParams& p,
-                          const PairSched& ps, int pairs, cudaStream_t s) {
+                          const TileSched& ps, int pairs, cudaStream_t s) {
   switch (epi) {
     case kEpiStore: return run_pair<kEpiStore>(maps, n1, n2, p, ps, pairs, s);
     case kEpiResid: return run_pair<kEpiResid>(maps, n1, n2, p, ps, pairs, s);
@@ -993,20 +1042,37 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
   // pair wave takes 0.84..0.96 of a one-CTA wave, but pairing 128-row tiles
   // can leave half a pair empty and add a wave, and in a single short-K wave
   // the pair's extra synchronisation costs 1..4%, so pairs are taken when they
-  // save waves at kPairTileCost each, and in one wave only for deep K.
-  PairSched ps{};
+  // save waves at kPairTileCost each, and in one wave only for deep K.  Where
+  // the one-CTA plan splits the last waves' k-blocks (deep K, ragged last
+  // wave), the pairs split them instead.
+  TileSched ps{};
   int pairs = 0;
-  if (BN == P_BN && ts.sk_iters == 0) {
+  if (BN == P_BN) {
     const int slots = pair_slots_for(epi);
-    ps.mp_tiles = (m_tiles + 1) / 2;
+    ps.m_tiles = (m_tiles + 1) / 2;  // 256-row tiles
     ps.n_tiles = ts.n_tiles;
     ps.num_kb = ts.num_kb;
-    ps.total = ps.mp_tiles * ps.n_tiles;
-    if (slots > 0) {
+    ps.total = ps.m_tiles * ps.n_tiles;
+    ps.ws = ts.ws;
+    ps.flags = ts.flags;
+    if (slots > 0 && ts.sk_iters == 0) {
       const int waves_pair = (ps.total + slots - 1) / slots;
       const int waves_one = (ts.total + sms - 1) / sms;
-      if (waves_pair * kPairTileCost < waves_one && (waves_one >= 2 || ps.num_kb >= 64))
+      if (waves_pair * kPairTileCost < waves_one && (waves_one >= 2 || ps.num_kb >= 64)) {
+        ps.dp_tiles = ps.total;
+        ps.sk_iters = 0;
         pairs = ps.total < slots ? ps.total : slots;
+      }
+    } else if (slots > 0 && 2 * slots <= kMaxGemmCtas &&
+               static_cast<size_t>(2 * slots) * BM * P_BN <= p.splitk_ws_elems) {
+      // deep K with a ragged last wave: the same stream-K split over the pairs
+      pairs = slots;
+      ps.dp_tiles = ps.total >= 2 * pairs ? (ps.total / pairs - 1) * pairs : 0;
+      ps.sk_iters = static_cast<long long>(ps.total - ps.dp_tiles) * ps.num_kb;
+      if (ps.dp_tiles == 0) {  // small problem: keep at least 8 k-blocks per pair
+        const long long g = ps.sk_iters / 8;
+        pairs = static_cast<int>(g < 1 ? 1 : (g < slots ? g : slots));
+      }
     }
   }
   TcMaps maps;

@@ -76,3 +76,46 @@ def test_pair_deterministic(z):
     z.zsaa_device_status()
     assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
 
+
+
+# Deep K (64 k-blocks and more) with a ragged last wave: the last tiles' k-blocks
+# are split over the pairs.  1100 rows x 1040 columns: 25 pair tiles over all
+# pairs, so most tiles have three or four contributing pairs; 5000 rows x 2048:
+# whole tiles for one wave of pairs, the rest split.
+@pytest.mark.parametrize("M,N", [(1100, 1040), (5000, 2048)])
+@pytest.mark.parametrize("epi", ["store_f32", "resid"])
+def test_pair_streamk_plain(z, epi, M, N):
+    out, ref, tol = linear_case(z, epi, M, N, 4096, 1000 + M + N)
+    check_linear(out, ref, tol, epi, f"{epi} M={M} N={N}")
+
+
+def test_pair_streamk_swiglu(z):
+    out, ref, tol = linear_case(z, "swiglu", 1100, 1088, 4096, 1100)
+    check_linear(out, ref, tol, "swiglu", "M=1100 K=4096")
+
+
+def test_pair_streamk_rope(z):
+    # Llama-3.1-8B QKV layout: 16 query + 4 key heads rotated, 4 value heads, hd 128
+    out, ref, tol = linear_case(z, "rope", 1100, 3072, 4096, 1200, hd=128, rope_cols=2560)
+    check_linear(out, ref, tol, "rope", "hd=128 K=4096")
+
+
+def test_pair_streamk_down_1b(z):
+    # the 1B down projection at 3296 kept rows: 104 pair tiles of 128 k-blocks
+    out, ref, tol = linear_case(z, "resid", 3296, 2048, 8192, 1300)
+    check_linear(out, ref, tol, "resid", "down M=3296")
+
+
+def test_pair_streamk_deterministic(z):
+    # split tiles add their partials in pair order: repeated calls agree bit for bit
+    M, N, K = 1100, 1040, 4096
+    A = rand_bf16((M, K), 21)
+    W = rand_bf16((N, K), 22, 0.05)
+    outs = []
+    for _ in range(3):
+        out = torch.empty(M, N, device="cuda", dtype=torch.float32)
+        z.zsaa_op_linear(A, W, None, None, out, M, N, K, z.ZSAA_BF16, z.EPI_STORE_F32)
+        outs.append(out)
+    torch.cuda.synchronize()
+    z.zsaa_device_status()
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
