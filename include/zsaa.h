@@ -334,8 +334,12 @@ zsaa_status zsaa_score_select_noalloc(const void* hidden, int B, int L, int d, i
  * the tcgen05 GEMMs (M <= 16 without RoPE: the weight-streaming GEMM; up to a
  * few hundred rows, by epilogue: the swapped-operand GEMM whose thread-block
  * cluster adds its split-K partials in a fixed order, so results do not depend
- * on timing; larger M: the persistent tiled GEMM), ZSAA_F32 the fp32 CUDA-core
- * GEMM.  The bf16 kernels start reading W before the
+ * on timing; larger M: the persistent tiled GEMM, on clusters of two CTAs
+ * sharing 256 x 256 tiles through the 2-SM MMA where that saves waves, its
+ * split-K partials also added in a fixed order), ZSAA_F32 the fp32 CUDA-core
+ * GEMM.  ZSAA_GEMM_PAIRS=0 in the environment (read once per process) keeps
+ * the tiled GEMM on one CTA, a diagnostic switch with the same results up to
+ * summation order.  The bf16 kernels start reading W before the
  * previous library kernel on the stream has finished: W and W2 must not be
  * written by that kernel.  epilogue:
  *   0 store (out has dtype; bf16 rounds once),

@@ -28,6 +28,7 @@
 // word, the other roles stop waiting, in-flight copies are drained (bounded)
 // and TMEM is freed before the CTA exits.
 #include <cstdio>
+#include <cstdlib>
 #include <mutex>
 
 #include "common.cuh"
@@ -934,6 +935,18 @@ int pair_slots() {
   return n > 0 ? n : 0;
 }
 
+// ZSAA_GEMM_PAIRS=0 in the environment (read once per process) keeps every
+// tiled GEMM on one CTA: a diagnostic switch, so the one-CTA kernel's whole
+// and split paths -- the fallback where CTA pairs cannot be scheduled -- can
+// be tested and timed against the pairs on a GPU that has them.
+bool pairs_enabled() {
+  static const bool on = [] {
+    const char* e = std::getenv("ZSAA_GEMM_PAIRS");
+    return !(e != nullptr && e[0] == '0');
+  }();
+  return on;
+}
+
 int pair_slots_for(int epi) {
   switch (epi) {
     case kEpiStore: return pair_slots<kEpiStore>();
@@ -1047,7 +1060,7 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
   // wave), the pairs split them instead.
   TileSched ps{};
   int pairs = 0;
-  if (BN == P_BN) {
+  if (BN == P_BN && pairs_enabled()) {
     const int slots = pair_slots_for(epi);
     ps.m_tiles = (m_tiles + 1) / 2;  // 256-row tiles
     ps.n_tiles = ts.n_tiles;

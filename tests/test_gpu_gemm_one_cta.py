@@ -1,0 +1,46 @@
+"""Parity of the one-CTA tiled GEMM on the shapes that otherwise run on CTA
+pairs: its whole-tile path and its stream-K path (deep K, ragged last wave),
+the fallback where pairs cannot be scheduled, against the same float64
+references as the pair tests.  ZSAA_GEMM_PAIRS=0 is read once per process,
+so the cases run in a child process with it set."""
+
+import os
+import subprocess
+import sys
+
+import pytest
+
+from tests.helpers import check_linear, linear_case, need_gpu
+
+pytestmark = pytest.mark.gpu
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+# (epilogue, M, N, K): whole tiles (two waves), then deep K split over the CTAs
+# (1100 x 1040: 45 tiles of 64 k-blocks over all SMs; 5000 x 2048: one wave
+# whole, the rest split; the 1B down projection at 3296 rows)
+CASES = [("store", 2056, 2064, 512), ("swiglu", 2300, 1088, 512), ("rope", 2300, 3072, 512),
+         ("store_f32", 1100, 1040, 4096), ("resid", 5000, 2048, 4096), ("swiglu", 1100, 1088, 4096),
+         ("rope", 1100, 3072, 4096), ("resid", 3296, 2048, 8192)]
+
+
+def _run_cases():
+    from paper_2509_01190_gb300 import zsaa as z
+    for i, (epi, M, N, K) in enumerate(CASES):
+        out, ref, tol = linear_case(z, epi, M, N, K, 1400 + i, hd=64, rope_cols=2560)
+        check_linear(out, ref, tol, epi, f"one CTA {epi} M={M} N={N} K={K}")
+        print(f"ok {epi} M={M} N={N} K={K}", flush=True)
+
+
+def test_one_cta_tiled_paths(zlib):
+    need_gpu()
+    env = dict(os.environ, ZSAA_GEMM_PAIRS="0")
+    r = subprocess.run([sys.executable, "-m", "tests.test_gpu_gemm_one_cta"], cwd=ROOT, env=env,
+                       capture_output=True, text=True, timeout=900)
+    assert r.returncode == 0, r.stdout[-3000:] + r.stderr[-3000:]
+    assert r.stdout.count("ok ") == len(CASES), r.stdout
+
+
+if __name__ == "__main__":
+    sys.path.insert(0, ROOT)
+    _run_cases()
