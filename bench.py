@@ -348,6 +348,7 @@ def main():
         print(json.dumps(line))
         return
 
+    from paper_2509_01190_gb300 import replicas as R
     from paper_2509_01190_gb300 import zsaa
 
     if world > 1:
@@ -361,20 +362,13 @@ def main():
     stream = torch.cuda.current_stream()
 
     def barrier():
-        torch.cuda.synchronize()
-        if dist is not None:
-            dist.barrier()
-        torch.cuda.synchronize()
+        R.barrier(dist, torch.cuda.synchronize)
 
     def max_over_ranks(x):
-        if dist is None:
-            return x
-        t = torch.tensor([x], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+        return R.max_over_ranks(x, dist, dev)
 
     weights = I.make_weights(shape, device=dev)
-    tokens = I.make_tokens(B, L, shape.vocab, seed=I.TOKEN_SEED + rank)
+    tokens = I.make_tokens(B, L, shape.vocab, seed=R.rank_token_seed(I.TOKEN_SEED, rank))
     tok_dev = torch.from_numpy(tokens).to(dev)
     cfg = zsaa.config_from_shape(shape)
     model = zsaa.Model(cfg, weights, B, L)
@@ -414,7 +408,7 @@ def main():
     sampler = ClockSampler(local) if rank == 0 else None
     ms_head = timed(args.accel, args.steps, args.warmup, sampler)
     sched, alpha = zsaa.zsaa_plan(model, L, args.accel)
-    value = world * B * L / (ms_head / 1e3)
+    value = R.job_tokens_per_s(world, B, L, ms_head)
     clocks = sampler.summary() if sampler else None
 
     line = {"metric": "prefill_tokens_per_s", "value": value, "unit": "tokens/s", "n_gpus": world,
@@ -439,7 +433,7 @@ def main():
             s_a, al_a = zsaa.zsaa_plan(model, L, a)
             if a == 1.0:
                 base_ms = ms
-            sweep[f"{a:g}"] = {"ms": ms, "tokens_per_s": world * B * L / (ms / 1e3), "alpha": al_a,
+            sweep[f"{a:g}"] = {"ms": ms, "tokens_per_s": R.job_tokens_per_s(world, B, L, ms), "alpha": al_a,
                                "final_rows": s_a[-1],
                                "modelled_flop_reduction": full_cost / O.model_cost(ocfg, s_a)}
         for k, v in sweep.items():
@@ -566,7 +560,7 @@ def main():
             zsaa.zsaa_sync(model)
             ms_m = max_over_ranks(sum(a.elapsed_time(b) for a, b in evs) / args.steps)
             line["masked_mode"] = {"accel": args.accel, "ms_per_step": ms_m,
-                                   "tokens_per_s": world * B * L / (ms_m / 1e3),
+                                   "tokens_per_s": R.job_tokens_per_s(world, B, L, ms_m),
                                    "vs_compacted": ms_m / ms_head, "final_rows": n_fin,
                                    "note": "zsaa_forward_masked, eager launches"}
 
