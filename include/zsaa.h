@@ -403,6 +403,16 @@ zsaa_status zsaa_sync(zsaa_model* m, zsaa_stream stream);
  * zsaa_op_*): synchronises the device, returns it and clears it. */
 zsaa_status zsaa_device_status(void);
 
+/* Self-test of the device failure path (bounded waits that report a status,
+ * never a trap: the error model above).  Launches on `stream` one CTA whose two roles wait,
+ * with the same bounded mbarrier wait as every pipelined kernel, for a barrier
+ * phase that nothing completes.  The wait gives up after its limit (2 s), sets
+ * the timeout bit of the status word shared by the model-less calls, and the
+ * kernel returns; the context stays usable.  Waits for the stream and returns
+ * that status (then clears it): ZSAA_ERR_TIMEOUT when the path works, ZSAA_OK
+ * if the wait ended some other way.  Takes about 2 s of GPU time. */
+zsaa_status zsaa_selftest_wait_timeout(zsaa_stream stream);
+
 /* Message of the last failing call on this thread ("" if none). */
 const char* zsaa_last_error(void);
 

@@ -1377,6 +1377,25 @@ zsaa_status read_status(int* word, cudaStream_t s, bool whole_device) {
   return ZSAA_OK;
 }
 
+// Self-test of the failure path every pipelined kernel takes: two roles wait,
+// with the library's bounded mbarrier wait, for a phase of a barrier whose one
+// expected arrival never comes (a producer that stopped).  The first wait to
+// run out (kWaitLimitNs) sets the timeout bit of the status word and the CTA's
+// stop flag; the other role sees the flag and stops; the kernel returns.  No
+// trap, no fault: the context stays usable.
+__global__ void wait_timeout_selftest_kernel(int* status) {
+  __shared__ uint64_t bar;
+  __shared__ int stop;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    stop = 0;
+    fence_barrier_init();
+  }
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) mbar_wait_ab(&bar, 0, status, reinterpret_cast<volatile int*>(&stop));
+  __syncthreads();
+}
+
 // cos/sin of RoPE for positions [0, n_pos): angle(p, i) = p * theta^(-2i/hd), in double.
 void rope_host_table(double theta, int hd, int n_pos, std::vector<float>* cs, std::vector<float>* sn) {
   const int half = hd / 2;
@@ -2086,6 +2105,15 @@ zsaa_status zsaa_device_status(void) {
   int* w = shared_status();
   if (w == nullptr) return fail(ZSAA_ERR_CUDA, "status word allocation failed");
   return read_status(w, nullptr, true);
+}
+
+zsaa_status zsaa_selftest_wait_timeout(zsaa_stream stream) {
+  int* w = shared_status();
+  if (w == nullptr) return fail(ZSAA_ERR_CUDA, "status word allocation failed");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  wait_timeout_selftest_kernel<<<1, 64, 0, s>>>(w);
+  ZCK(cudaGetLastError());
+  return read_status(w, s, false);
 }
 
 }  // extern "C"

@@ -30,7 +30,7 @@ EXPORTED = [
     "zsaa_score_select_noalloc", "zsaa_model_set_graphs", "zsaa_cache_create", "zsaa_cache_destroy",
     "zsaa_prefill", "zsaa_decode_step", "zsaa_cache_layer", "zsaa_cache_bytes",
     "zsaa_op_attention_ex", "zsaa_op_colmass_ex", "zsaa_plan_varlen_config", "zsaa_plan_varlen",
-    "zsaa_forward_varlen", "zsaa_forward_masked",
+    "zsaa_forward_varlen", "zsaa_forward_masked", "zsaa_selftest_wait_timeout",
 ]
 
 
@@ -103,6 +103,7 @@ def lib():
             "zsaa_op_colmass_ex": ([_P, _P, _I, _I, _I, _I, _I, _I, _I, _P, _P], _I),
             "zsaa_sync": ([_P, _P], _I),
             "zsaa_device_status": ([], _I),
+            "zsaa_selftest_wait_timeout": ([_P], _I),
             "zsaa_last_error": ([], C.c_char_p),
             "zsaa_version": ([], C.c_char_p),
             "zsaa_trace_begin": ([_P], _I),
@@ -454,6 +455,12 @@ def zsaa_op_colmass_ex(qkv, lse, B: int, N: int, Hq: int, Hkv: int, hd: int, dty
 
 def zsaa_device_status():
     _check(lib().zsaa_device_status())
+
+
+def zsaa_selftest_wait_timeout(stream=None) -> int:
+    """Run the bounded-wait self-test; returns its status code (ZSAA_ERR_TIMEOUT
+    when a wait that nothing completes gives up and reports, as it should)."""
+    return int(lib().zsaa_selftest_wait_timeout(_stream(stream)))
 
 
 def zsaa_last_error() -> str:
