@@ -79,7 +79,8 @@ struct GemmParams {
 };
 
 // Stream-K workspace a caller should provide: one 128 x 256 fp32 tile per CTA
-// (at most kMaxGemmCtas CTAs), and 4 flags per CTA.
+// (at most kMaxGemmCtas CTAs; the pair kernel counts both CTAs of a pair), and
+// 4 flags per CTA.
 constexpr int kMaxGemmCtas = 256;
 constexpr size_t kSplitKWorkspaceElems = static_cast<size_t>(kMaxGemmCtas) * 128 * 256;
 constexpr size_t kSplitKFlags = static_cast<size_t>(kMaxGemmCtas) * 4;
@@ -94,6 +95,11 @@ struct TcWeights {
   const void* w2;
   int n1, n2;
 };
+// Routing by rows: up to kSkinnyMaxM the weight-streaming kernel; up to the
+// swap_preferred limit the swapped-operand kernel; else the persistent tiled
+// kernel (k_gemm_tc.cu) on one CTA per SM, or on clusters of two CTAs sharing
+// 256 x 256 tiles through the 2-SM MMA where that saves waves or splits a deep
+// K (ZSAA_GEMM_PAIRS=0 in the environment keeps one CTA).
 cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
                            const GemmParams& p, cudaStream_t s);
 
