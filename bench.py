@@ -48,12 +48,12 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # of one forward.  Reported only while the sources it was measured on are
 # unchanged (sha256 below), else null.
 GATE_UP_TRAFFIC = {
-    "bytes_per_launch": 74129520.0,
+    "bytes_per_launch": 74152480.0,
     "sources": {
         "paper_2509_01190_gb300/csrc/k_gemm_tc.cu": "ddc8d600807e9f44c045b53ca23655630f067cd92efa283e0fce0da8bc0edb2c",
         "paper_2509_01190_gb300/csrc/k_gemm_swap.cu": "36ffbbf0ac0ad5b7c817381f5591920cef6253be33ef3ddcea386543f6a40c46",
         "paper_2509_01190_gb300/csrc/common.cuh": "8d770ec1038f925c2dff1202d62b07c60ac07893cae579860cb5e285868bca05",
-        "paper_2509_01190_gb300/csrc/kernels.h": "6903cca528c43eba183afd4b0c08d40c55cab2b211699400c663d495b3a645ae",
+        "paper_2509_01190_gb300/csrc/kernels.h": "0948b1ead255b4c00af6b57bb1cf37f4b647833fbcc93065231146e1f4cf4807",
     },
 }
 
@@ -72,6 +72,19 @@ def measured_traffic(kernel_name):
         except OSError:
             return None
     return GATE_UP_TRAFFIC["bytes_per_launch"]
+
+
+def _tensors(obj):
+    """Every tensor in a nest of dicts, lists and tuples."""
+    import torch
+    if isinstance(obj, torch.Tensor):
+        yield obj
+    elif isinstance(obj, dict):
+        for v in obj.values():
+            yield from _tensors(v)
+    elif isinstance(obj, (list, tuple)):
+        for v in obj:
+            yield from _tensors(v)
 
 
 def load_peaks():
@@ -368,6 +381,7 @@ def main():
         return R.max_over_ranks(x, dist, dev)
 
     weights = I.make_weights(shape, device=dev)
+    w_gb = sum(t.numel() * t.element_size() for t in _tensors(weights)) / 1e9
     tokens = I.make_tokens(B, L, shape.vocab, seed=R.rank_token_seed(I.TOKEN_SEED, rank))
     tok_dev = torch.from_numpy(tokens).to(dev)
     cfg = zsaa.config_from_shape(shape)
@@ -418,7 +432,7 @@ def main():
             "config": {"workload": workload_name, "model": shape.name, "global_batch": B * world,
                        "seq_len": L, "accel": args.accel, "alpha": alpha, "schedule": sched,
                        "parallelism": f"replicas x{world} (independent sequences, no collective)",
-                       "l2": "flushed between timed steps (256 MiB write); weights 2.5 GB > L2"},
+                       "l2": f"flushed between timed steps (256 MiB write); weights {w_gb:.1f} GB > L2"},
             "clocks": clocks}
 
     if not args.no_extras:
