@@ -381,7 +381,7 @@ def main():
         return R.max_over_ranks(x, dist, dev)
 
     weights = I.make_weights(shape, device=dev)
-    w_gb = sum(t.numel() * t.element_size() for t in _tensors(weights)) / 1e9
+    w_gb = sum({t.data_ptr(): t.numel() * t.element_size() for t in _tensors(weights)}.values()) / 1e9  # tied: once
     tokens = I.make_tokens(B, L, shape.vocab, seed=R.rank_token_seed(I.TOKEN_SEED, rank))
     tok_dev = torch.from_numpy(tokens).to(dev)
     cfg = zsaa.config_from_shape(shape)

@@ -38,6 +38,15 @@ __global__ void embed_kernel(const uint4* __restrict__ E, const int32_t* __restr
 
 // ---------------------------------------------------------------- RMSNorm
 
+// The norm weights of a row (n16 16-byte vectors) are never written by a
+// kernel: a warp asks L2 for them, one 128-byte line per lane, before it waits
+// for the previous kernel, so they are not a round trip on the row's chain of
+// dependent loads.
+__device__ __forceinline__ void prefetch_norm_weights(const uint4* w, int n16, int lane) {
+  for (int line = lane; line * 8 < n16; line += 32)
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(w + line * 8));
+}
+
 template <typename T>
 __global__ void rmsnorm_kernel(const T* __restrict__ h, const T* __restrict__ w, int rows, int d,
                                float eps, T* __restrict__ x) {
@@ -63,9 +72,10 @@ __global__ void rmsnorm_bf16_vec_kernel(const uint4* __restrict__ h, const uint4
                                         int rows, int vec_per_row, float eps,
                                         uint4* __restrict__ x) {
   pdl_trigger();
-  pdl_wait();
   const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
+  if (threadIdx.x < 32) prefetch_norm_weights(w, vec_per_row, lane);
+  pdl_wait();
   if (r >= rows) return;
   const uint4* hr = h + static_cast<size_t>(r) * vec_per_row;
   uint4* xr = x + static_cast<size_t>(r) * vec_per_row;
@@ -379,9 +389,10 @@ __global__ void rows_norm_bf16_kernel(const uint4* __restrict__ src, const int32
                                       const int* __restrict__ cu_src, const int* __restrict__ cu_dst,
                                       int nseq) {
   pdl_trigger();
-  pdl_wait();
   const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
+  if (threadIdx.x < 32) prefetch_norm_weights(w, vec, lane);
+  pdl_wait();
   if (r >= rows) return;
   size_t srow;
   int p;
