@@ -53,14 +53,6 @@ constexpr int SW_MAX_CLUSTER = 8;
 constexpr int SW_RING_BUDGET = 220 * 1024;  // bytes of stage ring per CTA
 constexpr int SW_MAX_STAGES = 8;
 
-// Internal epilogue id: float32 store for very wide outputs (the LM head):
-// each CTA owns sh.nb adjacent 128-row weight bands, one TMEM accumulator per
-// band at columns i * sh.band_cols, all fed by the same activation tile, no
-// split-K, logits written straight from TMEM.  The activation rows are then
-// streamed once per nb bands instead of once per band.
-constexpr int kSwapHeadF32 = 6;
-constexpr int kSwapHeadMinN = 32768;
-
 struct SwMaps {
   CUtensorMap x, w0, w1, w2;
 };
@@ -69,8 +61,6 @@ struct SwShape {
   int Mp;         // activation rows per row block (multiple of 16, <= 256): the MMA's N
   int stages;     // depth of the stage ring
   int ksub;       // k-blocks of 64 per stage
-  int nb;         // weight bands per CTA (kSwapHeadF32; else 1)
-  int band_cols;  // TMEM columns between the bands' accumulators
   int nkb;        // k-blocks of 64
   int n1, n2;     // weight row blocks (non-SwiGLU): w0 [0, n1), w1 [n1, n2), w2 [n2, N)
   uint32_t tmem_cols;
@@ -277,12 +267,11 @@ template <int EPI>
 __global__ void __launch_bounds__(SW_THREADS, 1)
     gemm_swap_kernel(const __grid_constant__ SwMaps maps, const SwShape sh, const GemmParams p) {
   constexpr bool DUAL = EPI == kEpiSwiGLU;
-  constexpr bool HEAD = EPI == kSwapHeadF32;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   const int X_BYTES = sh.Mp * SW_BK * 2;  // one activation sub-tile [Mp x 64]
-  const int WSUB = (HEAD ? sh.nb : 1) * SW_W_BYTES;  // weight bytes of one k-block
+  const int WSUB = SW_W_BYTES;  // weight bytes of one k-block
   const int STAGES = sh.stages, KSUB = sh.ksub;
   uint8_t* sW = smem;                                     // [STAGES][KSUB] weight sub-tiles
   uint8_t* sX = smem + STAGES * KSUB * WSUB;              // [STAGES][KSUB] activation sub-tiles
@@ -332,9 +321,6 @@ __global__ void __launch_bounds__(SW_THREADS, 1)
       if (DUAL) {
         wm0 = &maps.w0;
         wy = band * (SW_BAND / 2);
-      } else if (HEAD) {
-        wm0 = &maps.w0;
-        wy = band * sh.nb * SW_BAND;
       } else {
         const int n0 = band * SW_BAND;
         wm0 = n0 >= sh.n2 ? &maps.w2 : (n0 >= sh.n1 ? &maps.w1 : &maps.w0);
@@ -346,11 +332,7 @@ __global__ void __launch_bounds__(SW_THREADS, 1)
         for (int u = 0; u < nsub_of(j); ++u) {
           uint8_t* d = sW + (s * KSUB + u) * WSUB;
           const int x = (kb0 + j * KSUB + u) * SW_BK;
-          if (HEAD) {  // nb bands; rows past N read as zeros
-            for (int i = 0; i < sh.nb; ++i) tma_load_2d(d + i * SW_W_BYTES, wm0, x, wy + i * SW_BAND, &full[s]);
-          } else {
-            tma_load_2d(d, wm0, x, wy, &full[s]);
-          }
+          tma_load_2d(d, wm0, x, wy, &full[s]);
           if (DUAL) tma_load_2d(d + (SW_BAND / 2) * 128, wm1, x, wy, &full[s]);
         }
       };
@@ -408,14 +390,7 @@ __global__ void __launch_bounds__(SW_THREADS, 1)
 #pragma unroll
           for (int k = 0; k < SW_BK / 16; ++k) {
             const uint32_t acc = (j > 0 || u > 0 || k > 0) ? 1u : 0u;
-            if (HEAD) {
-              for (int i = 0; i < sh.nb; ++i)
-                tc_mma_bf16(tmem + static_cast<uint32_t>(i * sh.band_cols),
-                            sdesc_sw128(w_base + i * SW_W_BYTES + k * 32), sdesc_sw128(x_base + k * 32),
-                            idesc, acc);
-            } else {
-              tc_mma_bf16(tmem, sdesc_sw128(w_base + k * 32), sdesc_sw128(x_base + k * 32), idesc, acc);
-            }
+            tc_mma_bf16(tmem, sdesc_sw128(w_base + k * 32), sdesc_sw128(x_base + k * 32), idesc, acc);
           }
         }
         tc_commit(&empty[s]);
@@ -431,28 +406,7 @@ __global__ void __launch_bounds__(SW_THREADS, 1)
     const int h = (warp - 2) >> 2;
     const int n = quad * 32 + lane;
     const bool ok = __all_sync(0xffffffffu, mbar_wait_ab(acc_full, 0, p.status, abort_flag));
-    if (ok && HEAD) {
-      // logits[row0 + m, (band*nb + i)*128 + n] straight from TMEM: a warp stores
-      // 32 adjacent floats of one row per instruction
-      pdl_wait();
-      tc_fence_after();
-      const uint32_t tb = tmem + (static_cast<uint32_t>(quad * 32) << 16);
-      float* out = static_cast<float*>(p.out);
-      for (int i = 0; i < sh.nb; ++i) {
-        const int col = (band * sh.nb + i) * SW_BAND + n;
-#pragma unroll 1
-        for (int c = 16 * h; c < sh.Mp; c += 32) {
-          uint32_t r[16];
-          tmem_ld16(tb + static_cast<uint32_t>(i * sh.band_cols + c), r);
-          tmem_ld_wait();
-          if (col < p.N) {
-#pragma unroll
-            for (int e = 0; e < 16; ++e)
-              if (c + e < rows) out[static_cast<size_t>(row0 + c + e) * p.ldo + col] = __uint_as_float(r[e]);
-          }
-        }
-      }
-    } else if (ok) {
+    if (ok) {
       tc_fence_after();
       fence_proxy_async_smem();  // the ring was last written by TMA, read by the MMAs
       const uint32_t tb = tmem + (static_cast<uint32_t>(quad * 32) << 16);
@@ -477,7 +431,7 @@ __global__ void __launch_bounds__(SW_THREADS, 1)
   // ---- reduction over the cluster and epilogue: CTA `rank` finishes rows
   // [rank rows / S, (rank + 1) rows / S) of this block.
   pdl_wait();
-  if (!HEAD && *abort_flag == 0) {
+  if (*abort_flag == 0) {
     uint32_t src[SW_MAX_CLUSTER];
     const uint32_t red_local = smem_u32(red);
 #pragma unroll
@@ -568,7 +522,6 @@ cudaError_t run_swap(const void* A, int lda, const TcWeights& W, const GemmParam
   cudaError_t e = ensure_attr<EPI>();
   if (e != cudaSuccess) return e;
   constexpr bool DUAL = EPI == kEpiSwiGLU;
-  constexpr bool HEAD = EPI == kSwapHeadF32;
   // row blocks of at most 256 rows, as even as 16-row granularity allows
   const int nrb = (p.M + kSwapRowBlock - 1) / kSwapRowBlock;
   const int per = (p.M + nrb - 1) / nrb;
@@ -579,12 +532,7 @@ cudaError_t run_swap(const void* A, int lda, const TcWeights& W, const GemmParam
   // a stage holds, so a stage takes as many 64-wide k-blocks (up to 4) as
   // still leaves two stages in the ring (a TMA probe on one SM streamed best
   // with about 100 KB per stage).
-  // HEAD: as many 128-row bands per CTA as TMEM holds accumulators for (up to 4)
-  sh.band_cols = 32;
-  while (sh.band_cols < sh.Mp) sh.band_cols += 32;
-  sh.nb = HEAD ? 512 / sh.band_cols : 1;
-  if (sh.nb > 4) sh.nb = 4;
-  const int kblock = sh.nb * SW_W_BYTES + sh.Mp * SW_BK * 2;
+  const int kblock = SW_W_BYTES + sh.Mp * SW_BK * 2;
   sh.ksub = SW_RING_BUDGET / (2 * kblock);
   if (sh.ksub > 4) sh.ksub = 4;
   if (sh.ksub < 1) sh.ksub = 1;
@@ -595,18 +543,16 @@ cudaError_t run_swap(const void* A, int lda, const TcWeights& W, const GemmParam
   sh.n2 = DUAL ? p.N : W.n2;
   uint32_t cols = 32;
   while (cols < static_cast<uint32_t>(sh.Mp)) cols <<= 1;
-  sh.tmem_cols = HEAD ? 512 : cols;
-  const int bands = DUAL   ? (p.N + SW_BAND / 2 - 1) / (SW_BAND / 2)
-                    : HEAD ? (p.N + sh.nb * SW_BAND - 1) / (sh.nb * SW_BAND)
-                           : (p.N + SW_BAND - 1) / SW_BAND;
-  const size_t smem = smem_bytes(sh.nb * SW_W_BYTES, sh.Mp, sh.stages, sh.ksub);
+  sh.tmem_cols = cols;
+  const int bands = DUAL ? (p.N + SW_BAND / 2 - 1) / (SW_BAND / 2) : (p.N + SW_BAND - 1) / SW_BAND;
+  const size_t smem = smem_bytes(SW_W_BYTES, sh.Mp, sh.stages, sh.ksub);
 
   // Cluster size: fewest k-blocks per CTA over the waves the clusters need;
   // a wave costs about two k-blocks of fixed work (launch, TMEM, reduction).
   const int units = bands * nrb2;
   int best = 1;
   double best_cost = 1e30;
-  for (int S = 1; S <= (HEAD ? 1 : SW_MAX_CLUSTER) && S <= sh.nkb; ++S) {  // HEAD: no split-K
+  for (int S = 1; S <= SW_MAX_CLUSTER && S <= sh.nkb; ++S) {
     const int mc = max_clusters<EPI>(S, smem);
     if (mc <= 0) continue;
     const int waves = (units + mc - 1) / mc;
@@ -667,11 +613,14 @@ bool swap_supported(const void* A, int lda, const TcWeights& W, int epi, const G
   return true;
 }
 
-bool swap_preferred(int epi, int M) {
+bool swap_preferred(int epi, int M, int N) {
   // Crossovers measured on GB300 for the Llama-3.2-1B and -8B projections
   // (CUDA-graph timed, weights streamed from HBM): above these row counts the
   // persistent tiled kernel keeps more SMs busy (SwiGLU needs two waves of
-  // 128-row bands from 257 rows on) or streams its tiles faster.
+  // 128-row bands from 257 rows on) or streams its tiles faster.  Very wide
+  // float32 outputs (LM heads, N >= 32768) stream their weights faster on the
+  // tiled kernel at every row count (1B head at 40..456 rows: 0.68..0.94x).
+  if (epi == kEpiStoreF32 && N >= 32768) return false;
   const int limit = epi == kEpiSwiGLU ? 256 : (epi == kEpiResid ? 1024 : 768);
   return M <= limit;
 }
@@ -682,9 +631,7 @@ cudaError_t launch_gemm_swap(const void* A, int lda, const TcWeights& W, int epi
     case kEpiStore: return run_swap<kEpiStore>(A, lda, W, p, s);
     case kEpiResid: return run_swap<kEpiResid>(A, lda, W, p, s);
     case kEpiSwiGLU: return run_swap<kEpiSwiGLU>(A, lda, W, p, s);
-    case kEpiStoreF32:  // very wide outputs (the LM head): several bands per CTA
-      return p.N >= kSwapHeadMinN ? run_swap<kSwapHeadF32>(A, lda, W, p, s)
-                                  : run_swap<kEpiStoreF32>(A, lda, W, p, s);
+    case kEpiStoreF32: return run_swap<kEpiStoreF32>(A, lda, W, p, s);
     case kEpiRope: return run_swap<kEpiRope>(A, lda, W, p, s);
     default: return cudaErrorInvalidValue;
   }

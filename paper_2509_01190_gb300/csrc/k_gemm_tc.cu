@@ -1000,7 +1000,7 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
   // most SMs; stream the weights instead
   if (skinny_supported(A, lda, W, epi, p)) return launch_gemm_skinny(A, lda, W, epi, p, s);
   // a few hundred rows: weight band as the 128-row operand, K split over a cluster
-  if (swap_preferred(epi, p.M) && swap_supported(A, lda, W, epi, p))
+  if (swap_preferred(epi, p.M, p.N) && swap_supported(A, lda, W, epi, p))
     return launch_gemm_swap(A, lda, W, epi, p, s);
   const int sms = num_sms();
   const int vn = epi == kEpiSwiGLU ? 2 * p.N : p.N;

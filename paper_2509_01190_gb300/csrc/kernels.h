@@ -121,8 +121,9 @@ cudaError_t launch_gemm_skinny(const void* A, int lda, const TcWeights& W, int e
 constexpr int kSwapMaxM = 1024;
 constexpr int kSwapRowBlock = 256;
 bool swap_supported(const void* A, int lda, const TcWeights& W, int epi, const GemmParams& p);
-// Whether launch_gemm_tc takes the swapped kernel for this epilogue and row count.
-bool swap_preferred(int epi, int M);
+// Whether launch_gemm_tc takes the swapped kernel for this epilogue, row count
+// and output width (wide float32 heads go to the tiled kernel).
+bool swap_preferred(int epi, int M, int N);
 cudaError_t launch_gemm_swap(const void* A, int lda, const TcWeights& W, int epi,
                              const GemmParams& p, cudaStream_t s);
 

@@ -119,3 +119,12 @@ def test_pair_streamk_deterministic(z):
     torch.cuda.synchronize()
     z.zsaa_device_status()
     assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
+
+
+# Very wide float32 outputs (LM heads, N >= 32768) run on the tiled kernel at
+# every row count: one CTA or CTA pairs by waves.  40000 columns end in a
+# partial tile; 17 and 144 rows leave most of a 256-row pair tile empty.
+@pytest.mark.parametrize("M", [17, 144, 300, 600])
+def test_tiled_wide_head_f32(z, M):
+    out, ref, tol = linear_case(z, "store_f32", M, 40000, 256, 500 + M)
+    check_linear(out, ref, tol, "store_f32", f"head M={M}")
