@@ -82,6 +82,10 @@ class OracleConfig:
     prune_point: str = "layer"
     # Eq. 1's mask M: causal (decoder) or none (bidirectional encoder)
     causal: bool = True
+    # arithmetic between the storage points: "f64" (the oracle proper) or
+    # "f32" (a control: the same storage points, float32 sums and products,
+    # to measure how far two correct bf16-storage implementations drift apart)
+    arith: str = "f64"
 
 
 # --------------------------------------------------------------------------
@@ -121,11 +125,20 @@ class _Store:
 # --------------------------------------------------------------------------
 
 
-def rmsnorm(h: np.ndarray, w: np.ndarray, eps: float) -> np.ndarray:
+def _ft(cfg: "OracleConfig"):
+    """numpy type of the arithmetic between storage points (``cfg.arith``)."""
+    if cfg.arith == "f64":
+        return np.float64
+    if cfg.arith == "f32":
+        return np.float32
+    raise ValueError(cfg.arith)
+
+
+def rmsnorm(h: np.ndarray, w: np.ndarray, eps: float, ft=np.float64) -> np.ndarray:
     """Root-mean-square normalisation of each row, scaled by w (pre-norm)."""
-    h = np.asarray(h, dtype=np.float64)
+    h = np.asarray(h, dtype=ft)
     ms = np.mean(h * h, axis=-1, keepdims=True)
-    return h / np.sqrt(ms + eps) * np.asarray(w, dtype=np.float64)
+    return h / np.sqrt(ms + ft(eps)) * np.asarray(w, dtype=ft)
 
 
 def rope_angles(pos: np.ndarray, head_dim: int, theta: float):
@@ -141,8 +154,8 @@ def apply_rope(x: np.ndarray, cos: np.ndarray, sin: np.ndarray) -> np.ndarray:
     half = x.shape[-1] // 2
     x1 = x[..., :half]
     x2 = x[..., half:]
-    c = cos[:, None, :]
-    s = sin[:, None, :]
+    c = cos[:, None, :].astype(x.dtype)
+    s = sin[:, None, :].astype(x.dtype)
     return np.concatenate([x1 * c - x2 * s, x2 * c + x1 * s], axis=-1)
 
 
@@ -350,48 +363,149 @@ def _as64(a) -> np.ndarray:
 
 def attention_block(cfg: OracleConfig, lw: Dict[str, np.ndarray], h: np.ndarray, pos: np.ndarray,
                     store: _Store, key_mask: Optional[np.ndarray] = None,
-                    kv_out: Optional[list] = None):
+                    kv_out: Optional[list] = None, detail: Optional[dict] = None):
     """Pre-norm attention branch of one layer on rows h [n, d].
 
     Returns (new residual h, P [H, n, n], v [n, Hkv, hd]).  If ``kv_out`` is a
     list, the layer's stored keys (after RoPE) and values are appended to it.
+    If ``detail`` is a dict, the stored intermediates go into it: ``x``
+    (normed rows), ``q``/``k``/``v``, ``o`` (attention output before the
+    O-projection) and ``h1`` (the residual after the branch).
     """
     n = h.shape[0]
     H, G, hd = cfg.n_heads, cfg.n_kv_heads, cfg.head_dim
-    x = store(rmsnorm(h, lw["attn_norm"], cfg.rms_eps))
+    ft = _ft(cfg)
+
+    def W(name):
+        return np.asarray(lw[name], dtype=ft)
+
+    x = store(rmsnorm(h, lw["attn_norm"], cfg.rms_eps, ft))
+    xf = np.asarray(x, dtype=ft)
     cos, sin = rope_angles(pos, hd, cfg.rope_theta)
-    q = store(apply_rope((x @ _as64(lw["wq"]).T).reshape(n, H, hd), cos, sin))
-    k = store(apply_rope((x @ _as64(lw["wk"]).T).reshape(n, G, hd), cos, sin))
-    v = store((x @ _as64(lw["wv"]).T).reshape(n, G, hd))
+    q = store(apply_rope((xf @ W("wq").T).reshape(n, H, hd), cos, sin))
+    k = store(apply_rope((xf @ W("wk").T).reshape(n, G, hd), cos, sin))
+    v = store((xf @ W("wv").T).reshape(n, G, hd))
     if kv_out is not None:
         kv_out.append((k, v))
     per = H // G
-    P = np.empty((H, n, n))
-    o = np.empty((n, H, hd))
+    P = np.empty((H, n, n), dtype=ft)
+    o = np.empty((n, H, hd), dtype=ft)
     for hh in range(H):
         g = hh // per
-        P[hh] = attention_probs(q[:, hh, :], k[:, g, :], key_mask, cfg.causal)
-        o[:, hh, :] = P[hh] @ v[:, g, :]
+        P[hh] = attention_probs(np.asarray(q[:, hh, :], dtype=ft), np.asarray(k[:, g, :], dtype=ft),
+                               key_mask, cfg.causal)
+        o[:, hh, :] = P[hh] @ np.asarray(v[:, g, :], dtype=ft)
     o = store(o.reshape(n, H * hd))
-    h = store(h + o @ _as64(lw["wo"]).T)
-    return h, P, v
+    h1 = store(np.asarray(h, dtype=ft) + np.asarray(o, dtype=ft) @ W("wo").T)
+    if detail is not None:
+        detail.update(x=x, q=q, k=k, v=v, o=o, h1=h1)
+    return h1, P, v
 
 
-def mlp_block(cfg: OracleConfig, lw: Dict[str, np.ndarray], h: np.ndarray, store: _Store) -> np.ndarray:
-    """Pre-norm SwiGLU branch: h + (silu(x Wg^T) * (x Wu^T)) Wd^T."""
-    x = store(rmsnorm(h, lw["mlp_norm"], cfg.rms_eps))
-    a = store(silu(x @ _as64(lw["wg"]).T) * (x @ _as64(lw["wu"]).T))
-    return store(h + a @ _as64(lw["wd"]).T)
+def mlp_block(cfg: OracleConfig, lw: Dict[str, np.ndarray], h: np.ndarray, store: _Store,
+              detail: Optional[dict] = None) -> np.ndarray:
+    """Pre-norm SwiGLU branch: h + (silu(x Wg^T) * (x Wu^T)) Wd^T.
+
+    If ``detail`` is a dict, ``x2`` (normed rows), ``a`` (the SwiGLU product)
+    and ``h2`` (the residual after the branch) go into it."""
+    ft = _ft(cfg)
+    x = store(rmsnorm(h, lw["mlp_norm"], cfg.rms_eps, ft))
+    xf = np.asarray(x, dtype=ft)
+    a = store(silu(xf @ np.asarray(lw["wg"], ft).T) * (xf @ np.asarray(lw["wu"], ft).T))
+    h2 = store(np.asarray(h, dtype=ft) + np.asarray(a, dtype=ft) @ np.asarray(lw["wd"], ft).T)
+    if detail is not None:
+        detail.update(x2=x, a=a, h2=h2)
+    return h2
 
 
 def head(cfg: OracleConfig, weights, h: np.ndarray, store: _Store) -> np.ndarray:
     """Final RMSNorm, then the LM head on every kept row, or the d x n_classes
     classifier on the last kept row (last-position pooling)."""
-    x = store(rmsnorm(h, weights["final_norm"], cfg.rms_eps))
-    W = _as64(weights["head"])
+    ft = _ft(cfg)
+    x = np.asarray(store(rmsnorm(h, weights["final_norm"], cfg.rms_eps, ft)), dtype=ft)
+    W = np.asarray(weights["head"], dtype=ft)
     if cfg.n_classes > 0:
-        return x[-1] @ W.T
-    return x @ W.T
+        return np.asarray(x[-1] @ W.T, dtype=np.float64)
+    return np.asarray(x @ W.T, dtype=np.float64)
+
+
+def decoder_layer(cfg: OracleConfig, lw: Dict[str, np.ndarray], layer: int, h: np.ndarray,
+                  pos: np.ndarray, k_keep: int, store: _Store, forced: Optional[np.ndarray] = None,
+                  kv_out: Optional[list] = None, detail: Optional[dict] = None):
+    """One pre-norm decoder layer (Appendix A) on rows h [n, d] at original
+    positions pos, with the Sec. 3.3 elimination when ``layer`` is a pruning
+    layer: every row is scored (R1), the top ``k_keep`` are kept (ties by
+    lower index, the last row forced when ``cfg.force_keep_last``) unless
+    ``forced`` gives the kept indices, and the kept rows are compacted in
+    order.  ``cfg.prune_point`` places the compaction after the MLP ("layer",
+    R3) or between attention and MLP ("attention"); the kept rows come out
+    the same either way.
+
+    Returns (h, pos, idx, scores); idx and scores are None if the layer does
+    not prune.  ``detail`` collects the blocks' intermediates (see
+    ``attention_block`` / ``mlp_block``; the MLP's are on the rows it ran on).
+    """
+    if cfg.prune_point not in ("layer", "attention"):
+        raise ValueError(cfg.prune_point)
+    h, P, v = attention_block(cfg, lw, h, pos, store, kv_out=kv_out, detail=detail)
+    if cfg.prune_point == "layer":
+        h = mlp_block(cfg, lw, h, store, detail=detail)
+    idx = s = None
+    if layer in set(cfg.prune_layers):
+        C = column_mass(P, cfg.n_kv_heads)
+        s = position_scores(C, v, cfg.score_mode)
+        if forced is not None:
+            idx = np.asarray(forced, dtype=np.int64)
+        elif k_keep == h.shape[0]:
+            idx = np.arange(h.shape[0])
+        else:
+            idx = select_topk(s, k_keep, cfg.force_keep_last)
+        h = h[idx]
+        pos = pos[idx]
+    if cfg.prune_point == "attention":
+        h = mlp_block(cfg, lw, h, store, detail=detail)
+    return h, pos, idx, s
+
+
+def layer_rows(cfg: OracleConfig, lw: Dict[str, np.ndarray], h: np.ndarray, pos: np.ndarray,
+               rows: Sequence[int], detail: Optional[dict] = None) -> np.ndarray:
+    """Outputs of a layer that does not prune, for the listed rows only.
+
+    Row i of a layer's output depends on row i and, through Eq. 1, on the keys
+    and values of the rows it may attend to (rows 0..i for the causal mask,
+    every row otherwise), so every row's key and value is computed and the
+    attention, O-projection and MLP run for the listed query rows alone.
+    Returns h_out [len(rows), d]; ``detail`` as ``attention_block`` /
+    ``mlp_block``, for the listed rows.
+    """
+    rows = np.asarray(rows, dtype=np.int64)
+    n = h.shape[0]
+    H, G, hd = cfg.n_heads, cfg.n_kv_heads, cfg.head_dim
+    ft = _ft(cfg)
+    store = _Store(cfg.dtype)
+
+    def W(name):
+        return np.asarray(lw[name], dtype=ft)
+
+    x = store(rmsnorm(h, lw["attn_norm"], cfg.rms_eps, ft)).astype(ft)
+    cos, sin = rope_angles(pos, hd, cfg.rope_theta)
+    k = store(apply_rope((x @ W("wk").T).reshape(n, G, hd), cos, sin))
+    v = store((x @ W("wv").T).reshape(n, G, hd))
+    q = store(apply_rope((x[rows] @ W("wq").T).reshape(len(rows), H, hd), cos[rows], sin[rows]))
+    per = H // G
+    o = np.empty((len(rows), H, hd), dtype=ft)
+    for r, i in enumerate(rows):
+        nk = i + 1 if cfg.causal else n
+        for hh in range(H):
+            g = hh // per
+            logits = (k[:nk, g, :].astype(ft) @ q[r, hh].astype(ft)) / math.sqrt(hd)
+            e = np.exp(logits - np.max(logits))
+            o[r, hh] = (e / np.sum(e)) @ v[:nk, g, :].astype(ft)
+    o = store(o.reshape(len(rows), H * hd))
+    h1 = store(np.asarray(h[rows], dtype=ft) + o.astype(ft) @ W("wo").T)
+    if detail is not None:
+        detail.update(x=store(x[rows]), q=q, k=k[rows], v=v[rows], o=o, h1=h1)
+    return mlp_block(cfg, lw, h1, store, detail=detail)
 
 
 def forward(cfg: OracleConfig, weights, tokens: np.ndarray, accel: Optional[float] = None,
@@ -436,29 +550,15 @@ def forward(cfg: OracleConfig, weights, tokens: np.ndarray, accel: Optional[floa
             if collect:
                 inputs_all.setdefault(layer, []).append((h, pos))
             kv: list = []
-            h, P, v = attention_block(cfg, lw, h, pos, store, kv_out=kv)
+            fi = forced_idx[layer][b] if forced_idx is not None and layer in forced_idx else None
+            h, pos_new, idx, s = decoder_layer(cfg, lw, layer, h, pos, sched[layer], store, forced=fi,
+                                               kv_out=kv)
             if collect_cache:
                 cache_all.setdefault(layer, []).append((kv[0][0], kv[0][1], pos))
-            if cfg.prune_point not in ("layer", "attention"):
-                raise ValueError(cfg.prune_point)
-            if cfg.prune_point == "layer":
-                h = mlp_block(cfg, lw, h, store)
-            k_keep = sched[layer]
-            if layer in set(cfg.prune_layers):
-                C = column_mass(P, cfg.n_kv_heads)
-                s = position_scores(C, v, cfg.score_mode)
-                if forced_idx is not None and layer in forced_idx:
-                    idx = np.asarray(forced_idx[layer][b], dtype=np.int64)
-                elif k_keep == h.shape[0]:
-                    idx = np.arange(h.shape[0])
-                else:
-                    idx = select_topk(s, k_keep, cfg.force_keep_last)
+            pos = pos_new
+            if idx is not None:
                 idx_all.setdefault(layer, []).append(idx)
                 scores_all.setdefault(layer, []).append(s)
-                h = h[idx]
-                pos = pos[idx]
-            if cfg.prune_point == "attention":
-                h = mlp_block(cfg, lw, h, store)
         logits.append(head(cfg, weights, h, store))
         kept_pos.append(pos)
         finals.append(h)

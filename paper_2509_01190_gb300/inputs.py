@@ -151,3 +151,15 @@ def make_hidden(B: int, L: int, d: int, seed: int = MICROBENCH_SEED, device="cpu
     z = torch.randn(B, L, 1, generator=g, device=device, dtype=torch.float32)
     x = torch.randn(B, L, d, generator=g, device=device, dtype=torch.float32)
     return (x * torch.exp(z)).to(dtype)
+
+
+def make_positions(B: int, N: int, L: int, seed: int) -> np.ndarray:
+    """Original positions [B, N] int32 of N rows kept out of L, as a compaction
+    leaves them: per sequence a sorted uniform sample of [0, L) without
+    repeats that always holds the last position L - 1."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    out = np.empty((B, N), dtype=np.int32)
+    for b in range(B):
+        rest = rng.choice(L - 1, size=N - 1, replace=False) if N > 1 else np.zeros(0, np.int64)
+        out[b] = np.sort(np.append(rest, L - 1))
+    return out

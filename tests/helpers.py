@@ -115,3 +115,73 @@ def check_linear(out, ref, tol, epi, what):
     else:
         assert np.all(bf16_ulp_close(got, ref, 2, tol)), what
         assert np.mean(bf16_ulp_close(got, ref, 1)) > 0.995, what
+
+
+def bf16_ulp(x):
+    """One bf16 unit in the last place of each |x| (2^-133 at zero)."""
+    mag = np.abs(np.asarray(x, np.float64))
+    return np.where(mag > 0, 2.0 ** (np.floor(np.log2(np.maximum(mag, 1e-38))) - 7), 2.0 ** -133)
+
+
+def layer_noise_scale(det, lw):
+    """Rounding-noise scale of each element of a decoder layer's output rows.
+
+    A bf16-storage layer computed with float32 sums differs from the float64
+    oracle only through 1-ulp flips at its storage points, which propagate
+    through the next product.  For the output h2 = round(h1 + a Wd^T) with
+    h1 = round(h + o Wo^T) (from identical inputs h), each flip of o or a moves
+    an output by one ulp times its weight, with an arbitrary sign, so the
+    scale of the difference is
+        sigma^2 = ulp(h2)^2 + ulp(h1)^2 + ulp(o)^2 (Wo^2)^T + ulp(a)^2 (Wd^2)^T
+    per element (the upstream flips of x, q, k, v and x2 surface as flips of
+    o and a).  ``det`` holds the oracle's o, h1, a, h2 for the compared rows."""
+    wo = np.asarray(lw["wo"], np.float64)
+    wd = np.asarray(lw["wd"], np.float64)
+    s2 = bf16_ulp(det["h2"]) ** 2 + bf16_ulp(det["h1"]) ** 2
+    s2 = s2 + (bf16_ulp(det["o"]) ** 2) @ (wo * wo).T + (bf16_ulp(det["a"]) ** 2) @ (wd * wd).T
+    return np.sqrt(s2)
+
+
+def layer_error_stats(got, ref, sigma):
+    """Per-element comparison of layer outputs: z = |got - ref| / sigma, and
+    the fractions of elements within 0, 1 and 2 bf16 ulps."""
+    got = np.asarray(got, np.float64)
+    ref = np.asarray(ref, np.float64)
+    err = np.abs(got - ref)
+    z = err / sigma
+    ulp = bf16_ulp(np.maximum(np.abs(got), np.abs(ref)))
+    return dict(z_max=float(z.max()), z_mean=float(z.mean()), exact=float(np.mean(err == 0)),
+                ulp1=float(np.mean(err <= ulp)), ulp2=float(np.mean(err <= 2 * ulp)),
+                rel_mean=float(err.mean() / max(np.abs(ref).mean(), 1e-30)), n=int(err.size))
+
+
+def oracle_pruning_layer_at(cfg, lw, h, pos, ks, rows_for_k, store):
+    """decoder_layer with the compaction between attention and MLP, for
+    several kept counts at once: the attention branch and the scores (Sec. 3.2,
+    R1) do not depend on k, the top-k (Sec. 3.3) and the compaction do, and the
+    MLP acts on each kept row alone, so it runs for the kept rows
+    ``rows_for_k(k, idx)`` (indices into the kept set) only.
+
+    Returns (scores [n], {k: (idx [k], rows, h_out [len(rows), d], det)}) where
+    det holds o, h1, a, h2 of those rows (``layer_noise_scale``)."""
+    det = {}
+    h1, P, v = O.attention_block(cfg, lw, h, pos, store, detail=det)
+    s = O.position_scores(O.column_mass(P, cfg.n_kv_heads), v, cfg.score_mode)
+    del P
+    out = {}
+    for k in ks:
+        idx = np.arange(h.shape[0]) if k == h.shape[0] else O.select_topk(s, k, cfg.force_keep_last)
+        rows = np.asarray(rows_for_k(k, idx), dtype=np.int64)
+        sel = idx[rows]
+        dm = {}
+        h2 = O.mlp_block(cfg, lw, h1[sel], store, detail=dm)
+        out[k] = (idx, rows, h2, dict(o=det["o"][sel], h1=h1[sel], a=dm["a"], h2=h2))
+    return s, out
+
+
+def sample_rows(n, count, seed):
+    """``count`` distinct row indices of [0, n), always with the last one, sorted."""
+    if n <= count:
+        return np.arange(n)
+    rng = np.random.default_rng(seed)
+    return np.sort(np.append(rng.choice(n - 1, count - 1, replace=False), n - 1))

@@ -3,6 +3,7 @@ itself (a library routine, a closed form, an invariant, brute force or a
 hand-worked example from the paper), so that a dropped term, a wrong sign or
 index, or a transposed operand fails at least one test."""
 
+import dataclasses
 import itertools
 import math
 import os
@@ -602,3 +603,98 @@ def test_forward_varlen_runs_each_sequence_at_the_batch_rate():
         np.testing.assert_array_equal(out["logits"][b], r["logits"][0])
         np.testing.assert_array_equal(out["kept_pos"][b], r["kept_pos"][0])
         assert out["kept_pos"][b][-1] == len(t) - 1
+
+
+# ---------------------------------------------------------------- sampled rows, per-layer entry, f32 control
+
+@pytest.mark.parametrize("causal", [True, False])
+def test_layer_rows_matches_torch_composition(causal):
+    # A one-layer model: the head applied to layer_rows' outputs for a few rows
+    # must equal those rows' logits from the torch-composed decoder.
+    cfg = _cfg(n_layers=1, prune_layers=[], causal=causal)
+    w = _tiny_weights(cfg, seed=21)
+    tokens = np.random.default_rng(22).integers(0, cfg.vocab, (1, 17))
+    ref = _torch_forward_unpruned(cfg, w, tokens, all_rows=True)[0]
+    rows = [0, 5, 11, 16]
+    h0 = w["embed"][tokens[0]]
+    out = O.layer_rows(cfg, w["layers"][0], h0, np.arange(17), rows)
+    got = O.head(cfg, w, out, O._Store("f32"))
+    np.testing.assert_allclose(got, ref[rows], rtol=1e-9, atol=1e-9)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_layer_rows_equals_rows_of_the_full_layer(dtype):
+    # At original positions that skip (as after a compaction), sampled rows of a
+    # non-pruning layer equal the same rows of decoder_layer's full output.
+    cfg = _cfg(dtype=dtype, prune_layers=[], n_layers=1)
+    w = _tiny_weights(cfg, seed=23)
+    rng = np.random.default_rng(24)
+    h = O.bf16_round(rng.standard_normal((29, cfg.d_model)))
+    pos = np.sort(rng.choice(200, 29, replace=False))
+    full, pos_out, idx, s = O.decoder_layer(cfg, w["layers"][0], 1, h, pos, 29, O._Store(dtype))
+    assert idx is None and s is None and np.array_equal(pos_out, pos)
+    rows = [0, 3, 28, 14]
+    det = {}
+    got = O.layer_rows(cfg, w["layers"][0], h, pos, rows, detail=det)
+    if dtype == "f32":
+        np.testing.assert_allclose(got, full[rows], rtol=1e-12, atol=1e-12)
+    else:  # a different matmul shape may flip a rare bf16 rounding
+        assert np.mean(got == full[rows]) > 0.99
+        assert np.max(np.abs(got - full[rows])) <= 2.0 ** -7 * np.max(np.abs(full[rows]))
+    assert np.array_equal(det["h2"], got) and det["a"].shape == (4, cfg.ffn_dim)
+
+
+def test_decoder_layer_is_the_forward_step():
+    # forward() is decoder_layer applied layer by layer: running the layers by
+    # hand from the embedded rows reproduces its logits, indices and scores.
+    cfg = _cfg(dtype="bf16")
+    w = _tiny_weights(cfg, seed=25)
+    tokens = np.random.default_rng(26).integers(0, cfg.vocab, (1, 31))
+    ref = O.forward(cfg, w, tokens, alpha=0.6)
+    store = O._Store("bf16")
+    h, pos = store(w["embed"][tokens[0]]), np.arange(31)
+    for layer in range(1, cfg.n_layers + 1):
+        h, pos, idx, s = O.decoder_layer(cfg, w["layers"][layer - 1], layer, h, pos, ref["schedule"][layer], store)
+        if layer in cfg.prune_layers:
+            np.testing.assert_array_equal(idx, ref["idx"][layer][0])
+            np.testing.assert_array_equal(s, ref["scores"][layer][0])
+    np.testing.assert_array_equal(O.head(cfg, w, h, store), ref["logits"][0])
+    np.testing.assert_array_equal(pos, ref["kept_pos"][0])
+
+
+def test_f32_arithmetic_control_drifts_within_the_format_floor():
+    # The control keeps every bf16 storage point and sums in float32: it must
+    # really compute in float32 (it differs from the float64 oracle), stay close
+    # to it (a few bf16 ulps per layer), and pick the same rows where forced.
+    cfg = _cfg(dtype="bf16", n_layers=4, d_model=128, n_heads=4, n_kv_heads=2, head_dim=32,
+               ffn_dim=256, vocab=300)
+    w = _tiny_weights(cfg, seed=27, scale=0.1)
+    tokens = np.random.default_rng(28).integers(0, cfg.vocab, (2, 40))
+    ref = O.forward(cfg, w, tokens, alpha=0.7)
+    ctl = O.forward(dataclasses.replace(cfg, arith="f32"), w, tokens, alpha=0.7, forced_idx=ref["idx"])
+    np.testing.assert_array_equal(ctl["kept_pos"], ref["kept_pos"])
+    gap = np.abs(ctl["logits"] - ref["logits"])
+    assert gap.max() > 0
+    assert gap.mean() <= 2.0 ** -7 * np.sqrt(cfg.n_layers) * ref["logits"].std()
+    with pytest.raises(ValueError):
+        O.forward(dataclasses.replace(cfg, arith="f16"), w, tokens, alpha=0.7)
+
+
+def test_pruning_layer_at_several_k_equals_decoder_layer():
+    # The full-size tests run one attention branch for several kept counts and
+    # the MLP on sampled kept rows; that must be decoder_layer's result.
+    from tests.helpers import oracle_pruning_layer_at
+    cfg = _cfg(dtype="bf16", prune_point="attention")
+    w = _tiny_weights(cfg, seed=29, scale=0.2)
+    rng = np.random.default_rng(30)
+    h = O.bf16_round(rng.standard_normal((37, cfg.d_model)))
+    pos = np.sort(rng.choice(90, 37, replace=False))
+    store = O._Store("bf16")
+    s, per_k = oracle_pruning_layer_at(cfg, w["layers"][0], h, pos, [37, 20, 7],
+                                       lambda k, idx: np.arange(0, k, 2), store)
+    for k, (idx, rows, h2, det) in per_k.items():
+        ref, pref, iref, sref = O.decoder_layer(cfg, w["layers"][0], 1, h, pos, k, store)
+        np.testing.assert_array_equal(idx, iref)
+        np.testing.assert_array_equal(s, sref)
+        np.testing.assert_array_equal(h2, ref[rows])
+        np.testing.assert_array_equal(det["h2"], h2)
