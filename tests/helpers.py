@@ -155,22 +155,28 @@ def layer_error_stats(got, ref, sigma):
                 rel_mean=float(err.mean() / max(np.abs(ref).mean(), 1e-30)), n=int(err.size))
 
 
-def oracle_pruning_layer_at(cfg, lw, h, pos, ks, rows_for_k, store):
+def oracle_pruning_layer_at(cfg, lw, h, pos, ks, rows_for_k, store, forced=None):
     """decoder_layer with the compaction between attention and MLP, for
     several kept counts at once: the attention branch and the scores (Sec. 3.2,
     R1) do not depend on k, the top-k (Sec. 3.3) and the compaction do, and the
     MLP acts on each kept row alone, so it runs for the kept rows
     ``rows_for_k(k, idx)`` (indices into the kept set) only.
 
-    Returns (scores [n], {k: (idx [k], rows, h_out [len(rows), d], det)}) where
-    det holds o, h1, a, h2 of those rows (``layer_noise_scale``)."""
+    ``forced`` ({k: idx}) replaces the top-k choice (the scores are still
+    computed).  Returns (scores [n], {k: (idx [k], rows, h_out [len(rows), d],
+    det)}) where det holds o, h1, a, h2 of those rows (``layer_noise_scale``)."""
     det = {}
     h1, P, v = O.attention_block(cfg, lw, h, pos, store, detail=det)
     s = O.position_scores(O.column_mass(P, cfg.n_kv_heads), v, cfg.score_mode)
     del P
     out = {}
     for k in ks:
-        idx = np.arange(h.shape[0]) if k == h.shape[0] else O.select_topk(s, k, cfg.force_keep_last)
+        if forced is not None and k in forced:
+            idx = np.asarray(forced[k], dtype=np.int64)
+        elif k == h.shape[0]:
+            idx = np.arange(h.shape[0])
+        else:
+            idx = O.select_topk(s, k, cfg.force_keep_last)
         rows = np.asarray(rows_for_k(k, idx), dtype=np.int64)
         sel = idx[rows]
         dm = {}
