@@ -201,6 +201,23 @@ zsaa_status zsaa_forward_masked(zsaa_model* m, const int32_t* token_ids, int B, 
                                 float* logits_out, int32_t* kept_pos_out,
                                 const zsaa_forward_opts* opts, zsaa_stream stream);
 
+/* zsaa_forward_marked: Appendix B's figure, where a row marked as pruned can
+ * be reactivated at a later layer.  Reading: a row hidden as a key receives no
+ * soft-score (Eq. 1) and so could never come back, so this mode hides and
+ * removes nothing.  Every layer runs on all B*L rows exactly as the unpruned
+ * forward does; each pruning layer marks as preserved the top N_l of ALL L
+ * rows of each sequence by that layer's scores (Sec. 3.3 ranking, ties to the
+ * lower position, the last position kept; N_l from the Eq. 2 schedule of
+ * zsaa_plan), whatever the earlier marks.  Outputs: the logits of the rows
+ * preserved at the last pruning layer (the unpruned forward's logits at those
+ * positions) and their positions, laid out as zsaa_forward's.  opts as
+ * zsaa_forward_masked (POSITIONS [B, N_l] and scores [B, L] per pruning layer).
+ * Same limits as zsaa_forward_masked; the cost is that of the unpruned
+ * forward plus the scoring of every pruning layer. */
+zsaa_status zsaa_forward_marked(zsaa_model* m, const int32_t* token_ids, int B, int L, double accel,
+                                float* logits_out, int32_t* kept_pos_out,
+                                const zsaa_forward_opts* opts, zsaa_stream stream);
+
 /* ---- Variable-length batches.
  *
  * Sec. 3.4 picks the preservation rate per inference call.  For one call over
@@ -321,7 +338,10 @@ zsaa_status zsaa_score_select_ex(const void* hidden, int B, int L, int d, int dt
  *   Arguments, layouts and results are those of zsaa_score_select.
  *   B*L above 1,048,576 is rejected with ZSAA_ERR_INVALID_ARG before any work.
  *   The first call on a device looks up the array's device address with that
- *   device current; make that first call before any stream capture.
+ *   device current; make that first call before any stream capture.  The
+ *   address is kept per device together with the id of the context it was
+ *   found in; after a reset of that device's context (cudaDeviceReset) the
+ *   next call looks it up again, so call once more outside capture then.
  *   All calls share the one array: calls whose work can overlap on the GPU
  *   (different streams, or different host threads) race on it and must be
  *   ordered by the caller. */

@@ -22,6 +22,8 @@ Every function follows one passage of the paper:
   with the Sec. 3.3 elimination applied after each pruning layer.
 * ``forward_masked`` -- Appendix B: the "marked as pruned but not removed"
   formulation, an independent second route to the same kept-row outputs.
+* ``forward_marked`` -- Appendix B's figure, where marked rows may be
+  reactivated at a later layer (reading R18: nothing is removed or hidden).
 * ``decode_step`` / ``generate`` -- Sec. 3.3 carried into generation: a row
   eliminated before layer l is absent from layer l, so a generated token
   attends, in layer l, to the keys and values of the rows that layer kept.
@@ -622,6 +624,54 @@ def forward_masked(cfg: OracleConfig, weights, tokens: np.ndarray, sched: Sequen
         "logits": np.stack(logits),
         "kept_pos": np.stack(kept_pos),
         "kept_by_layer": {k: np.stack(v) for k, v in kept_by_layer.items()},
+    }
+
+
+def forward_marked(cfg: OracleConfig, weights, tokens: np.ndarray, sched: Sequence[int]):
+    """Appendix B's figure: every hidden activation stays, including those
+    marked as pruned, and a row marked at one layer can be reactivated at a
+    later one.
+
+    Reading (R18): a row hidden as a key receives soft-score zero in every
+    later layer (Eq. 1 gives it no probability), so under the R1 score it
+    could never come back; reactivation needs the marked rows to stay in the
+    computation.  So nothing is removed or hidden: every layer runs on all L
+    rows as the unpruned decoder does, and each pruning layer marks as
+    preserved the top N_l of ALL L rows by that layer's scores (R1, ties and
+    the forced last row as ``select_topk``), whatever the earlier marks.  The
+    output is the logits of the rows preserved at the last pruning layer,
+    i.e. the unpruned forward's logits at those positions.
+
+    Returns ``logits``, ``kept_pos`` [B, N_n], and per pruning layer
+    ``kept_by_layer`` [B, N_l] and ``scores`` [B, L].
+    """
+    tokens = np.asarray(tokens)
+    B, L = tokens.shape
+    store = _Store(cfg.dtype)
+    emb = _as64(weights["embed"])
+    G = cfg.n_kv_heads
+    logits, kept_pos, kept_by_layer, scores_by_layer = [], [], {}, {}
+    for b in range(B):
+        h = store(emb[tokens[b]])
+        pos = np.arange(L)
+        keep = pos
+        for layer in range(1, cfg.n_layers + 1):
+            lw = weights["layers"][layer - 1]
+            h, P, v = attention_block(cfg, lw, h, pos, store)
+            if layer in set(cfg.prune_layers):
+                s = position_scores(column_mass(P, G), v, cfg.score_mode)
+                k_keep = sched[layer]
+                keep = select_topk(s, k_keep, cfg.force_keep_last) if k_keep < L else np.arange(L)
+                kept_by_layer.setdefault(layer, []).append(keep)
+                scores_by_layer.setdefault(layer, []).append(s)
+            h = mlp_block(cfg, lw, h, store)
+        logits.append(head(cfg, weights, h[keep], store))
+        kept_pos.append(keep)
+    return {
+        "logits": np.stack(logits),
+        "kept_pos": np.stack(kept_pos),
+        "kept_by_layer": {k: np.stack(v) for k, v in kept_by_layer.items()},
+        "scores": {k: np.stack(v) for k, v in scores_by_layer.items()},
     }
 
 

@@ -616,7 +616,9 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
     {
       const double pairs = static_cast<double>(B) * Hq * n_pairs(N);
       TRACE("attention", 4.0 * pairs * hd, Md * (m->ld_qkv + m->dq) * es + static_cast<double>(B) * Hq * N * 4.0);
-      if (attention_tc_supported(dt, hd, nullptr, nullptr, m->status, m->vt) && attention_tc_preferred(N)) {
+      if (attention_pp_supported(dt, hd, Hq, Hkv, nullptr, nullptr, m->status)) {
+        ZCK(launch_attention_pp(m->qkv, B, N, Hq, Hkv, hd, m->attn, m->lse, causal, m->status, s));
+      } else if (attention_tc_supported(dt, hd, nullptr, nullptr, m->status, m->vt) && attention_tc_preferred(N)) {
         trace_scope_.kernels = 2;  // V transpose + attention
         ZCK(launch_attention_tc(m->qkv, m->vt, B, N, Hq, Hkv, hd, m->attn, m->lse, causal, m->status, s));
       } else {
@@ -838,9 +840,12 @@ zsaa_status run_forward(zsaa_model* m, const int32_t* tok, int B, int L, double 
 // from the layer after its marking on, its query adds nothing to later column
 // masses, and only unmarked rows compete at a selection.  The kept rows'
 // outputs equal those of the compacted forward; the cost is that of accel 1.
+// With reactivate (Appendix B's figure, reading R18) nothing is hidden: every
+// layer is the unpruned one, and each pruning layer marks the top N_l of all L
+// rows by its own scores, whatever the earlier marks.
 zsaa_status run_forward_masked(zsaa_model* m, const int32_t* tok, int B, int L, double accel,
                                float* logits, int32_t* kept_pos, const zsaa_forward_opts* opts,
-                               cudaStream_t s) {
+                               cudaStream_t s, bool reactivate = false) {
   const zsaa_config& c = m->cfg;
   const int d = c.d_model, hd = c.head_dim, Hq = c.n_heads, Hkv = c.n_kv_heads, n = c.n_layers;
   if (c.dtype != ZSAA_BF16 || d % 8 != 0 || d > kRowsNormMaxD)
@@ -902,7 +907,7 @@ zsaa_status run_forward_masked(zsaa_model* m, const int32_t* tok, int B, int L, 
     {
       TRACE("attention", 4.0 * pairs * hd, Md * (m->ld_qkv + m->dq) * es + static_cast<double>(B) * Hq * L * 4.0);
       ZCK(launch_attention(dt, m->qkv, B, L, Hq, Hkv, hd, m->attn, m->lse, causal, s, nullptr,
-                           m->alive));
+                           reactivate ? nullptr : m->alive));
     }
     // O-projection beside the column mass and selection (see run_forward);
     // the MLP's RMSNorm joins it
@@ -932,24 +937,27 @@ zsaa_status run_forward_masked(zsaa_model* m, const int32_t* tok, int B, int L, 
       const bool want_scores = opts && opts->scores_out;
       const bool forced = opts && opts->forced_idx;
       const bool want_idx = opts && opts->idx_out;
-      if (k < sched[l - 1] || want_scores || want_idx) {
+      if ((reactivate ? k < L : k < sched[l - 1]) || want_scores || want_idx) {
         int n_qc = 1;
         {
           TRACE("colmass", 2.0 * pairs * hd, Md * (m->dq + 2 * m->dkv) * es);
           ZCK(launch_position_parts(dt, m->qkv, m->lse, m->vnorm, B, L, Hq, Hkv, hd, c.score_mode,
-                                    m->colmass, &n_qc, m->status, causal, s, nullptr, 0, m->alive));
+                                    m->colmass, &n_qc, m->status, causal, s, nullptr, 0,
+                                    reactivate ? nullptr : m->alive));
         }
         {
           TRACE("select", 0.0, static_cast<double>(n_qc) * B * Hkv * L * 4.0 + static_cast<double>(B) * k * 4.0);
           ZCK(launch_select_parts(m->colmass, n_qc, B, Hkv, L, k, c.force_keep_last, m->idx,
                                   want_scores ? opts->scores_out + off_scores : nullptr, s, nullptr,
-                                  nullptr, forced ? nullptr : m->alive));
+                                  nullptr, (forced || reactivate) ? nullptr : m->alive));
         }
         kept = m->idx;
         if (forced) {
           kept = opts->forced_idx + off_forced;
-          TRACE("select", 0.0, static_cast<double>(B) * (L + 4.0 * k));
-          ZCK(launch_flags_from_idx(kept, B, L, k, m->alive, m->status, s));
+          if (!reactivate) {  // the marks hide rows from later layers
+            TRACE("select", 0.0, static_cast<double>(B) * (L + 4.0 * k));
+            ZCK(launch_flags_from_idx(kept, B, L, k, m->alive, m->status, s));
+          }
         }
         if (want_idx)
           ZCK(cudaMemcpyAsync(opts->idx_out + off_idx, kept, sizeof(int32_t) * B * k,
@@ -1839,7 +1847,11 @@ zsaa_status zsaa_op_attention_ex(const void* qkv, int B, int N, int Hq, int Hkv,
   if (dtype == ZSAA_F32 && (hd < 1 || hd > 128)) return fail(ZSAA_ERR_UNSUPPORTED, "f32 attention needs hd <= 128");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   int* status = shared_status();
-  if (dtype == ZSAA_BF16 && status != nullptr) {  // the tcgen05 kernel, V^T scratch
+  if (attention_pp_supported(dtype, hd, Hq, Hkv, nullptr, nullptr, status)) {
+    ZCK(launch_attention_pp(qkv, B, N, Hq, Hkv, hd, out, lse, causal ? 1 : 0, status, s));
+    return ZSAA_OK;
+  }
+  if (dtype == ZSAA_BF16 && status != nullptr) {  // the one-tile tcgen05 kernel, V^T scratch
     void* vt = nullptr;
     ZCK(cudaMallocAsync(&vt, attention_tc_vt_elems(B, N, Hkv, hd) * 2, s));
     cudaError_t e = launch_attention_tc(qkv, vt, B, N, Hq, Hkv, hd, out, lse, causal ? 1 : 0, status, s);
@@ -1917,6 +1929,14 @@ zsaa_status zsaa_forward_masked(zsaa_model* m, const int32_t* token_ids, int B, 
   if (m == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null model");
   return run_forward_masked(m, token_ids, B, L, accel, logits_out, kept_pos_out, opts,
                             reinterpret_cast<cudaStream_t>(stream));
+}
+
+zsaa_status zsaa_forward_marked(zsaa_model* m, const int32_t* token_ids, int B, int L, double accel,
+                                float* logits_out, int32_t* kept_pos_out,
+                                const zsaa_forward_opts* opts, zsaa_stream stream) {
+  if (m == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null model");
+  return run_forward_masked(m, token_ids, B, L, accel, logits_out, kept_pos_out, opts,
+                            reinterpret_cast<cudaStream_t>(stream), true);
 }
 
 zsaa_status zsaa_plan_varlen_config(const zsaa_config* cfg, const int32_t* lengths, int B,

@@ -30,7 +30,7 @@ EXPORTED = [
     "zsaa_score_select_noalloc", "zsaa_model_set_graphs", "zsaa_cache_create", "zsaa_cache_destroy",
     "zsaa_prefill", "zsaa_decode_step", "zsaa_cache_layer", "zsaa_cache_bytes",
     "zsaa_op_attention_ex", "zsaa_op_colmass_ex", "zsaa_plan_varlen_config", "zsaa_plan_varlen",
-    "zsaa_forward_varlen", "zsaa_forward_masked", "zsaa_selftest_wait_timeout",
+    "zsaa_forward_varlen", "zsaa_forward_masked", "zsaa_forward_marked", "zsaa_selftest_wait_timeout",
 ]
 
 
@@ -100,6 +100,7 @@ def lib():
             "zsaa_plan_varlen": ([_P, _P, _I, _D, C.POINTER(_I), C.POINTER(_D)], _I),
             "zsaa_forward_varlen": ([_P, _P, _P, _I, _D, _P, _P, C.POINTER(zsaa_forward_opts), _P], _I),
             "zsaa_forward_masked": ([_P, _P, _I, _I, _D, _P, _P, C.POINTER(zsaa_forward_opts), _P], _I),
+            "zsaa_forward_marked": ([_P, _P, _I, _I, _D, _P, _P, C.POINTER(zsaa_forward_opts), _P], _I),
             "zsaa_op_colmass_ex": ([_P, _P, _I, _I, _I, _I, _I, _I, _I, _P, _P], _I),
             "zsaa_sync": ([_P, _P], _I),
             "zsaa_device_status": ([], _I),
@@ -302,6 +303,18 @@ def zsaa_forward_masked(model: Model, token_ids, B: int, L: int, accel: float, l
         opts = C.byref(zsaa_forward_opts(_ptr(forced_pos), _ptr(scores_out), _ptr(idx_out), None,
                                          0, None, None, 0, 0))
     _check(lib().zsaa_forward_masked(model.handle, _ptr(token_ids), B, L, float(accel),
+                                     _ptr(logits_out), _ptr(kept_pos_out), opts, _stream(stream)))
+
+
+def zsaa_forward_marked(model: Model, token_ids, B: int, L: int, accel: float, logits_out,
+                        kept_pos_out=None, forced_pos=None, scores_out=None, idx_out=None,
+                        stream=None):
+    """Appendix B figure mode (marked rows may be reactivated); hooks as zsaa_forward_masked."""
+    opts = None
+    if forced_pos is not None or scores_out is not None or idx_out is not None:
+        opts = C.byref(zsaa_forward_opts(_ptr(forced_pos), _ptr(scores_out), _ptr(idx_out), None,
+                                         0, None, None, 0, 0))
+    _check(lib().zsaa_forward_marked(model.handle, _ptr(token_ids), B, L, float(accel),
                                      _ptr(logits_out), _ptr(kept_pos_out), opts, _stream(stream)))
 
 

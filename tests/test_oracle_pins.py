@@ -698,3 +698,44 @@ def test_pruning_layer_at_several_k_equals_decoder_layer():
         np.testing.assert_array_equal(s, sref)
         np.testing.assert_array_equal(h2, ref[rows])
         np.testing.assert_array_equal(det["h2"], h2)
+
+
+# ---------------------------------------------------------------- Appendix B figure mode (reactivation)
+
+def test_marked_mode_logits_are_the_unpruned_decoders_at_the_kept_rows():
+    cfg = _cfg(prune_layers=[1, 2, 3])
+    w = _tiny_weights(cfg, seed=31)
+    tokens = np.random.default_rng(32).integers(0, cfg.vocab, (2, 33))
+    sched = O.schedule(33, 0.6, cfg.n_layers, cfg.prune_layers, cfg.tau)
+    r = O.forward_marked(cfg, w, tokens, sched)
+    ref = _torch_forward_unpruned(cfg, w, tokens, all_rows=True)
+    for b in range(2):
+        np.testing.assert_allclose(r["logits"][b], ref[b][r["kept_pos"][b]], rtol=1e-9, atol=1e-9)
+    for layer in cfg.prune_layers:
+        marks = r["kept_by_layer"][layer]
+        assert marks.shape == (2, sched[layer])
+        assert np.all(np.diff(marks, axis=1) > 0) and np.all(marks[:, -1] == 32)
+
+
+def test_marked_mode_first_layer_matches_compaction_and_later_layers_reactivate():
+    # The first pruning layer sees every row in both modes, so its marks are
+    # the compacted forward's choice; later layers rank all rows again, and on
+    # random inputs some row marked as pruned comes back.
+    cfg = _cfg(prune_layers=[1, 2, 3], n_layers=4)
+    w = _tiny_weights(cfg, seed=33)
+    tokens = np.random.default_rng(34).integers(0, cfg.vocab, (3, 41))
+    alpha = 0.7
+    sched = O.schedule(41, alpha, cfg.n_layers, cfg.prune_layers, cfg.tau)
+    r = O.forward_marked(cfg, w, tokens, sched)
+    c = O.forward(cfg, w, tokens, alpha=alpha)
+    np.testing.assert_array_equal(r["kept_by_layer"][1], c["idx"][1])
+    np.testing.assert_array_equal(r["scores"][1], c["scores"][1])
+    back = 0
+    for b in range(3):
+        for l in (2, 3):
+            back += len(set(r["kept_by_layer"][l][b]) - set(r["kept_by_layer"][l - 1][b]))
+    assert back > 0
+    # accel 1: nothing is marked, every row's logits are the unpruned ones
+    r1 = O.forward_marked(cfg, w, tokens, [41] * 5)
+    np.testing.assert_allclose(r1["logits"], _torch_forward_unpruned(cfg, w, tokens, all_rows=True),
+                               rtol=1e-9, atol=1e-9)
