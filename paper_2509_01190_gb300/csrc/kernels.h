@@ -132,6 +132,15 @@ cudaError_t launch_gemm_f32(const float* A, int lda, const float* W, const float
                             const GemmParams& p, cudaStream_t s);
 
 // ---- attention (k_attn.cu)
+// Two-tile tcgen05 attention (k_attn_pp.cu) for bf16 heads of 64 or 128 dims,
+// fixed lengths, an even number of query heads per KV head: persistent CTAs
+// walk (sequence, KV group, pair of query heads, 128 queries) items, O kept
+// in TMEM, V read from the qkv rows.  Same outputs as launch_attention;
+// bounded waits report through status.
+bool attention_pp_supported(int dtype, int hd, int Hq, int Hkv, const int* cu, const uint8_t* key_alive,
+                            int* status);
+cudaError_t launch_attention_pp(const void* qkv, int B, int N, int Hq, int Hkv, int hd, void* out, float* lse,
+                                int causal, int* status, cudaStream_t s);
 // tcgen05 attention (k_attn_tc.cu) for bf16 heads of 64 or 128 dims, fixed
 // lengths: a transpose kernel writes V^T into vt (attention_tc_vt_elems bf16
 // elements), then persistent CTAs walk (128 queries, head, sequence) items.

@@ -265,10 +265,16 @@ def _oracle_attention(qkv, B, N, Hq, Hkv, hd, causal=True):
     return np.stack(outs), np.stack(lses), Ps, x
 
 
+# Shapes with an even number of query heads per KV head run the two-tile
+# kernel (k_attn_pp.cu) at every length, the short kept lengths of the deep
+# pruned layers included (18..255 keys); odd ratios run the one-tile kernel.
 @pytest.mark.parametrize("B,N,Hq,Hkv,hd", [(2, 1, 4, 2, 64), (2, 65, 4, 2, 64), (1, 200, 4, 1, 128),
                                            (2, 130, 8, 2, 128), (1, 64, 2, 2, 64), (2, 300, 4, 2, 64),
                                            (1, 517, 8, 2, 64), (1, 1024, 4, 4, 64), (2, 300, 4, 2, 128),
-                                           (1, 517, 8, 2, 128), (1, 1024, 4, 4, 128), (3, 63, 2, 1, 128)])
+                                           (1, 517, 8, 2, 128), (1, 1024, 4, 4, 128), (3, 63, 2, 1, 128),
+                                           (3, 18, 8, 2, 64), (2, 47, 8, 2, 128), (4, 128, 8, 2, 64),
+                                           (2, 129, 8, 2, 128), (2, 255, 8, 2, 64), (1, 2048, 8, 2, 128),
+                                           (1, 700, 16, 2, 64)])
 def test_attention_and_colmass_bf16(z, B, N, Hq, Hkv, hd):
     qkv = _qkv(B, N, Hq, Hkv, hd, 20 + N, torch.bfloat16)
     out = torch.empty(B * N, Hq * hd, device="cuda", dtype=torch.bfloat16)

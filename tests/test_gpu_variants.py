@@ -25,7 +25,7 @@ def z(zlib):
 
 
 @pytest.mark.parametrize("B,N,Hq,Hkv,hd", [(2, 1, 4, 2, 64), (2, 65, 4, 2, 64), (1, 200, 4, 1, 128),
-                                           (2, 130, 8, 2, 128), (1, 300, 4, 2, 64)])
+                                           (2, 130, 8, 2, 128), (1, 300, 4, 2, 64), (1, 600, 8, 2, 128)])
 def test_bidirectional_attention_and_colmass_bf16(z, B, N, Hq, Hkv, hd):
     qkv = _qkv(B, N, Hq, Hkv, hd, 60 + N, torch.bfloat16)
     out = torch.empty(B * N, Hq * hd, device="cuda", dtype=torch.bfloat16)
