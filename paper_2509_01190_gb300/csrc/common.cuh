@@ -9,11 +9,43 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <mutex>
 #include <utility>
 
 #include "../../include/zsaa.h"
 
 namespace zsaa {
+
+// A kernel's dynamic shared-memory limit (cudaFuncSetAttribute) is state of the
+// current device only.  OncePerDevice runs a set-up step once per device,
+// under a lock, and returns that device's result on every later call.
+class OncePerDevice {
+ public:
+  template <typename Fn>
+  cudaError_t run(Fn&& fn) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMax) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(mu_);
+    if (!done_[dev]) {
+      err_[dev] = fn();
+      done_[dev] = true;
+    }
+    return err_[dev];
+  }
+
+ private:
+  static constexpr int kMax = 64;
+  std::mutex mu_;
+  bool done_[kMax] = {};
+  cudaError_t err_[kMax] = {};
+};
+
+template <typename Kern>
+cudaError_t set_smem_limit_once(OncePerDevice& once, Kern kernel, int bytes) {
+  return once.run([&] { return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes); });
+}
 
 typedef __nv_bfloat16 bf16;
 

@@ -488,12 +488,8 @@ cudaError_t run_attention_tc(const void* qkv, void* vt, int B, int N, int Hq, in
     return cudaErrorInvalidValue;
   if (!encode(&tm_vt, vt, static_cast<uint64_t>(ldt), static_cast<uint64_t>(B) * Hkv * HD, ldt, 64, HD))
     return cudaErrorInvalidValue;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [] {
-    attr_err = cudaFuncSetAttribute(attn_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    static_cast<int>(C::SMEM));
-  });
+  static OncePerDevice once;
+  const cudaError_t attr_err = set_smem_limit_once(once, attn_tc_kernel<HD>, static_cast<int>(C::SMEM));
   if (attr_err != cudaSuccess) return attr_err;
   AtArgs a;
   a.lse2 = lse;

@@ -350,12 +350,8 @@ int cm_num_sms() {
 template <int HD>
 cudaError_t run_cm(const CUtensorMap& tm, const CmArgs& a, int sms, cudaStream_t s) {
   using C = CmCfg<HD>;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [] {
-    attr_err = cudaFuncSetAttribute(colmass_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    static_cast<int>(C::SMEM));
-  });
+  static OncePerDevice once;
+  const cudaError_t attr_err = set_smem_limit_once(once, colmass_tc_kernel<HD>, static_cast<int>(C::SMEM));
   // Two CTAs per SM when their shared memory fits (hd 64): they hide each
   // other's epilogue latency (TMEM: 2 x 256 columns; registers: 2 x 320 x 96).
   constexpr int per_sm = 2 * (C::SMEM + 1024) <= 227 * 1024 ? 2 : 1;

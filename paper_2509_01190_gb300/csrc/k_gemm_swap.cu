@@ -467,13 +467,8 @@ size_t smem_bytes(int wsub, int Mp, int stages, int ksub) {
 
 template <int EPI>
 cudaError_t ensure_attr() {
-  static std::once_flag once;
-  static cudaError_t err = cudaSuccess;
-  std::call_once(once, [] {
-    err = cudaFuncSetAttribute(gemm_swap_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               SW_RING_BUDGET + 1024 + 256);
-  });
-  return err;
+  static OncePerDevice once;
+  return set_smem_limit_once(once, gemm_swap_kernel<EPI>, SW_RING_BUDGET + 1024 + 256);
 }
 
 cudaLaunchConfig_t make_cfg(dim3 grid, size_t smem, cudaStream_t s, cudaLaunchAttribute (&attr)[2],

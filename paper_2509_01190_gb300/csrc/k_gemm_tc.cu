@@ -860,13 +860,8 @@ template <int BN, int EPI>
 cudaError_t run_tc(const TcMaps& maps, int n1, int n2, const GemmParams& p, const TileSched& ts,
                    int grid, cudaStream_t s) {
   using C = TcCfg<BN>;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [] {
-    attr_err = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    static_cast<int>(C::SMEM));
-  });
+  static OncePerDevice once;
+  const cudaError_t attr_err = set_smem_limit_once(once, gemm_tc_kernel<BN, EPI>, static_cast<int>(C::SMEM));
   if (attr_err != cudaSuccess) return attr_err;
   ZSAA_LAUNCH(gemm_tc_kernel<BN, EPI>, dim3(grid), dim3(kThreads), C::SMEM, s, maps, n1, n2, p, ts);
   if (p.launches) *p.launches += 1;
@@ -888,13 +883,8 @@ cudaError_t dispatch_epi(int epi, const TcMaps& maps, int n1, int n2, const Gemm
 
 template <int EPI>
 cudaError_t pair_attr() {
-  static std::once_flag once;
-  static cudaError_t err = cudaSuccess;
-  std::call_once(once, [] {
-    err = cudaFuncSetAttribute(gemm_pair_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               static_cast<int>(P_SMEM));
-  });
-  return err;
+  static OncePerDevice once;
+  return set_smem_limit_once(once, gemm_pair_kernel<EPI>, static_cast<int>(P_SMEM));
 }
 
 cudaLaunchConfig_t pair_cfg(int pairs, cudaStream_t s, cudaLaunchAttribute (&attr)[2]) {

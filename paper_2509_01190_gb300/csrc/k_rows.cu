@@ -581,9 +581,9 @@ cudaError_t launch_select_parts(const float* parts, int n_qc, int B, int G, int 
                                 int force_last, int32_t* idx, float* scores_out, cudaStream_t s,
                                 const int* cu_in, const int* cu_out, uint8_t* alive) {
   const size_t smem = static_cast<size_t>(N) * sizeof(float);
-  static cudaError_t attr = cudaFuncSetAttribute(select_topk_kernel<true>,
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 static_cast<int>(kSelectPartsMaxN * sizeof(float)));
+  static OncePerDevice once;
+  const cudaError_t attr = set_smem_limit_once(once, select_topk_kernel<true>,
+                                               static_cast<int>(kSelectPartsMaxN * sizeof(float)));
   if (attr != cudaSuccess) return attr;
   ZSAA_LAUNCH(select_topk_kernel<true>, dim3(B), dim3(kSelThreads), smem, s,
               static_cast<const float*>(nullptr), N, k, force_last, idx, parts, n_qc, B, G, scores_out,
