@@ -1,24 +1,29 @@
 #!/usr/bin/env python
 """Benchmark of the pruned prefill (Zero-Shot Adjustable Acceleration) on GB300.
 
-Default workload: the Llama-3.2-1B-shaped decoder (16 layers, d=2048, 32/8
-heads, SwiGLU 8192, vocab 128256), bf16, random-init N(0, 0.02) weights,
-batch 8 x 512 uniform random tokens.  One step = one pruned prefill of the
-whole batch at the headline acceleration factor (--accel, default 4), i.e.
-every row of the path: plan, embed, per layer RMSNorm / QKV+RoPE / attention /
-O+residual / RMSNorm / SwiGLU MLP + residual / column mass / score / top-k /
-gather, then the LM head on the kept rows.
+Headline workload: the Llama-3-8B-shaped decoder (32 layers, d=4096, 32/8
+heads of 128, SwiGLU 14336, vocab 128256), bf16, random-init N(0, 0.02)
+weights, batch 4 x 2048 uniform random tokens -- the largest of the model
+workloads, and one GPU holds it.  One step = one pruned prefill of the whole
+batch at the headline acceleration factor (--accel, default 4): every row of
+the path (plan, embed, per layer RMSNorm / QKV+RoPE / attention / O+residual
+/ column mass / score / top-k / gather + RMSNorm / SwiGLU MLP + residual,
+then the LM head on the kept rows).
 
 Prints ONE JSON line (rank 0).  value = prefill tokens/s (B*L input tokens per
 forward, all ranks) timed with CUDA events on the launch stream, L2 flushed
-(256 MiB write) between timed steps.  Extra keys: the accel sweep (tokens/s,
-speedup over the same library's unpruned forward, modelled FLOP reduction),
-the roofline of the dominant kernel from the library's per-kernel trace, an
-end-to-end number through zsaa_forward_host with pinned host buffers, the CPU
-oracle timed on the host cores, and SM clocks sampled during the timed region.
+(256 MiB write) between timed steps.  The other keys: the roofline of the
+dominant kernel class and every GEMM class against its own bound (from the
+library's per-kernel trace), the end-to-end rate through zsaa_forward_host
+with pinned host buffers, the CPU oracle on the host cores, SM clocks during
+the timed region, and (last on the line, short) the accel sweep with the
+speedup over the same library's unpruned forward, the isolated
+score/select/gather microbench and the sweeps of the 1B workloads.
 
---impl reference times the CPU oracle (the reference arm for this build) on
-a bounded sample of the same workload: one sequence per step.
+--impl reference times the CPU oracle (the reference arm for this build) on a
+bounded sample of the same workload: the oracle's forward of the first
+sequence, one decoder layer per step (the head with the last layer), rated by
+the modelled FLOPs of the layers it ran.
 Multi-GPU (torchrun): every rank runs its own batch (sequences are
 independent; no collective on the data path), value = all ranks' tokens /
 max over ranks of the timed span.
@@ -27,6 +32,8 @@ max over ranks of the timed span.
 from __future__ import annotations
 
 import argparse
+
+import numpy as np
 import json
 import os
 import statistics
@@ -42,36 +49,27 @@ if ROOT not in sys.path:
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
-# DRAM bytes per launch of the dominant kernel class (gate/up + SwiGLU GEMM) in
-# this forward, from one ncu capture (profiles/gemm_gate_up_swiglu_1b_traffic.md):
-# the mean of dram__bytes_read.sum + dram__bytes_write.sum over the 16 launches
-# of one forward.  Reported only while the sources it was measured on are
-# unchanged (sha256 below), else null.
-GATE_UP_TRAFFIC = {
-    "bytes_per_launch": 74144992.0,
-    "sources": {
-        "paper_2509_01190_gb300/csrc/k_gemm_tc.cu": "77030fcb2467843a49afe1b6d32dddd3516d4f09df67e73fc6de0bf40fb44fda",
-        "paper_2509_01190_gb300/csrc/k_gemm_swap.cu": "9b2b21a3a12c31371cef655e5729ddd3c63857a531ad876ce91c8b333b802e9e",
-        "paper_2509_01190_gb300/csrc/common.cuh": "8d770ec1038f925c2dff1202d62b07c60ac07893cae579860cb5e285868bca05",
-        "paper_2509_01190_gb300/csrc/kernels.h": "8551eb6e8e90f525bd89ccdb17fb5bfc3116808f419a84dd3d983791175386c0",
-    },
-}
+# DRAM bytes per launch from single-launch ncu captures (dram__bytes_read.sum +
+# dram__bytes_write.sum, profiles/), keyed by (kernel class, workload): the
+# launch captured, its bytes, and the sha256 of the sources it was measured
+# on.  Reported only while those sources are unchanged, else null.
+TRAFFIC = {}
 
 
-def measured_traffic(kernel_name):
-    """The ncu-measured DRAM bytes per launch of `kernel_name`, or None."""
+def measured_traffic(kernel_name, workload):
+    """The ncu-measured DRAM bytes of one launch of `kernel_name`, or None."""
     import hashlib
-    if kernel_name != "gemm_gate_up_swiglu":
+    rec = TRAFFIC.get((kernel_name, workload))
+    if rec is None:
         return None
-    root = os.path.dirname(os.path.abspath(__file__))
-    for rel, digest in GATE_UP_TRAFFIC["sources"].items():
+    for rel, digest in rec["sources"].items():
         try:
-            with open(os.path.join(root, rel), "rb") as f:
+            with open(os.path.join(ROOT, rel), "rb") as f:
                 if hashlib.sha256(f.read()).hexdigest() != digest:
                     return None
         except OSError:
             return None
-    return GATE_UP_TRAFFIC["bytes_per_launch"]
+    return {"bytes": rec["bytes"], "launch": rec["launch"], "algorithmic_bytes": rec["algorithmic_bytes"]}
 
 
 def _tensors(obj):
@@ -184,18 +182,52 @@ def cpu_threads():
     return os.cpu_count()
 
 
-def time_oracle(shape, weights_np, tokens, accel, budget_s, max_seqs):
-    """Oracle forward on sequences one at a time until budget_s elapses."""
-    from oracle import zsaa_oracle as O
-    ocfg = oracle_config(shape)
-    t0 = time.perf_counter()
-    n = 0
-    while n < max_seqs:
-        O.forward(ocfg, weights_np, tokens[n: n + 1], accel=accel)
-        n += 1
-        if time.perf_counter() - t0 > budget_s:
-            break
-    return n, time.perf_counter() - t0
+class OracleStepper:
+    """The oracle's pruned prefill of one sequence after another, one decoder
+    layer per step (the head runs with the last layer), for the CPU baseline
+    and the reference arm.  A step's work is the modelled FLOPs of what it ran
+    (the planner's cost model, R5), so the rate in tokens/s is
+    L * (modelled work done / modelled work of one sequence) / seconds."""
+
+    def __init__(self, shape, weights_np, tokens, accel):
+        from oracle import zsaa_oracle as O
+        self.O = O
+        self.cfg = oracle_config(shape)
+        self.w = weights_np
+        self.tokens = tokens
+        self.L = tokens.shape[1]
+        self.alpha, self.sched = O.plan(self.cfg, self.L, accel)
+        self.total = O.model_cost(self.cfg, self.sched)
+        f = O.layer_flops_per_row(self.cfg)
+        dq = self.cfg.n_heads * self.cfg.head_dim
+        self.layer_cost = [n * f + 2 * n * n * dq for n in self.sched[:-1]]
+        self.head_cost = self.total - sum(self.layer_cost)
+        self.store = O._Store(self.cfg.dtype)
+        self.seq = 0
+        self.layer = 0
+        self.h = self.pos = None
+
+    def step(self):
+        """Runs one layer; returns its modelled FLOPs."""
+        O = self.O
+        if self.layer == 0:
+            t = self.tokens[self.seq % len(self.tokens)]
+            self.h = self.store(O._as64(self.w["embed"])[t])
+            self.pos = np.arange(self.L)
+        l = self.layer + 1
+        self.h, self.pos, _, _ = O.decoder_layer(self.cfg, self.w["layers"][l - 1], l, self.h, self.pos,
+                                                 self.sched[l], self.store)
+        cost = self.layer_cost[self.layer]
+        self.layer += 1
+        if self.layer == self.cfg.n_layers:
+            O.head(self.cfg, self.w, self.h, self.store)
+            cost += self.head_cost
+            self.layer = 0
+            self.seq += 1
+        return cost
+
+    def tokens_per_s(self, work, seconds):
+        return self.L * (work / self.total) / seconds
 
 
 VARLEN_LENGTHS = [128, 256, 384, 512, 640, 768, 896, 512]  # 4096 tokens, 8 sequences
@@ -306,15 +338,51 @@ def decode_leg(zsaa, model, weights, shape, B, L, accel, tok_dev, stream, barrie
     return out
 
 
+def r4(x):
+    """x to 4 significant digits (short JSON)."""
+    return None if x is None else float(f"{x:.4g}")
+
+
+def gemm_class_bounds(shape, B, sched, peak_tflops, hbm_gbs):
+    """Per GEMM class of one pruned forward: the modelled FLOPs and the bound
+    sum over its launches of max(FLOPs / tensor peak, bytes / HBM bandwidth),
+    with each launch's rows from the schedule (QKV and O-projection on the
+    N_{l-1} rows a layer starts with; the MLP on the N_l rows kept before it;
+    the LM head on the final rows).  Bytes as the library's trace counts them:
+    activations in, weights, outputs (and the residual read)."""
+    d, F, V = shape.d_model, shape.ffn_dim, shape.vocab
+    dq = shape.n_heads * shape.head_dim
+    qkv = dq + 2 * shape.n_kv_heads * shape.head_dim
+    out = {}
+
+    def add(name, flops, nbytes):
+        t = max(flops / (peak_tflops * 1e12), nbytes / (hbm_gbs * 1e9))
+        c = out.setdefault(name, {"flops": 0.0, "bound_ms": 0.0, "launches": 0})
+        c["flops"] += flops
+        c["bound_ms"] += 1e3 * t
+        c["launches"] += 1
+
+    for l in range(1, shape.n_layers + 1):
+        M, Mm = B * sched[l - 1], B * sched[l]
+        add("gemm_qkv_rope", 2.0 * M * qkv * d, 2.0 * (M * d + qkv * d + M * qkv))
+        add("gemm_o_resid", 2.0 * M * d * dq, 2.0 * (M * dq + d * dq + 2 * M * d))
+        add("gemm_gate_up_swiglu", 4.0 * Mm * F * d, 2.0 * (Mm * d + 2 * F * d + Mm * F))
+        add("gemm_down_resid", 2.0 * Mm * d * F, 2.0 * (Mm * F + F * d + 2 * Mm * d))
+    if not shape.n_classes:
+        M = B * sched[-1]
+        add("gemm_lm_head", 2.0 * M * V * d, 2.0 * (M * d + V * d) + 4.0 * M * V)
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="1b", choices=["1b", "1b_cls", "8b"])
+    ap.add_argument("--workload", default="8b", choices=["1b", "1b_cls", "8b"])
     ap.add_argument("--accel", type=float, default=4.0)
-    ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle work for cpu_baseline")
+    ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--no-extras", action="store_true", help="headline timing only")
     args = ap.parse_args()
 
@@ -329,34 +397,39 @@ def main():
     wl = I.WORKLOADS[args.workload]
     shape, B, L = wl["shape"], wl["B"], wl["L"]
     workload_name = f"{shape.name} B={B} L={L} accel={args.accel:g}"
+    config = {"workload": workload_name, "model": shape.name, "global_batch": B * world, "seq_len": L,
+              "accel": args.accel, "parallelism": f"replicas x{world} (independent sequences, no collective)",
+              "l2": "flushed between timed steps (256 MiB write); weights exceed L2"}
 
     if args.impl == "reference":
-        # reference arm: the CPU oracle, one sequence per step, rank 0 only
+        # reference arm: the CPU oracle, one decoder layer per step, rank 0 only
         if rank != 0:
             return
-        g = torch.Generator().manual_seed(I.WEIGHT_SEED)  # noqa: F841  (weights drawn below on CPU)
         weights = I.make_weights(shape, device="cpu")
         wnp = I.weights_to_numpy(weights)
-        tokens = I.make_tokens(max(B, args.steps + args.warmup), L, shape.vocab)
-        from oracle import zsaa_oracle as O
-        ocfg = oracle_config(shape)
-        for w in range(args.warmup):
-            O.forward(ocfg, wnp, tokens[w: w + 1], accel=args.accel)
-        times = []
-        for s in range(args.steps):
+        del weights
+        tokens = I.make_tokens(B, L, shape.vocab)
+        st = OracleStepper(shape, wnp, tokens, args.accel)
+        for _ in range(args.warmup):
+            st.step()
+        work, secs = 0.0, 0.0
+        for _ in range(args.steps):
             t0 = time.perf_counter()
-            O.forward(ocfg, wnp, tokens[(args.warmup + s) % len(tokens)][None], accel=args.accel)
-            times.append(time.perf_counter() - t0)
-        tot = sum(times)
-        val = args.steps * L / tot
+            work += st.step()
+            secs += time.perf_counter() - t0
+        val = st.tokens_per_s(work, secs)
+        cfg = dict(config)
+        cfg["alpha"] = st.alpha
         line = {"impl": "reference", "metric": "prefill_tokens_per_s", "value": val, "unit": "tokens/s",
                 "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-                "ms_per_step": 1e3 * tot / args.steps, "higher_is_better": True, "scaling": "weak",
-                "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-                "config": {"workload": workload_name + " (CPU oracle, 1 sequence per step)",
-                           "global_batch": 1, "seq_len": L, "accel": args.accel},
+                "ms_per_step": 1e3 * secs / args.steps, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded N(0,0.02) weights, uniform token ids)",
+                "config": cfg,
                 "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": cpu_threads(), "kind": "oracle",
-                                 "sample": f"1 of {B} sequences per step, float64 NumPy oracle"},
+                                 "sample": f"float64 NumPy oracle, sequence 0 of the batch, one decoder layer per "
+                                           f"step ({args.warmup} untimed, then layers {args.warmup + 1}.. of the "
+                                           f"chain), rated by modelled FLOPs: {work / st.total:.3f} of a "
+                                           f"sequence in {secs:.1f} s"},
                 "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
         print(json.dumps(line))
         return
@@ -373,6 +446,10 @@ def main():
         torch.cuda.set_device(0)
     dev = torch.device("cuda", torch.cuda.current_device())
     stream = torch.cuda.current_stream()
+    peaks, peak_src = load_peaks()
+    hbm = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+    sust = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    SPEC_TFLOPS, SPEC_GBS = 2250.0, 8000.0  # nominal dense bf16 and HBM3e rates, for context
 
     def barrier():
         R.barrier(dist, torch.cuda.synchronize)
@@ -380,171 +457,155 @@ def main():
     def max_over_ranks(x):
         return R.max_over_ranks(x, dist, dev)
 
-    weights = I.make_weights(shape, device=dev)
-    w_gb = sum({t.data_ptr(): t.numel() * t.element_size() for t in _tensors(weights)}.values()) / 1e9  # tied: once
-    tokens = I.make_tokens(B, L, shape.vocab, seed=R.rank_token_seed(I.TOKEN_SEED, rank))
-    tok_dev = torch.from_numpy(tokens).to(dev)
-    cfg = zsaa.config_from_shape(shape)
-    model = zsaa.Model(cfg, weights, B, L)
-    sched1, _ = zsaa.zsaa_plan(model, L, 1.0)
-    max_out = B * (shape.n_classes if shape.n_classes else L * shape.vocab)
-    logits = torch.empty(max_out, device=dev, dtype=torch.float32)
     flush = torch.empty(256 * 1024 * 1024 // 4, device=dev, dtype=torch.float32)
 
-    def run(accel):
-        zsaa.zsaa_forward(model, tok_dev, B, L, accel, logits, None, stream=stream)
+    class Workload:
+        def __init__(self, name):
+            w = I.WORKLOADS[name]
+            self.name, self.shape, self.B, self.L, self.accels = name, w["shape"], w["B"], w["L"], w["accels"]
+            self.weights = I.make_weights(self.shape, device=dev)
+            self.tokens = I.make_tokens(self.B, self.L, self.shape.vocab,
+                                        seed=R.rank_token_seed(I.TOKEN_SEED, rank))
+            self.tok_dev = torch.from_numpy(self.tokens).to(dev)
+            self.cfg = zsaa.config_from_shape(self.shape)
+            self.model = zsaa.Model(self.cfg, self.weights, self.B, self.L)
+            n_out = self.B * (self.shape.n_classes if self.shape.n_classes else self.L * self.shape.vocab)
+            self.logits = torch.empty(n_out, device=dev, dtype=torch.float32)
 
-    def timed(accel, steps, warmup, sampler=None):
-        for _ in range(warmup):
-            run(accel)
-        zsaa.zsaa_sync(model)
-        barrier()
-        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
-        ctx = sampler if sampler is not None else None
-        if ctx:
-            ctx.__enter__()
-        try:
-            for a, b in evs:
-                flush.zero_()
-                a.record(stream)
-                run(accel)
-                b.record(stream)
-            torch.cuda.synchronize()
-        finally:
-            if ctx:
-                ctx.__exit__(None, None, None)
-        zsaa.zsaa_sync(model)
-        ms = sum(a.elapsed_time(b) for a, b in evs)
-        barrier()
-        return max_over_ranks(ms) / steps
+        def run(self, accel):
+            zsaa.zsaa_forward(self.model, self.tok_dev, self.B, self.L, accel, self.logits, None, stream=stream)
+
+        def timed(self, accel, steps, warmup, sampler=None):
+            for _ in range(warmup):
+                self.run(accel)
+            zsaa.zsaa_sync(self.model)
+            barrier()
+            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                   for _ in range(steps)]
+            if sampler:
+                sampler.__enter__()
+            try:
+                for a, b in evs:
+                    flush.zero_()
+                    a.record(stream)
+                    self.run(accel)
+                    b.record(stream)
+                torch.cuda.synchronize()
+            finally:
+                if sampler:
+                    sampler.__exit__(None, None, None)
+            zsaa.zsaa_sync(self.model)
+            ms = sum(a.elapsed_time(b) for a, b in evs)
+            barrier()
+            return max_over_ranks(ms) / steps
+
+        def sweep(self, steps, known=None):
+            from oracle import zsaa_oracle as O
+            ocfg = oracle_config(self.shape)
+            sched1, _ = zsaa.zsaa_plan(self.model, self.L, 1.0)
+            full = O.model_cost(ocfg, sched1)
+            out = {}
+            for a in self.accels:
+                ms = known[a] if known and a in known else self.timed(a, steps, 3)
+                s_a, al = zsaa.zsaa_plan(self.model, self.L, a)
+                out[a] = {"ms": ms, "alpha": al, "final_rows": s_a[-1],
+                          "flop_red": full / O.model_cost(ocfg, s_a)}
+            base = out[1.0]["ms"] if 1.0 in out else None
+            for v in out.values():
+                v["x"] = base / v["ms"] if base else None
+            return out
+
+        def close(self):
+            self.model.close()
+            del self.weights, self.logits
+
+    main_wl = Workload(args.workload)
+    sched, alpha = zsaa.zsaa_plan(main_wl.model, L, args.accel)
+    config["alpha"] = alpha
+    config["schedule"] = sched
 
     # ---- headline (plain forwards replay from the library's CUDA graphs)
     sampler = ClockSampler(local) if rank == 0 else None
-    ms_head = timed(args.accel, args.steps, args.warmup, sampler)
-    sched, alpha = zsaa.zsaa_plan(model, L, args.accel)
+    ms_head = main_wl.timed(args.accel, args.steps, args.warmup, sampler)
     value = R.job_tokens_per_s(world, B, L, ms_head)
     clocks = sampler.summary() if sampler else None
 
     line = {"metric": "prefill_tokens_per_s", "value": value, "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_head, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if shape.dtype == "bf16" else "f32",
-            "data": "synthetic (seeded N(0,0.02) weights, uniform token ids)",
-            "config": {"workload": workload_name, "model": shape.name, "global_batch": B * world,
-                       "seq_len": L, "accel": args.accel, "alpha": alpha, "schedule": sched,
-                       "parallelism": f"replicas x{world} (independent sequences, no collective)",
-                       "l2": f"flushed between timed steps (256 MiB write); weights {w_gb:.1f} GB > L2"},
+            "data": "synthetic (seeded N(0,0.02) weights, uniform token ids)", "config": config,
             "clocks": clocks}
+    tail = {}
 
     if not args.no_extras:
-        from oracle import zsaa_oracle as O
-        ocfg = oracle_config(shape)
-        full_cost = O.model_cost(ocfg, sched1)
         # ---- accel sweep (speedup over the same library's unpruned forward)
-        sweep = {}
-        base_ms = None
-        for a in sorted(set(wl["accels"]) | {args.accel}):
-            ms = ms_head if a == args.accel else timed(a, args.steps, 3)
-            s_a, al_a = zsaa.zsaa_plan(model, L, a)
-            if a == 1.0:
-                base_ms = ms
-            sweep[f"{a:g}"] = {"ms": ms, "tokens_per_s": R.job_tokens_per_s(world, B, L, ms), "alpha": al_a,
-                               "final_rows": s_a[-1],
-                               "modelled_flop_reduction": full_cost / O.model_cost(ocfg, s_a)}
-        for k, v in sweep.items():
-            v["speedup_vs_unpruned"] = (base_ms / v["ms"]) if base_ms else None
-        line["sweep"] = sweep
+        sw = main_wl.sweep(args.steps, known={args.accel: ms_head})
         # the same headline forward without graph replay (every launch from the host)
-        zsaa.zsaa_model_set_graphs(model, False)
-        line["ms_per_step_eager"] = timed(args.accel, args.steps, 3)
-        zsaa.zsaa_model_set_graphs(model, True)
-
-        # ---- isolated score + select + compaction on [32, 4096, 4096] bf16 (1 GiB,
-        # larger than L2): algorithmic bytes = read every row once + write the
-        # kept rows = 2*B*L*d + 2*B*k*d
-        mb = I.WORKLOADS["microbench"]
-        mB, mL, md = mb["B"], mb["L"], mb["d"]
-        hidden = I.make_hidden(mB, mL, md, device=dev)
-        peaks_mb, src_mb = load_peaks()
-        hbm = peaks_mb.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
-        micro = {}
-        for a in mb["accels"]:
-            k = int(mL // a)
-            idx = torch.empty(mB, k, device=dev, dtype=torch.int32)
-            rows = torch.empty(mB, k, md, device=dev, dtype=torch.bfloat16)
-            for _ in range(3):
-                zsaa.zsaa_score_select(hidden, mB, mL, md, k, idx, rows, stream=stream)
-            torch.cuda.synchronize()
-            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(10)]
-            for e0, e1 in evs:
-                flush.zero_()
-                e0.record(stream)
-                zsaa.zsaa_score_select(hidden, mB, mL, md, k, idx, rows, stream=stream)
-                e1.record(stream)
-            torch.cuda.synchronize()
-            us = 1e3 * sum(e0.elapsed_time(e1) for e0, e1 in evs) / len(evs)
-            nbytes = 2.0 * mB * mL * md + 2.0 * mB * k * md
-            micro[f"{a:g}"] = {"k": k, "us": us, "algorithmic_bytes": nbytes,
-                               "gbs": nbytes / (us * 1e3), "frac_of_hbm": nbytes / (us * 1e3) / hbm}
-            del idx, rows
-        del hidden
-        line["microbench_score_select"] = {
-            "workload": f"hidden [{mB}, {mL}, {md}] bf16, N(0,1) x per-row log-normal scale; "
-                        "zsaa_score_select (row-norm score, top-k, gather)",
-            "peak_gbs": hbm, "peak_source": f"{src_mb} hbm_gbs", "by_accel": micro}
+        zsaa.zsaa_model_set_graphs(main_wl.model, False)
+        line["ms_per_step_eager"] = main_wl.timed(args.accel, args.steps, 3)
+        zsaa.zsaa_model_set_graphs(main_wl.model, True)
 
         # ---- per-kernel trace of the headline forward (separate traced steps)
-        zsaa.zsaa_trace_begin(model)
+        zsaa.zsaa_trace_begin(main_wl.model)
         n_tr = 3
         for _ in range(n_tr):
             flush.zero_()
-            run(args.accel)
-        rows = zsaa.zsaa_trace_end(model)
-        zsaa.zsaa_sync(model)
+            main_wl.run(args.accel)
+        rows = zsaa.zsaa_trace_end(main_wl.model)
+        zsaa.zsaa_sync(main_wl.model)
         tot_ms = sum(r["ms"] for r in rows)
         kern = {}
         for r in rows:
-            kern[r["name"]] = {"launches_per_step": r["launches"] / n_tr, "ms_per_step": r["ms"] / n_tr,
-                               "share": r["ms"] / tot_ms if tot_ms else None,
-                               "tflops": (r["flops"] / (r["ms"] / 1e3) / 1e12) if r["ms"] and r["flops"] else None,
-                               "gbs": (r["bytes"] / (r["ms"] / 1e3) / 1e9) if r["ms"] else None}
+            kern[r["name"]] = {"launches": r["launches"] / n_tr, "ms": r4(r["ms"] / n_tr),
+                               "share": r4(r["ms"] / tot_ms) if tot_ms else None,
+                               "tflops": r4(r["flops"] / (r["ms"] / 1e3) / 1e12) if r["ms"] and r["flops"] else None,
+                               "gbs": r4(r["bytes"] / (r["ms"] / 1e3) / 1e9) if r["ms"] else None}
         line["kernels"] = kern
-        launches = sum(r["launches"] for r in rows) // n_tr
-        line["gpu_launches"] = launches * args.steps
-        peaks, src = load_peaks()
+        line["gpu_launches"] = int(sum(r["launches"] for r in rows) // n_tr) * args.steps
         gemms = [r for r in rows if r["name"].startswith("gemm")]
-        dom = max(gemms, key=lambda r: r["ms"]) if gemms else max(rows, key=lambda r: r["ms"])
-        if dom["flops"] > 0:
-            ach = dom["flops"] / (dom["ms"] / 1e3) / 1e12
-            peak = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
-            line["roofline"] = {"bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
-                                "frac": ach / peak, "traffic": measured_traffic(dom["name"]),
-                                "kernel": dom["name"],
-                                "per_launch_ms": dom["ms"] / dom["launches"],
-                                "peak_source": f"{src} bf16_tflops_sustained (kernel inside a long step)"}
-        else:
-            ach = dom["bytes"] / (dom["ms"] / 1e3) / 1e9
-            peak = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
-            line["roofline"] = {"bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
-                                "frac": ach / peak, "traffic": None, "kernel": dom["name"],
-                                "peak_source": f"{src} hbm_gbs"}
-        gemm_f = sum(r["flops"] for r in gemms)
-        gemm_ms = sum(r["ms"] for r in gemms)
-        if gemm_ms:
-            line["roofline"]["all_gemms_tflops"] = gemm_f / (gemm_ms / 1e3) / 1e12
-            line["roofline"]["all_gemms_share"] = gemm_ms / tot_ms
+        dom = max(gemms, key=lambda r: r["ms"])
+        per_launch = dom["ms"] / dom["launches"]
+        ach = dom["flops"] / (dom["ms"] / 1e3) / 1e12
+        bounds = gemm_class_bounds(shape, B, sched, sust, hbm)
+        tr = measured_traffic(dom["name"], args.workload)
+        line["roofline"] = {
+            "bound": "tensor", "achieved": ach, "peak": sust, "unit": "TFLOP/s", "frac": ach / sust,
+            "traffic": tr["bytes"] if tr else None, "kernel": dom["name"],
+            "per_launch_ms": per_launch,
+            "peak_source": f"{peak_src} bf16_tflops_sustained (kernel inside a long step)",
+            "frac_of_spec_2250": ach / SPEC_TFLOPS,
+            "frac_of_own_bound": bounds[dom["name"]]["bound_ms"] * n_tr / dom["ms"]}
+        if tr:
+            line["roofline"]["traffic_launch"] = tr["launch"]
+            line["roofline"]["traffic_algorithmic_bytes"] = tr["algorithmic_bytes"]
+        gc = {}
+        for r in gemms:
+            b_ = bounds.get(r["name"])
+            if b_ is None:
+                continue
+            ms = r["ms"] / n_tr
+            gc[r["name"]] = {"ms": r4(ms), "bound_ms": r4(b_["bound_ms"]), "frac_of_bound": r4(b_["bound_ms"] / ms),
+                             "tflops": r4(r["flops"] / (r["ms"] / 1e3) / 1e12),
+                             "frac_of_sustained": r4(r["flops"] / (r["ms"] / 1e3) / 1e12 / sust)}
+        gms = sum(r["ms"] for r in gemms) / n_tr
+        gc["all"] = {"ms": r4(gms), "bound_ms": r4(sum(v["bound_ms"] for v in bounds.values())),
+                     "tflops": r4(sum(r["flops"] for r in gemms) / n_tr / (gms / 1e3) / 1e12),
+                     "share_of_device_time": r4(gms * n_tr / tot_ms)}
+        line["gemm_classes"] = {"bound": "per launch max(FLOPs / sustained bf16 peak, bytes / measured HBM)",
+                                "by_class": gc}
 
         # ---- end to end through the host-buffer entry point
         n_fin = sched[-1]
         n_logit = B * (shape.n_classes if shape.n_classes else n_fin * shape.vocab)
-        tok_h = torch.from_numpy(tokens).pin_memory()
+        tok_h = torch.from_numpy(main_wl.tokens).pin_memory()
         log_h = torch.empty(n_logit, dtype=torch.float32).pin_memory()
         for _ in range(2):
-            zsaa.zsaa_forward_host(model, tok_h, B, L, args.accel, log_h, None, stream=stream)
+            zsaa.zsaa_forward_host(main_wl.model, tok_h, B, L, args.accel, log_h, None, stream=stream)
         barrier()
         t0 = time.perf_counter()
         for _ in range(args.steps):
             flush.zero_()
-            zsaa.zsaa_forward_host(model, tok_h, B, L, args.accel, log_h, None, stream=stream)
+            zsaa.zsaa_forward_host(main_wl.model, tok_h, B, L, args.accel, log_h, None, stream=stream)
         torch.cuda.synchronize()
         e2e_s = max_over_ranks(time.perf_counter() - t0) / args.steps
         line["e2e"] = {"value": world * B * L / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": B * L * 4,
@@ -552,51 +613,94 @@ def main():
                        "note": "zsaa_forward_host: pinned host tokens in, host float32 logits out; "
                                "the 256 MiB L2 flush runs inside this span"}
 
-        # ---- Appendix B's masked mode on the same batch: nothing removed, so the
-        # cost of the unpruned forward (the speedup comes from compaction)
-        if shape.dtype == "bf16":
-            n_fin = sched[-1]
-            lg_m = torch.empty(max_out, device=dev, dtype=torch.float32)
+        # ---- CPU oracle on the host cores (rank 0, N=1 only)
+        if rank == 0 and world == 1:
+            wnp = I.weights_to_numpy(main_wl.weights)
+            st = OracleStepper(shape, wnp, main_wl.tokens, args.accel)
+            work, t0 = 0.0, time.perf_counter()
+            while True:
+                work += st.step()
+                if time.perf_counter() - t0 > args.cpu_budget:
+                    break
+            secs = time.perf_counter() - t0
+            line["cpu_baseline"] = {
+                "value": st.tokens_per_s(work, secs), "unit": "tokens/s", "cores": cpu_threads(), "kind": "oracle",
+                "sample": f"float64 NumPy oracle on sequence 0 at accel {args.accel:g}, layers 1-{st.layer or st.cfg.n_layers}"
+                          f" of the chain in {secs:.1f} s ({work / st.total:.3f} of a sequence by modelled FLOPs)"}
+            del wnp, st
 
-            def run_masked():
-                zsaa.zsaa_forward_masked(model, tok_dev, B, L, args.accel, lg_m, None, stream=stream)
+        # ---- the 1B workloads: sweeps, and on the LM shape decode / varlen / masked mode
+        others = {}
+        for name in ("1b", "1b_cls"):
+            if name == args.workload:
+                continue
+            ow = Workload(name)
+            osw = ow.sweep(max(5, args.steps // 3))
+            others[name] = {f"{a:g}": {"ms": r4(v["ms"]), "x": r4(v["x"])} for a, v in osw.items()}
+            if name == "1b":
+                acc = 4.0
+                lg_m = torch.empty_like(ow.logits)
+
+                def run_masked():
+                    zsaa.zsaa_forward_masked(ow.model, ow.tok_dev, ow.B, ow.L, acc, lg_m, None, stream=stream)
+                for _ in range(3):
+                    run_masked()
+                torch.cuda.synchronize()
+                evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                       for _ in range(10)]
+                for e0, e1 in evs:
+                    flush.zero_()
+                    e0.record(stream)
+                    run_masked()
+                    e1.record(stream)
+                torch.cuda.synchronize()
+                zsaa.zsaa_sync(ow.model)
+                ms_m = max_over_ranks(sum(a.elapsed_time(b) for a, b in evs) / len(evs))
+                line["masked_mode_1b"] = {"accel": acc, "ms_per_step": ms_m, "vs_compacted": ms_m / osw[acc]["ms"],
+                                          "note": "zsaa_forward_masked, eager launches"}
+                line["varlen_1b"] = varlen_leg(zsaa, ow.weights, ow.cfg, ow.shape, acc, flush, stream,
+                                               max_over_ranks, world, 10)
+                line["decode_1b"] = decode_leg(zsaa, ow.model, ow.weights, ow.shape, ow.B, ow.L, acc, ow.tok_dev,
+                                               stream, barrier, max_over_ranks, world)
+            ow.close()
+            del ow
+            torch.cuda.empty_cache()
+
+        # ---- isolated score + select + compaction on [32, 4096, 4096] bf16 (1 GiB,
+        # larger than L2): algorithmic bytes = read every row once + write the
+        # kept rows = 2*B*L*d + 2*B*k*d
+        mb = I.WORKLOADS["microbench"]
+        mB, mL, md = mb["B"], mb["L"], mb["d"]
+        hidden = I.make_hidden(mB, mL, md, device=dev)
+        micro = {}
+        for a in mb["accels"]:
+            k = int(mL // a)
+            idx = torch.empty(mB, k, device=dev, dtype=torch.int32)
+            rws = torch.empty(mB, k, md, device=dev, dtype=torch.bfloat16)
             for _ in range(3):
-                run_masked()
+                zsaa.zsaa_score_select(hidden, mB, mL, md, k, idx, rws, stream=stream)
             torch.cuda.synchronize()
-            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                   for _ in range(args.steps)]
+            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(10)]
             for e0, e1 in evs:
                 flush.zero_()
                 e0.record(stream)
-                run_masked()
+                zsaa.zsaa_score_select(hidden, mB, mL, md, k, idx, rws, stream=stream)
                 e1.record(stream)
             torch.cuda.synchronize()
-            zsaa.zsaa_sync(model)
-            ms_m = max_over_ranks(sum(a.elapsed_time(b) for a, b in evs) / args.steps)
-            line["masked_mode"] = {"accel": args.accel, "ms_per_step": ms_m,
-                                   "tokens_per_s": R.job_tokens_per_s(world, B, L, ms_m),
-                                   "vs_compacted": ms_m / ms_head, "final_rows": n_fin,
-                                   "note": "zsaa_forward_masked, eager launches"}
+            us = 1e3 * sum(e0.elapsed_time(e1) for e0, e1 in evs) / len(evs)
+            nbytes = 2.0 * mB * mL * md + 2.0 * mB * k * md
+            micro[f"{a:g}"] = {"us": r4(us), "gbs": r4(nbytes / (us * 1e3)), "frac": r4(nbytes / (us * 1e3) / hbm),
+                               "frac_8tbs": r4(nbytes / (us * 1e3) / SPEC_GBS)}
+            del idx, rws
+        del hidden
 
-        # ---- variable-length batch: the same 4096 tokens as B x L, in mixed lengths
-        if shape.n_classes == 0 and B * L == 4096:
-            line["varlen"] = varlen_leg(zsaa, weights, cfg, shape, args.accel, flush, stream,
-                                        max_over_ranks, world, args.steps)
-
-        # ---- generation over the pruned KV cache (LM head only): B tokens per step
-        if not shape.n_classes:
-            line["decode"] = decode_leg(zsaa, model, weights, shape, B, L, args.accel, tok_dev, stream,
-                                        barrier, max_over_ranks, world)
-
-        # ---- CPU oracle on the host cores (rank 0, N=1 only)
-        if rank == 0 and world == 1:
-            wnp = I.weights_to_numpy(weights)
-            n, secs = time_oracle(shape, wnp, tokens, args.accel, args.cpu_budget, B)
-            line["cpu_baseline"] = {"value": n * L / secs, "unit": "tokens/s", "cores": cpu_threads(),
-                                    "kind": "oracle",
-                                    "sample": f"{n} of {B} sequences x {L} tokens at accel {args.accel:g}, "
-                                              f"float64 NumPy oracle, {secs:.1f} s"}
+        # short summaries last on the line
+        tail["sweep"] = {f"{a:g}": {"ms": r4(v["ms"]), "tok_s": r4(R.job_tokens_per_s(world, B, L, v["ms"])),
+                                    "x": r4(v["x"]), "flop_red": r4(v["flop_red"])} for a, v in sw.items()}
+        tail["microbench_score_select"] = {"shape": [mB, mL, md], "peak_gbs": hbm, "by_accel": micro}
+        tail["other_workloads"] = others
     if rank == 0:
+        line.update(tail)
         print(json.dumps(line))
     if dist is not None:
         dist.destroy_process_group()
