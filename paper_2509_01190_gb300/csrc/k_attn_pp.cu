@@ -67,6 +67,15 @@ struct PpItem {
   int qb, b, g, h0, n_kb;
 };
 
+// The r-th work item of this CTA: items are numbered longest query blocks
+// first and dealt to the CTAs in a snake order (0..G-1, then G-1..0, ...), so
+// the causal triangle's long and short items even out across CTAs.  Returns
+// an index >= total once the CTA has none left (the sequence only grows).
+__device__ __forceinline__ int pp_item_index(int r) {
+  const int G = gridDim.x, i = blockIdx.x;
+  return r * G + ((r & 1) ? G - 1 - i : i);
+}
+
 // Work item t, longest query blocks first.
 __device__ __forceinline__ PpItem pp_item(int t, const PpArgs& a) {
   PpItem it;
@@ -113,6 +122,31 @@ __device__ __forceinline__ void tc_mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem,
       "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
       "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
+}
+
+// Packed pairs of floats (sm_100 f32x2 arithmetic: one instruction, two lanes of work).
+__device__ __forceinline__ uint64_t f2pack(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ void f2unpack(uint64_t v, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
+}
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ uint64_t fsub2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
 }
 
 // Warp-collective: lane i reads / writes TMEM lane (base + i), 32 consecutive columns.
@@ -202,7 +236,7 @@ __global__ void __launch_bounds__(PP_THREADS, 1)
     if (lane == 0) {
       bool ok = true;
       uint32_t J = 0, items = 0, q_issued = 0;
-      for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++items) {
+      for (int t = pp_item_index(0); t < total && ok; t = pp_item_index(++items)) {
         const PpItem it = pp_item(t, a);
         const int row0 = it.b * a.N;
         if (!mbar_wait_ab(q_empty, (items & 1) ^ 1, a.status, abort_flag)) {
@@ -266,7 +300,7 @@ __global__ void __launch_bounds__(PP_THREADS, 1)
                            sdesc_sw128_mn(va + kk * 16 * 128, kVChunkStride), idesc_o,
                            (first && part == 0 && kk == 0) ? 0u : 1u);
       };
-      for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++items) {
+      for (int t = pp_item_index(0); t < total && ok; t = pp_item_index(++items)) {
         const PpItem it = pp_item(t, a);
         if (!mbar_wait_ab(q_full, items & 1, a.status, abort_flag)) {
           ok = false;
@@ -336,7 +370,7 @@ __global__ void __launch_bounds__(PP_THREADS, 1)
       __syncwarp();
       if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
     };
-    for (int t = blockIdx.x; t < total; t += gridDim.x, ++items) {
+    for (int t = pp_item_index(0); t < total; t = pp_item_index(++items)) {
       const PpItem it = pp_item(t, a);
       const int q = it.qb * PP_BM + row;
       float m = -INFINITY, l = 0.f;
@@ -390,25 +424,34 @@ __global__ void __launch_bounds__(PP_THREADS, 1)
           }
           // pass 2: P as a bf16 pair over the S columns just read; the next
           // chunk's load is in flight while this one is converted
-          const float nm = -m;
+          // P = 2^(s*scale - m) split as hi = P rounded to bf16 and lo = P - hi
+          // (exact in fp32, then rounded to bf16), so hi + lo carries P to
+          // about 17 bits
+          const uint64_t scale2 = f2pack(a.scale_log2, a.scale_log2);
+          const uint64_t nm2 = f2pack(-m, -m);
           auto emit = [&](const uint32_t (&r)[32], int c) {
             uint32_t hi[16], lo[16];
-            float lsum0 = 0.f, lsum1 = 0.f;
+            uint64_t lsum = f2pack(0.f, 0.f);
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
-              const int k = 32 * c + 2 * e;
-              float p0 = ex2_fast(fmaf(__uint_as_float(r[2 * e]), a.scale_log2, nm));
-              float p1 = ex2_fast(fmaf(__uint_as_float(r[2 * e + 1]), a.scale_log2, nm));
+              float t0, t1;
+              f2unpack(ffma2(f2pack(__uint_as_float(r[2 * e]), __uint_as_float(r[2 * e + 1])), scale2, nm2), t0, t1);
+              float p0 = ex2_fast(t0), p1 = ex2_fast(t1);
               if (masked) {
+                const int k = 32 * c + 2 * e;
                 p0 = k < lim ? p0 : 0.f;
                 p1 = k + 1 < lim ? p1 : 0.f;
               }
-              lsum0 += p0;
-              lsum1 += p1;
+              const uint64_t pp = f2pack(p0, p1);
+              lsum = fadd2(lsum, pp);
               hi[e] = pack_bf16x2(p0, p1);
-              lo[e] = pack_bf16x2(p0 - bf16lo(hi[e]), p1 - bf16hi(hi[e]));
+              float r0, r1;
+              f2unpack(fsub2(pp, f2pack(bf16lo(hi[e]), bf16hi(hi[e]))), r0, r1);
+              lo[e] = pack_bf16x2(r0, r1);
             }
-            l += lsum0 + lsum1;
+            float l0, l1;
+            f2unpack(lsum, l0, l1);
+            l += l0 + l1;
             tmem_st16(s_addr + 32 * c, hi);
             tmem_st16(s_addr + 32 * c + 16, lo);
           };
