@@ -8,10 +8,7 @@
 // encoder), and its epilogue warps -- one TMEM lane,
 // i.e. one key, per thread -- accumulate exp2(s * c - lse2[q]) over the
 // queries q >= key of each block.  That is the column sum of the normalised
-// soft-score P (the row normalisers lse2 come from the attention kernel;
-// each step's 128 are loaded a step ahead into registers and kept negated in
-// shared memory, so a pair of terms costs one packed fused multiply-add, two
-// exp2 and one packed add).
+// soft-score P (the row normalisers lse2 come from the attention kernel).
 // Each head writes its own partial, optionally times ||v_key|| of group g (the
 // position score of R1 is linear in the column mass; the norms come from the
 // QKV projection's epilogue):   parts[hh][b][g][key]
@@ -21,7 +18,8 @@
 // through a 4-stage ring), warp 1 MMA issuer, warps 2..9 epilogue (warp w
 // reads TMEM lanes 32*(w%4)..+32, columns half (w-2)/4 of each 128-query
 // block; the halves are added in shared memory at the end of a tile).  Two
-// TMEM accumulators let a block's epilogue overlap the next block's MMAs.
+// TMEM accumulators let a block's epilogue overlap the next block's MMAs, and
+// the next block's query normalisers are fetched with cp.async meanwhile.
 // All waits are bounded; epilogue warps never leave the step loop early, so
 // their named barriers cannot strand the others.
 #include <mutex>
@@ -65,26 +63,6 @@ __device__ __forceinline__ float ex2_ftz(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
-}
-
-// Packed pairs of floats (sm_100 f32x2 arithmetic).
-__device__ __forceinline__ uint64_t f2pack(float a, float b) {
-  uint64_t r;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
-  return r;
-}
-__device__ __forceinline__ void f2unpack(uint64_t v, float& a, float& b) {
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
-}
-__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
-  uint64_t r;
-  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
-  return r;
-}
-__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
-  uint64_t r;
-  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
-  return r;
 }
 
 __device__ __forceinline__ void cm_tile(int t, const CmArgs& a, int& b, int& g, int& hh, int& kb) {
@@ -257,30 +235,35 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
     const int ew = warp - 2;
     const int quad = warp & 3, half = ew / 4;
     const int krow = quad * 32 + lane;  // key within the tile
-    const int et = ew * 32 + lane;      // 0..255: threads 0..127 load one normaliser each
-    // The normaliser of query q of step (t, qb), negated: exp2(s * c - lse2)
-    // is then one fused multiply-add and an exp2.  A hidden query (masked
-    // mode) gets -inf, so it adds nothing; a query past the sequence gets 0
-    // (its columns are masked anyway).
-    auto neg_lse = [&](int t, int qb) -> float {
-      if (et >= CM_BN) return 0.f;
-      int b, g, hh, kb, row0, n_b;
-      cm_tile(t, a, b, g, hh, kb);
-      cm_seq(a, b, row0, n_b);
-      const int h = g * (a.Hq / a.Hkv) + hh;
-      const int q = qb * CM_BN + et;
-      if (q >= n_b) return 0.f;
-      if (a.q_alive != nullptr && a.q_alive[static_cast<size_t>(b) * a.N + q] == 0) return -INFINITY;
-      return -__ldg(a.lse2 + (static_cast<size_t>(b) * a.Hq + h) * a.N + q);
+    const int et = ew * 32 + lane;      // 0..255: loader of one normaliser
+    // fetch the normalisers of step (t, qb) into s_lse[buf]
+    auto fetch = [&](int t, int qb, int buf) {
+      if (et < CM_BN) {
+        int b, g, hh, kb, row0, n_b;
+        cm_tile(t, a, b, g, hh, kb);
+        cm_seq(a, b, row0, n_b);
+        const int h = g * (a.Hq / a.Hkv) + hh;
+        const int q = qb * CM_BN + et;
+        float* dst = s_lse + buf * CM_BN + et;
+        if (q < n_b && a.q_alive != nullptr && a.q_alive[static_cast<size_t>(b) * a.N + q] == 0) {
+          *dst = INFINITY;  // exp2(s * c - inf) = 0: a hidden query contributes nothing
+        } else if (q < n_b) {
+          asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)),
+                       "l"(a.lse2 + (static_cast<size_t>(b) * a.Hq + h) * a.N + q)
+                       : "memory");
+        } else {
+          *dst = 0.f;
+        }
+      }
+      cp_async_commit();
     };
-    const uint64_t scale2 = f2pack(a.scale_log2, a.scale_log2);
     int i = 0;
     bool ok = true;
     const int t_first = cm_next(blockIdx.x, a);
-    if (t_first < a.total && et < CM_BN) {
+    if (t_first < a.total) {
       int b, g, hh, kb;
       cm_tile(t_first, a, b, g, hh, kb);
-      s_lse[et] = neg_lse(t_first, a.causal ? kb : 0);
+      fetch(t_first, a.causal ? kb : 0, 0);
     }
     for (int t = t_first; t < a.total; t = cm_next(t + gridDim.x, a)) {
       int b, g, hh, kb, row0, n_b;
@@ -288,26 +271,24 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
       cm_seq(a, b, row0, n_b);
       const int n_qb = (n_b + CM_BN - 1) / CM_BN;
       const int key = kb * CM_BM + krow;
-      uint64_t acc2a = f2pack(0.f, 0.f), acc2b = f2pack(0.f, 0.f);
       float acc = 0.f;
       for (int qb = a.causal ? kb : 0; qb < n_qb; ++qb, ++i) {
         const int ab = i & 1;
         const uint32_t use = static_cast<uint32_t>(i >> 1);
+        cp_async_wait<0>();
         // this step's normalisers are in s_lse[ab]; every warp is done with step i-1
         asm volatile("bar.sync 1, %0;" ::"n"(CM_EPI_WARPS * 32) : "memory");
-        // the next step's normalisers, loaded now and stored after this step
-        float nxt = 0.f;
         if (qb + 1 < n_qb) {
-          nxt = neg_lse(t, qb + 1);
+          fetch(t, qb + 1, ab ^ 1);
         } else {
           const int tn = cm_next(t + gridDim.x, a);
           if (tn < a.total) {
             int b2, g2, hh2, kb2;
             cm_tile(tn, a, b2, g2, hh2, kb2);
-            nxt = neg_lse(tn, a.causal ? kb2 : 0);
+            fetch(tn, a.causal ? kb2 : 0, ab ^ 1);
           }
         }
-        const float* NL = s_lse + ab * CM_BN;
+        const float* L = s_lse + ab * CM_BN;
         ok = ok && __all_sync(0xffffffffu, mbar_wait_ab(&acc_full[ab], use & 1, a.status, abort_flag));
         tc_fence_after();
         if (ok) {
@@ -324,34 +305,20 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
             const int q0 = qb * CM_BN + qc0;
             if ((!a.causal || q0 > key) && q0 + 32 <= n_b) {  // whole chunk inside the mask
 #pragma unroll
-              for (int e = 0; e < 32; e += 4) {
-                const float4 nl = *reinterpret_cast<const float4*>(NL + qc0 + e);
-                float t0, t1, t2, t3;
-                f2unpack(ffma2(f2pack(__uint_as_float(r[e]), __uint_as_float(r[e + 1])), scale2, f2pack(nl.x, nl.y)), t0, t1);
-                f2unpack(ffma2(f2pack(__uint_as_float(r[e + 2]), __uint_as_float(r[e + 3])), scale2, f2pack(nl.z, nl.w)), t2, t3);
-                acc2a = fadd2(acc2a, f2pack(ex2_ftz(t0), ex2_ftz(t1)));
-                acc2b = fadd2(acc2b, f2pack(ex2_ftz(t2), ex2_ftz(t3)));
-              }
+              for (int e = 0; e < 32; ++e) acc += ex2_ftz(__uint_as_float(r[e]) * a.scale_log2 - L[qc0 + e]);
             } else {
 #pragma unroll
               for (int e = 0; e < 32; ++e) {
                 const int q = q0 + e;
                 if ((!a.causal || q >= key) && q < n_b)
-                  acc += ex2_ftz(fmaf(__uint_as_float(r[e]), a.scale_log2, NL[qc0 + e]));
+                  acc += ex2_ftz(__uint_as_float(r[e]) * a.scale_log2 - L[qc0 + e]);
               }
             }
           }
         }
-        if (et < CM_BN) s_lse[(ab ^ 1) * CM_BN + et] = nxt;
         tc_fence_before();
         __syncwarp();
         if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&acc_empty[ab])) : "memory");
-      }
-      {
-        float x0, x1, x2, x3;
-        f2unpack(acc2a, x0, x1);
-        f2unpack(acc2b, x2, x3);
-        acc += (x0 + x1) + (x2 + x3);
       }
       // add the two column halves (fixed order: half 0 + half 1)
       if (half == 1) s_half[krow] = acc;
@@ -363,6 +330,7 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
       }
       // s_half is rewritten only after the next tile's first barrier
     }
+    cp_async_wait<0>();
   }
   tc_fence_before();
   __syncthreads();

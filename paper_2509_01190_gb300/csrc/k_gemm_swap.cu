@@ -542,8 +542,14 @@ cudaError_t run_swap(const void* A, int lda, const TcWeights& W, const GemmParam
   const int bands = DUAL ? (p.N + SW_BAND / 2 - 1) / (SW_BAND / 2) : (p.N + SW_BAND - 1) / SW_BAND;
   const size_t smem = smem_bytes(SW_W_BYTES, sh.Mp, sh.stages, sh.ksub);
 
-  // Cluster size: fewest k-blocks per CTA over the waves the clusters need;
-  // a wave costs about two k-blocks of fixed work (launch, TMEM, reduction).
+  // Cluster size: fewest k-blocks per CTA over the waves the clusters need,
+  // with a wave's fixed work (launch, TMEM, cluster reduction, epilogue)
+  // counted as a number of k-blocks.  Swept on GB300 over the 1B and 8B
+  // projections of the accel-4 forwards (2, 6, 12, 24): 24 is best for the
+  // RoPE epilogue (8B QKV at 192..316 rows 26.5 -> 20.1 us), 12 for the
+  // residual one (8B O at 516..744 rows 49 -> 29..33 us), 2 for SwiGLU (whose
+  // k-blocks carry twice the weights; larger values cost it 5-12%).
+  const double wave_cost = EPI == kEpiRope ? 24.0 : (EPI == kEpiResid ? 12.0 : 2.0);
   const int units = bands * nrb2;
   int best = 1;
   double best_cost = 1e30;
@@ -551,7 +557,7 @@ cudaError_t run_swap(const void* A, int lda, const TcWeights& W, const GemmParam
     const int mc = max_clusters<EPI>(S, smem);
     if (mc <= 0) continue;
     const int waves = (units + mc - 1) / mc;
-    const double cost = waves * (static_cast<double>((sh.nkb + S - 1) / S) + 2.0);
+    const double cost = waves * (static_cast<double>((sh.nkb + S - 1) / S) + wave_cost);
     if (cost < best_cost - 1e-9) {
       best_cost = cost;
       best = S;

@@ -171,9 +171,10 @@ __device__ __forceinline__ uint32_t order_key(float f) {
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
-constexpr int kSelThreads = 1024;
-
-// One block per sequence.  Radix select (4 passes of 8 bits) finds the key T of
+// One block per sequence, of THREADS threads (256 to 1024, by the sequence
+// length: the selection is a chain of block-wide barriers, which cost less in
+// a smaller block, and a 1024-thread block left most of its threads idle on
+// the few hundred kept rows of the deep pruned layers).  Radix select (4 passes of 8 bits) finds the key T of
 // the need-th best candidate and how many candidates equal to T are taken;
 // then an index-ordered ballot/prefix scan writes the kept indices ascending.
 // Ties (equal keys) keep lower indices first.  With force_last the last index
@@ -181,8 +182,8 @@ constexpr int kSelThreads = 1024;
 // FROM_PARTS: the scores are first summed from column-mass partials
 // parts[qc][b][g][j] (n_qc chunks, G groups) into shared memory (and copied to
 // scores_out when it is not null); otherwise they are read from `scores`.
-template <bool FROM_PARTS>
-__global__ void __launch_bounds__(kSelThreads)
+template <bool FROM_PARTS, int THREADS>
+__global__ void __launch_bounds__(THREADS)
     select_topk_kernel(const float* __restrict__ scores, int Ns, int ks, int force_last,
                        int32_t* __restrict__ idx_out, const float* __restrict__ parts, int n_qc,
                        int B, int G, float* __restrict__ scores_out, const int* __restrict__ cu_in,
@@ -197,12 +198,12 @@ __global__ void __launch_bounds__(kSelThreads)
   const int k = cu_out ? cu_out[b + 1] - cu_out[b] : ks;
   const size_t sc_row0 = cu_in ? static_cast<size_t>(cu_in[b]) : static_cast<size_t>(b) * Ns;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  constexpr int nwarps = kSelThreads / 32;
+  constexpr int nwarps = THREADS / 32;
   extern __shared__ float sscore[];
   const float* s = scores + static_cast<size_t>(b) * N;
   if (FROM_PARTS) {
     const size_t plane = static_cast<size_t>(B) * G * Ns;
-    for (int j = tid; j < N; j += kSelThreads) {
+    for (int j = tid; j < N; j += THREADS) {
       float acc = 0.f;
       for (int qc = 0; qc < n_qc; ++qc)
         for (int g = 0; g < G; ++g) acc += parts[qc * plane + (static_cast<size_t>(b) * G + g) * Ns + j];
@@ -228,9 +229,9 @@ __global__ void __launch_bounds__(kSelThreads)
   if (need > 0) {
     for (int pass = 0; pass < 4; ++pass) {
       const int shift = 24 - 8 * pass;
-      for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0;
+      for (int i = tid; i < 256; i += THREADS) hist[i] = 0;
       __syncthreads();
-      for (int j = tid; j < n_cand; j += kSelThreads) {
+      for (int j = tid; j < n_cand; j += THREADS) {
         if (al != nullptr && al[j] == 0) continue;  // masked mode: only unmarked rows compete
         const uint32_t key = order_key(s[j]);
         if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
@@ -269,7 +270,7 @@ __global__ void __launch_bounds__(kSelThreads)
   const uint32_t T = prefix;
   const uint32_t lt_mask = (1u << lane) - 1u;
   int base_gt = 0, base_eq = 0;
-  for (int j0 = 0; j0 < n_cand && need > 0; j0 += kSelThreads) {
+  for (int j0 = 0; j0 < n_cand && need > 0; j0 += THREADS) {
     const int j = j0 + tid;
     const bool in = j < n_cand && (al == nullptr || al[j] != 0);
     const uint32_t key = in ? order_key(s[j]) : 0u;
@@ -282,7 +283,7 @@ __global__ void __launch_bounds__(kSelThreads)
     }
     __syncthreads();
     if (warp == 0) {  // exclusive scan of the per-warp counts
-      int a = wgt[lane], e = weq[lane];
+      int a = lane < nwarps ? wgt[lane] : 0, e = lane < nwarps ? weq[lane] : 0;
       int ia = a, ie = e;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
@@ -292,8 +293,10 @@ __global__ void __launch_bounds__(kSelThreads)
           ie += ve;
         }
       }
-      wgt[lane] = ia - a;
-      weq[lane] = ie - e;
+      if (lane < nwarps) {
+        wgt[lane] = ia - a;
+        weq[lane] = ie - e;
+      }
       if (lane == 31) {
         tile_gt = ia;
         tile_eq = ie;
@@ -311,9 +314,9 @@ __global__ void __launch_bounds__(kSelThreads)
   if (force_last && tid == 0) out[k - 1] = N - 1;
   if (al != nullptr) {  // the kept rows stay unmarked, every other row is marked
     __syncthreads();
-    for (int j = tid; j < N; j += kSelThreads) al[j] = 0;
+    for (int j = tid; j < N; j += THREADS) al[j] = 0;
     __syncthreads();
-    for (int r = tid; r < k; r += kSelThreads) al[out[r]] = 1;
+    for (int r = tid; r < k; r += THREADS) al[out[r]] = 1;
   }
 }
 
@@ -568,27 +571,53 @@ cudaError_t launch_row_norm(int dtype, const void* h, int rows, int d, float* sc
   return cudaGetLastError();
 }
 
+// Threads of a selection block for sequences of up to N rows.
+inline int sel_threads(int N) { return N <= 512 ? 256 : (N <= 2048 ? 512 : 1024); }
+
+template <bool FROM_PARTS, int T>
+cudaError_t launch_select_t(const float* scores, const float* parts, int n_qc, int B, int G, int N, int k,
+                            int force_last, int32_t* idx, float* scores_out, size_t smem, cudaStream_t s,
+                            const int* cu_in, const int* cu_out, uint8_t* alive) {
+  if (FROM_PARTS) {
+    static OncePerDevice once;
+    const cudaError_t attr = set_smem_limit_once(once, select_topk_kernel<true, T>,
+                                                 static_cast<int>(kSelectPartsMaxN * sizeof(float)));
+    if (attr != cudaSuccess) return attr;
+  }
+  ZSAA_LAUNCH(select_topk_kernel<FROM_PARTS, T>, dim3(B), dim3(T), smem, s, scores, N, k, force_last, idx, parts,
+              n_qc, B, G, scores_out, cu_in, cu_out, alive);
+  return cudaGetLastError();
+}
+
+template <bool FROM_PARTS>
+cudaError_t launch_select_any(const float* scores, const float* parts, int n_qc, int B, int G, int N, int k,
+                              int force_last, int32_t* idx, float* scores_out, size_t smem, cudaStream_t s,
+                              const int* cu_in, const int* cu_out, uint8_t* alive) {
+  switch (sel_threads(N)) {
+    case 256:
+      return launch_select_t<FROM_PARTS, 256>(scores, parts, n_qc, B, G, N, k, force_last, idx, scores_out, smem,
+                                              s, cu_in, cu_out, alive);
+    case 512:
+      return launch_select_t<FROM_PARTS, 512>(scores, parts, n_qc, B, G, N, k, force_last, idx, scores_out, smem,
+                                              s, cu_in, cu_out, alive);
+    default:
+      return launch_select_t<FROM_PARTS, 1024>(scores, parts, n_qc, B, G, N, k, force_last, idx, scores_out,
+                                               smem, s, cu_in, cu_out, alive);
+  }
+}
+
 cudaError_t launch_select(const float* scores, int B, int N, int k, int force_last, int32_t* idx,
                           cudaStream_t s) {
-  ZSAA_LAUNCH(select_topk_kernel<false>, dim3(B), dim3(kSelThreads), 0, s, scores, N, k, force_last,
-              idx, static_cast<const float*>(nullptr), 0, B, 0, static_cast<float*>(nullptr),
-              static_cast<const int*>(nullptr), static_cast<const int*>(nullptr),
-              static_cast<uint8_t*>(nullptr));
-  return cudaGetLastError();
+  return launch_select_any<false>(scores, nullptr, 0, B, 0, N, k, force_last, idx, nullptr, 0, s, nullptr, nullptr,
+                                  nullptr);
 }
 
 cudaError_t launch_select_parts(const float* parts, int n_qc, int B, int G, int N, int k,
                                 int force_last, int32_t* idx, float* scores_out, cudaStream_t s,
                                 const int* cu_in, const int* cu_out, uint8_t* alive) {
   const size_t smem = static_cast<size_t>(N) * sizeof(float);
-  static OncePerDevice once;
-  const cudaError_t attr = set_smem_limit_once(once, select_topk_kernel<true>,
-                                               static_cast<int>(kSelectPartsMaxN * sizeof(float)));
-  if (attr != cudaSuccess) return attr;
-  ZSAA_LAUNCH(select_topk_kernel<true>, dim3(B), dim3(kSelThreads), smem, s,
-              static_cast<const float*>(nullptr), N, k, force_last, idx, parts, n_qc, B, G, scores_out,
-              cu_in, cu_out, alive);
-  return cudaGetLastError();
+  return launch_select_any<true>(nullptr, parts, n_qc, B, G, N, k, force_last, idx, scores_out, smem, s, cu_in,
+                                 cu_out, alive);
 }
 
 cudaError_t launch_flags_from_idx(const int32_t* idx, int B, int N, int k, uint8_t* flags,
