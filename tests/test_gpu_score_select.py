@@ -121,16 +121,26 @@ def test_score_select_f32_rows(z):
     assert torch.equal(gath, torch.gather(hidden, 1, idx.long()[:, :, None].expand(B, k, d)))
 
 
-@pytest.mark.parametrize("accel", [1.5, 11.0])
-def test_score_select_full_microbench_size(z, accel):
+@pytest.mark.parametrize("accel,keep_scores", [(1.5, True), (11.0, True), (4.0, False)])
+def test_score_select_full_microbench_size(z, accel, keep_scores):
+    # 1 GiB of hidden rows, eight times L2; without kept scores the scores go
+    # to a scratch buffer of the call's own.
     wl = I.WORKLOADS["microbench"]
     B, L, d = wl["B"], wl["L"], wl["d"]
     k = int(L // accel)
     hidden = I.make_hidden(B, L, d, device="cuda")
     idx = torch.empty(B, k, device="cuda", dtype=torch.int32)
-    scores = torch.empty(B, L, device="cuda", dtype=torch.float32)
     gath = torch.empty(B, k, d, device="cuda", dtype=torch.bfloat16)
-    z.zsaa_score_select_ex(hidden, B, L, d, z.ZSAA_BF16, k, 0, None, scores, idx, gath)
+    if keep_scores:
+        scores = torch.empty(B, L, device="cuda", dtype=torch.float32)
+        z.zsaa_score_select_ex(hidden, B, L, d, z.ZSAA_BF16, k, 0, None, scores, idx, gath)
+    else:
+        z.zsaa_score_select(hidden, B, L, d, k, idx, gath)
+        scores = torch.empty(B, L, device="cuda", dtype=torch.float32)
+        idx_ref = torch.empty_like(idx)
+        z.zsaa_score_select_ex(hidden, B, L, d, z.ZSAA_BF16, k, 0, None, scores, idx_ref, None)
+        torch.cuda.synchronize()
+        assert torch.equal(idx, idx_ref)
     torch.cuda.synchronize()
     sample = [0, 17, 31]
     hs = hidden[sample].float().cpu().numpy()
