@@ -614,7 +614,7 @@ bool swap_supported(const void* A, int lda, const TcWeights& W, int epi, const G
   return true;
 }
 
-bool swap_preferred(int epi, int M, int N) {
+bool swap_preferred(int epi, int M, int N, int K) {
   // Crossovers measured on GB300 for the Llama-3.2-1B and -8B projections
   // (CUDA-graph timed, weights streamed from HBM): above these row counts the
   // persistent tiled kernel keeps more SMs busy (SwiGLU needs two waves of
@@ -622,6 +622,16 @@ bool swap_preferred(int epi, int M, int N) {
   // float32 outputs (LM heads, N >= 32768) stream their weights faster on the
   // tiled kernel at every row count (1B head at 40..456 rows: 0.68..0.94x).
   if (epi == kEpiStoreF32 && N >= 32768) return false;
+  // Wide and deep weights (N, K >= 4096: every 8B projection) give the tiled
+  // kernel at least 16 column tiles and 64 k-blocks per tile, and a third
+  // 256-row block doubles the swapped kernel's weight passes: there the tiled
+  // kernel wins from 268 rows (QKV + RoPE: 25.2 vs 25.7 us), 516 rows (O and
+  // down + residual: 27.4 vs 28.9 us, 73.5 vs 92.3 us) and for SwiGLU at any
+  // row count (20 rows: 45.9 vs 46.4 us; 220 rows: 56.7 vs 74.8 us).
+  if (N >= 4096 && K >= 4096) {
+    const int wide_limit = epi == kEpiSwiGLU ? 0 : (epi == kEpiResid ? 512 : 256);
+    return M <= wide_limit;
+  }
   const int limit = epi == kEpiSwiGLU ? 256 : (epi == kEpiResid ? 1024 : 768);
   return M <= limit;
 }

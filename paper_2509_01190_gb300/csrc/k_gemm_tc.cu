@@ -617,6 +617,8 @@ constexpr int P_STAGE_BYTES = P_A_BYTES + P_B_BYTES;
 constexpr size_t P_SMEM = static_cast<size_t>(P_STAGES) * P_STAGE_BYTES + 1024 + 256;
 constexpr uint32_t P_TMEM_COLS = 2 * P_BN;  // two accumulators
 constexpr double kPairTileCost = 0.9;
+// K of at least this many 64-deep k-blocks counts as deep in the tile plan.
+constexpr int kDeepKb = 64;
 
 template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -990,84 +992,131 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
   // most SMs; stream the weights instead
   if (skinny_supported(A, lda, W, epi, p)) return launch_gemm_skinny(A, lda, W, epi, p, s);
   // a few hundred rows: weight band as the 128-row operand, K split over a cluster
-  if (swap_preferred(epi, p.M, p.N) && swap_supported(A, lda, W, epi, p))
+  if (swap_preferred(epi, p.M, p.N, p.K) && swap_supported(A, lda, W, epi, p))
     return launch_gemm_swap(A, lda, W, epi, p, s);
   const int sms = num_sms();
   const int vn = epi == kEpiSwiGLU ? 2 * p.N : p.N;
   const int m_tiles = (p.M + BM - 1) / BM;
-  // Tile width by problem size, from sweeps of the pruned-prefill shapes on
-  // GB300 (graph-timed): narrow tiles only while M is small enough that wide
-  // ones leave most SMs idle; the SwiGLU GEMM (2x the columns) always wide.
-  // (also wide whenever there are two waves of wide tiles: the LM head's
-  // 128256 columns would otherwise re-read the activation thousands of times)
-  const long wide_tiles = static_cast<long>(m_tiles) * ((vn + 255) / 256);
-  const int want = (epi == kEpiSwiGLU || wide_tiles >= 2L * sms)
-                       ? 256
-                       : (p.M <= 256 ? 64 : (p.M <= 768 ? 128 : 256));
+  const int num_kb = p.K / BK;
+  const int slots = (pairs_enabled() && bn_ok(P_BN, epi, W, p)) ? pair_slots_for(epi) : 0;
   int BN = 0;
-  for (int cand : {64, 128, 256})
-    if (bn_ok(cand, epi, W, p) && (BN == 0 || cand <= want)) BN = cand;
-  if (BN == 0) return cudaErrorInvalidValue;
+  bool plan_pairs = false;
+  if (num_kb >= kDeepKb) {
+    // Deep K (>= 64 k-blocks: every 8B projection, the 1B down projection):
+    // the plan with the least waves x cost of one k-block step -- one-CTA
+    // tiles 128 or 256 wide, or 256 x 256 tiles on CTA pairs (only with two
+    // or more 128-row tiles: a lone one would leave half of each pair tile
+    // empty).  The step costs are GB300 graph-timed averages over the 1B and
+    // 8B pruned-forward shapes with every SM streaming: 0.27 us (128-wide)
+    // and 0.36 us (256-wide) per 64-deep k-block, 0.34 us per pair step.
+    // Narrow tiles win only while they still fit one wave (8B QKV at 316
+    // rows: 25.2 us against 30.1 on pairs); pairs win while they add no wave
+    // (8B O at 744 rows: 27.7 us against 33.0 on the swapped kernel).
+    double best = 1e30;
+    for (int cand : {128, 256}) {
+      if (!bn_ok(cand, epi, W, p)) continue;
+      const long tiles = static_cast<long>(m_tiles) * ((vn + cand - 1) / cand);
+      const double cost = static_cast<double>((tiles + sms - 1) / sms) * (cand == 256 ? 0.36 : 0.27);
+      if (cost < best - 1e-9) {
+        best = cost;
+        BN = cand;
+      }
+    }
+    if (slots > 0 && m_tiles >= 2) {
+      const long ptiles = static_cast<long>((m_tiles + 1) / 2) * ((vn + P_BN - 1) / P_BN);
+      const double cost = static_cast<double>((ptiles + slots - 1) / slots) * 0.34;
+      if (cost < best - 1e-9) {
+        BN = P_BN;
+        plan_pairs = true;
+      }
+    }
+  }
+  if (BN == 0) {
+    // Tile width by problem size, from sweeps of the pruned-prefill shapes on
+    // GB300 (graph-timed): narrow tiles only while M is small enough that wide
+    // ones leave most SMs idle; the SwiGLU GEMM (2x the columns) always wide.
+    // (also wide whenever there are two waves of wide tiles: the LM head's
+    // 128256 columns would otherwise re-read the activation thousands of times)
+    const long wide_tiles = static_cast<long>(m_tiles) * ((vn + 255) / 256);
+    const int want = (epi == kEpiSwiGLU || wide_tiles >= 2L * sms)
+                         ? 256
+                         : (p.M <= 256 ? 64 : (p.M <= 768 ? 128 : 256));
+    for (int cand : {64, 128, 256})
+      if (bn_ok(cand, epi, W, p) && (BN == 0 || cand <= want)) BN = cand;
+    if (BN == 0) return cudaErrorInvalidValue;
+  }
   TileSched ts{};
   ts.m_tiles = m_tiles;
   ts.n_tiles = (vn + BN - 1) / BN;
-  ts.num_kb = p.K / BK;
+  ts.num_kb = num_kb;
   ts.total = ts.m_tiles * ts.n_tiles;
   ts.ws = p.splitk_ws;
   ts.flags = p.splitk_flags;
+  // Whole tiles, except with deep K and a ragged last wave of two or more:
+  // then stream-K over the last one-to-two waves (or over everything, for
+  // problems smaller than two waves), splitting k-blocks so no SM idles.
+  // Measured on GB300: the split pays at 128 and 224 k-blocks from a quarter
+  // of the last wave's SM-time idle (8B down at 1196 rows: 99.2 us split
+  // against 140.3 whole), but at 64 k-blocks only from 40% idle (8B QKV at
+  // 1732 rows, 26% idle: 79.3 split against 65.3 whole; 8B O at 1204 rows,
+  // 47% idle: 43.5 against 46.7), and never within one wave, where it only
+  // adds the partial hand-off (8B down at 744 rows: 81.5 against 74.6).
+  const double split_idle = num_kb >= 2 * kDeepKb ? 0.25 : 0.40;
   int grid;
-  // Whole tiles unless K is deep (>= 64 k-blocks, the MLP down projection) and
-  // the last wave of whole tiles would leave over a quarter of the SM-time
-  // idle; then stream-K over the last one-to-two waves (or over everything,
-  // for problems smaller than a wave).  Measured: stream-K loses to whole tiles
-  // at K = 2048 (the partial hand-off costs more than the tail it removes).
-  const int waves = (ts.total + sms - 1) / sms;
-  const double idle = 1.0 - static_cast<double>(ts.total) / (static_cast<double>(waves) * sms);
-  const bool can_split = p.splitk_ws != nullptr && p.splitk_flags != nullptr && sms <= kMaxGemmCtas &&
-                         static_cast<size_t>(sms) * BM * BN <= p.splitk_ws_elems;
-  if (!can_split || idle <= 0.25 || ts.num_kb < 64) {
-    ts.dp_tiles = ts.total;
-    ts.sk_iters = 0;
-    grid = ts.total < sms ? ts.total : sms;
-  } else {
-    ts.dp_tiles = ts.total >= 2 * sms ? (ts.total / sms - 1) * sms : 0;
-    ts.sk_iters = static_cast<long long>(ts.total - ts.dp_tiles) * ts.num_kb;
-    grid = sms;
-    if (ts.dp_tiles == 0) {  // small problem: keep at least 8 k-blocks per CTA
-      const long long g = ts.sk_iters / 8;
-      grid = static_cast<int>(g < 1 ? 1 : (g < sms ? g : sms));
+  {
+    const int waves = (ts.total + sms - 1) / sms;
+    const double idle = 1.0 - static_cast<double>(ts.total) / (static_cast<double>(waves) * sms);
+    const bool can_split = p.splitk_ws != nullptr && p.splitk_flags != nullptr && sms <= kMaxGemmCtas &&
+                           static_cast<size_t>(sms) * BM * BN <= p.splitk_ws_elems;
+    if (plan_pairs || !can_split || num_kb < kDeepKb || waves < 2 || idle <= split_idle) {
+      ts.dp_tiles = ts.total;
+      ts.sk_iters = 0;
+      grid = ts.total < sms ? ts.total : sms;
+    } else {
+      ts.dp_tiles = ts.total >= 2 * sms ? (ts.total / sms - 1) * sms : 0;
+      ts.sk_iters = static_cast<long long>(ts.total - ts.dp_tiles) * ts.num_kb;
+      grid = sms;
+      if (ts.dp_tiles == 0) {  // small problem: keep at least 8 k-blocks per CTA
+        const long long g = ts.sk_iters / 8;
+        grid = static_cast<int>(g < 1 ? 1 : (g < sms ? g : sms));
+      }
     }
   }
-  // CTA pairs (256 x 256 tiles on the 2-SM MMA) for whole-tile problems of
-  // several waves: per MMA step each SM streams 32 KB of operands instead of
-  // 48 KB, the stream that limits the one-CTA kernel at many rows.  Measured on
-  // GB300 (Llama-3.2-1B and -8B projections, 288..8192 rows, graph-timed): a
+  // CTA pairs (256 x 256 tiles on the 2-SM MMA): per MMA step each SM streams
+  // 32 KB of operands instead of 48 KB, the stream that limits the one-CTA
+  // kernel at many rows.  With deep K the plan above decides; otherwise
+  // (measured on the Llama-3.2-1B projections at K = 2048, 288..4096 rows) a
   // pair wave takes 0.84..0.96 of a one-CTA wave, but pairing 128-row tiles
   // can leave half a pair empty and add a wave, and in a single short-K wave
   // the pair's extra synchronisation costs 1..4%, so pairs are taken when they
-  // save waves at kPairTileCost each, and in one wave only for deep K.  Where
-  // the one-CTA plan splits the last waves' k-blocks (deep K, ragged last
-  // wave), the pairs split them instead.
+  // save waves at kPairTileCost each.
   TileSched ps{};
   int pairs = 0;
-  if (BN == P_BN && pairs_enabled()) {
-    const int slots = pair_slots_for(epi);
+  if (BN == P_BN && slots > 0) {
     ps.m_tiles = (m_tiles + 1) / 2;  // 256-row tiles
     ps.n_tiles = ts.n_tiles;
     ps.num_kb = ts.num_kb;
     ps.total = ps.m_tiles * ps.n_tiles;
     ps.ws = ts.ws;
     ps.flags = ts.flags;
-    if (slots > 0 && ts.sk_iters == 0) {
-      const int waves_pair = (ps.total + slots - 1) / slots;
+    const int waves_pair = (ps.total + slots - 1) / slots;
+    const double pair_idle = 1.0 - static_cast<double>(ps.total) / (static_cast<double>(waves_pair) * slots);
+    const bool pair_split_ok = 2 * slots <= kMaxGemmCtas &&
+                               static_cast<size_t>(2 * slots) * BM * P_BN <= p.splitk_ws_elems &&
+                               p.splitk_ws != nullptr && p.splitk_flags != nullptr;
+    bool whole = false, split = false;
+    if (plan_pairs) {
+      split = pair_split_ok && waves_pair >= 2 && pair_idle > split_idle;
+      whole = !split;
+    } else if (num_kb < kDeepKb) {
       const int waves_one = (ts.total + sms - 1) / sms;
-      if (waves_pair * kPairTileCost < waves_one && (waves_one >= 2 || ps.num_kb >= 64)) {
-        ps.dp_tiles = ps.total;
-        ps.sk_iters = 0;
-        pairs = ps.total < slots ? ps.total : slots;
-      }
-    } else if (slots > 0 && 2 * slots <= kMaxGemmCtas &&
-               static_cast<size_t>(2 * slots) * BM * P_BN <= p.splitk_ws_elems) {
+      whole = waves_pair * kPairTileCost < waves_one && waves_one >= 2;
+    }
+    if (whole) {
+      ps.dp_tiles = ps.total;
+      ps.sk_iters = 0;
+      pairs = ps.total < slots ? ps.total : slots;
+    } else if (split) {
       // deep K with a ragged last wave: the same stream-K split over the pairs
       pairs = slots;
       ps.dp_tiles = ps.total >= 2 * pairs ? (ps.total / pairs - 1) * pairs : 0;

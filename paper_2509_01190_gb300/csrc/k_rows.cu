@@ -202,11 +202,31 @@ __global__ void __launch_bounds__(THREADS)
   extern __shared__ float sscore[];
   const float* s = scores + static_cast<size_t>(b) * N;
   if (FROM_PARTS) {
+    // Partial t = qc * G + g lives at parts + qc * plane + (b * G + g) * Ns;
+    // the sum runs over t in increasing order.  The loads are issued kSumBatch
+    // at a time, ahead of their adds, so the chain waits for L2 once per
+    // batch instead of once per partial (the adds keep their order).
+    constexpr int kSumBatch = 16;
     const size_t plane = static_cast<size_t>(B) * G * Ns;
+    const int np = n_qc * G;
+    const float* pb = parts + static_cast<size_t>(b) * G * Ns;
     for (int j = tid; j < N; j += THREADS) {
       float acc = 0.f;
-      for (int qc = 0; qc < n_qc; ++qc)
-        for (int g = 0; g < G; ++g) acc += parts[qc * plane + (static_cast<size_t>(b) * G + g) * Ns + j];
+      int t = 0;
+      for (; t + kSumBatch <= np; t += kSumBatch) {
+        float v[kSumBatch];
+#pragma unroll
+        for (int u = 0; u < kSumBatch; ++u) {
+          const int qc = (t + u) / G, g = t + u - qc * G;
+          v[u] = pb[qc * plane + static_cast<size_t>(g) * Ns + j];
+        }
+#pragma unroll
+        for (int u = 0; u < kSumBatch; ++u) acc += v[u];
+      }
+      for (; t < np; ++t) {
+        const int qc = t / G, g = t - qc * G;
+        acc += pb[qc * plane + static_cast<size_t>(g) * Ns + j];
+      }
       sscore[j] = acc;
       if (scores_out != nullptr) scores_out[sc_row0 + j] = acc;
     }

@@ -123,7 +123,7 @@ constexpr int kSwapRowBlock = 256;
 bool swap_supported(const void* A, int lda, const TcWeights& W, int epi, const GemmParams& p);
 // Whether launch_gemm_tc takes the swapped kernel for this epilogue, row count
 // and output width (wide float32 heads go to the tiled kernel).
-bool swap_preferred(int epi, int M, int N);
+bool swap_preferred(int epi, int M, int N, int K);
 cudaError_t launch_gemm_swap(const void* A, int lda, const TcWeights& W, int epi,
                              const GemmParams& p, cudaStream_t s);
 

@@ -16,12 +16,13 @@ pytestmark = pytest.mark.gpu
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
-# (epilogue, M, N, K): whole tiles (two waves), then deep K split over the CTAs
-# (1100 x 1040: 45 tiles of 64 k-blocks over all SMs; 5000 x 2048: one wave
-# whole, the rest split; the 1B down projection at 3296 rows)
+# (epilogue, M, N, K): whole tiles (two waves; 5000 x 2048 at K = 4096: 320
+# tiles, a full last wave), then deep K split over the CTAs where the last of
+# two or more waves is ragged (1204 rows: 160 tiles of 64 k-blocks; 1700 rows of
+# RoPE: 168; the 1B down projection at 3296 rows: 208 tiles of 128 k-blocks)
 CASES = [("store", 2056, 2064, 512), ("swiglu", 2300, 1088, 512), ("rope", 2300, 3072, 512),
-         ("store_f32", 1100, 1040, 4096), ("resid", 5000, 2048, 4096), ("swiglu", 1100, 1088, 4096),
-         ("rope", 1100, 3072, 4096), ("resid", 3296, 2048, 8192)]
+         ("store_f32", 1204, 4096, 4096), ("resid", 5000, 2048, 4096), ("swiglu", 1204, 2048, 4096),
+         ("rope", 1700, 3072, 4096), ("resid", 3296, 2048, 8192)]
 
 
 def _run_cases():

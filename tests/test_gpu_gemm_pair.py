@@ -78,25 +78,26 @@ def test_pair_deterministic(z):
 
 
 
-# Deep K (64 k-blocks and more) with a ragged last wave: the last tiles' k-blocks
-# are split over the pairs.  1100 rows x 1040 columns: 25 pair tiles over all
-# pairs, so most tiles have three or four contributing pairs; 5000 rows x 2048:
-# whole tiles for one wave of pairs, the rest split.
-@pytest.mark.parametrize("M,N", [(1100, 1040), (5000, 2048)])
+# Deep K with two or more waves of pair tiles and a ragged last one: the last
+# tiles' k-blocks are split over the pairs (from 40% of the last wave idle at
+# 64 k-blocks, 25% at 128 and more).  1204 rows x 4096 columns at K = 4096: 80
+# pair tiles (5 x 16), fewer than two waves, so every tile is split, over one
+# or two pairs; 2440 x 2048 at K = 8192: 80 pair tiles of 128 k-blocks.
+@pytest.mark.parametrize("M,N,K", [(1204, 4096, 4096), (2440, 2048, 8192)])
 @pytest.mark.parametrize("epi", ["store_f32", "resid"])
-def test_pair_streamk_plain(z, epi, M, N):
-    out, ref, tol = linear_case(z, epi, M, N, 4096, 1000 + M + N)
-    check_linear(out, ref, tol, epi, f"{epi} M={M} N={N}")
+def test_pair_streamk_plain(z, epi, M, N, K):
+    out, ref, tol = linear_case(z, epi, M, N, K, 1000 + M + N)
+    check_linear(out, ref, tol, epi, f"{epi} M={M} N={N} K={K}")
 
 
 def test_pair_streamk_swiglu(z):
-    out, ref, tol = linear_case(z, "swiglu", 1100, 1088, 4096, 1100)
-    check_linear(out, ref, tol, "swiglu", "M=1100 K=4096")
+    out, ref, tol = linear_case(z, "swiglu", 1204, 2048, 4096, 1100)
+    check_linear(out, ref, tol, "swiglu", "M=1204 K=4096")
 
 
 def test_pair_streamk_rope(z):
-    # Llama-3.1-8B QKV layout: 16 query + 4 key heads rotated, 4 value heads, hd 128
-    out, ref, tol = linear_case(z, "rope", 1100, 3072, 4096, 1200, hd=128, rope_cols=2560)
+    # 16 query + 4 key heads rotated, 4 value heads, hd 128: 84 pair tiles (7 x 12)
+    out, ref, tol = linear_case(z, "rope", 1700, 3072, 4096, 1200, hd=128, rope_cols=2560)
     check_linear(out, ref, tol, "rope", "hd=128 K=4096")
 
 
@@ -106,9 +107,24 @@ def test_pair_streamk_down_1b(z):
     check_linear(out, ref, tol, "resid", "down M=3296")
 
 
+# Deep-K plans of the pruned Llama-3.1-8B forward at a few hundred rows, one
+# wave each: whole pair tiles (down-like, 48 pair tiles of 128 k-blocks),
+# 128-wide one-CTA tiles (QKV + RoPE, hd 128, 144 tiles) and 256-wide one-CTA
+# tiles for a single 128-row tile (gate/up + SwiGLU, 112 tiles).
+EIGHT_B_TILED = [("resid", 744, 4096, 8192, 64, 0), ("rope", 316, 6144, 4096, 128, 5120),
+                 ("swiglu", 92, 14336, 4096, 64, 0)]
+
+
+@pytest.mark.parametrize("epi,M,N,K,hd,rope_cols", EIGHT_B_TILED)
+def test_deep_k_one_wave_plans(z, epi, M, N, K, hd, rope_cols):
+    kw = dict(hd=hd, rope_cols=rope_cols) if epi == "rope" else {}
+    out, ref, tol = linear_case(z, epi, M, N, K, 1500 + M, **kw)
+    check_linear(out, ref, tol, epi, f"{epi} M={M} N={N} K={K}")
+
+
 def test_pair_streamk_deterministic(z):
     # split tiles add their partials in pair order: repeated calls agree bit for bit
-    M, N, K = 1100, 1040, 4096
+    M, N, K = 1204, 4096, 4096
     A = rand_bf16((M, K), 21)
     W = rand_bf16((N, K), 22, 0.05)
     outs = []

@@ -57,6 +57,18 @@ def test_swap_deep_1b_shapes(z, name, M, N, K):
     check_linear(out, ref, tol, epi, f"{name} M={M}")
 
 
+# The 8B projections below their crossovers to the tiled kernel (N, K >= 4096:
+# RoPE up to 256 rows, residual up to 512): QKV, O, and down with 14336-deep K.
+DEEP_8B = [("rope", 192, 6144, 4096), ("resid", 456, 4096, 4096), ("resid", 300, 4096, 14336)]
+
+
+@pytest.mark.parametrize("epi,M,N,K", DEEP_8B)
+def test_swap_deep_8b_shapes(z, epi, M, N, K):
+    kw = dict(hd=128, rope_cols=5120) if epi == "rope" else {}
+    out, ref, tol = linear_case(z, epi, M, N, K, 450 + M, **kw)
+    check_linear(out, ref, tol, epi, f"{epi} M={M} N={N} K={K}")
+
+
 def test_swap_deterministic(z):
     # the cluster adds its partial sums in rank order: repeated calls agree bit for bit
     M, N, K = 200, 2048, 4096
