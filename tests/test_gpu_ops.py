@@ -276,7 +276,36 @@ def _oracle_attention(qkv, B, N, Hq, Hkv, hd, causal=True):
                                            (2, 129, 8, 2, 128), (2, 255, 8, 2, 64), (1, 2048, 8, 2, 128),
                                            (1, 700, 16, 2, 64)])
 def test_attention_and_colmass_bf16(z, B, N, Hq, Hkv, hd):
-    qkv = _qkv(B, N, Hq, Hkv, hd, 20 + N, torch.bfloat16)
+    _check_attention_bf16(z, _qkv(B, N, Hq, Hkv, hd, 20 + N, torch.bfloat16), B, N, Hq, Hkv, hd)
+
+
+def _growing_scores_qkv(N, Hq, Hkv, hd, seed, rise_log2, wave):
+    """qkv rows whose scores q.k/sqrt(hd) climb along the keys by about
+    rise_log2 (log2 units) over the sequence, plus a wave of that amplitude
+    (wave > 0), so a query's running maximum keeps moving: inside a key block
+    by more than 2^8 (rescaling the block's P already written) and from block
+    to block (rescaling O)."""
+    g = torch.Generator().manual_seed(seed)
+    u = torch.randn(hd, generator=g)
+    u /= u.norm()
+    a = 8.0
+    j = torch.arange(N, dtype=torch.float64)
+    beta = (rise_log2 / 1.4426950408889634) * math.sqrt(hd) / a
+    amp = beta * (j / N + wave * torch.sin(j / 23.0))
+    x = 0.05 * torch.randn(N, Hq + 2 * Hkv, hd, generator=g, dtype=torch.float64)
+    x[:, :Hq] += a * u.double()
+    x[:, Hq:Hq + Hkv] += amp[:, None, None] * u.double()
+    return x.reshape(N, -1).to(torch.bfloat16).cuda()
+
+
+@pytest.mark.parametrize("hd,rise,wave", [(64, 150.0, 0.0), (128, 150.0, 0.0), (64, 60.0, 0.4),
+                                          (128, 400.0, 0.3)])
+def test_attention_running_max_rescales(z, hd, rise, wave):
+    N, Hq, Hkv = 300, 4, 2
+    _check_attention_bf16(z, _growing_scores_qkv(N, Hq, Hkv, hd, 7 + hd, rise, wave), 1, N, Hq, Hkv, hd)
+
+
+def _check_attention_bf16(z, qkv, B, N, Hq, Hkv, hd):
     out = torch.empty(B * N, Hq * hd, device="cuda", dtype=torch.bfloat16)
     lse = torch.empty(B, Hq, N, device="cuda", dtype=torch.float32)
     z.zsaa_op_attention(qkv, B, N, Hq, Hkv, hd, z.ZSAA_BF16, out, lse)
