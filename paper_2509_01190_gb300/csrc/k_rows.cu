@@ -10,6 +10,9 @@ namespace zsaa {
 namespace {
 
 constexpr int kWarpsPerBlock = 8;
+// Rows of up to 32 * kMaxVecPerLane 16-byte vectors (d <= 4096 in bf16) are
+// held in registers, a lane's vectors all in flight at once.
+constexpr int kMaxVecPerLane = 16;
 
 inline int row_blocks(int rows) { return (rows + kWarpsPerBlock - 1) / kWarpsPerBlock; }
 
@@ -67,7 +70,66 @@ __global__ void rmsnorm_kernel(const T* __restrict__ h, const T* __restrict__ w,
   for (int i = lane; i < d; i += 32) xr[i] = from_f<T>(to_f(hr[i]) * inv * to_f(w[i]));
 }
 
-// bf16 rows, 8 elements per 16-byte vector.
+// The norm weights (vec 16-byte vectors, never written by a kernel) staged in
+// the block's shared memory before the wait for the previous kernel: every
+// warp of the block reads them there instead of from L2.
+__device__ __forceinline__ void stage_norm_weights(const uint4* __restrict__ w, int vec, uint4* sw) {
+  for (int v = threadIdx.x; v < vec; v += blockDim.x) sw[v] = __ldg(w + v);
+  __syncthreads();
+}
+
+// bf16 rows of at most 32 * kMaxVecPerLane vectors: one warp per row, the row
+// loaded into registers once (every load of a lane in flight together), its
+// sum of squares, then x = h / rms * w with the weights from shared memory.
+__global__ void rmsnorm_bf16_reg_kernel(const uint4* __restrict__ h, const uint4* __restrict__ w,
+                                        int rows, int vec, float eps, uint4* __restrict__ x) {
+  extern __shared__ uint4 sw[];
+  pdl_trigger();
+  stage_norm_weights(w, vec, sw);
+  pdl_wait();
+  const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= rows) return;
+  const uint4* hr = h + static_cast<size_t>(r) * vec;
+  uint4* xr = x + static_cast<size_t>(r) * vec;
+  uint4 u[kMaxVecPerLane];
+  float ss = 0.f;
+#pragma unroll
+  for (int q = 0; q < kMaxVecPerLane; ++q) {
+    const int v = lane + 32 * q;
+    if (v < vec) u[q] = hr[v];
+  }
+#pragma unroll
+  for (int q = 0; q < kMaxVecPerLane; ++q) {
+    const int v = lane + 32 * q;
+    if (v < vec) {
+      const uint32_t e4[4] = {u[q].x, u[q].y, u[q].z, u[q].w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float a = bf16lo(e4[e]), c = bf16hi(e4[e]);
+        ss += a * a + c * c;
+      }
+    }
+  }
+  ss = warp_sum(ss);
+  const float inv = rsqrtf(ss / static_cast<float>(vec * 8) + eps);
+#pragma unroll
+  for (int q = 0; q < kMaxVecPerLane; ++q) {
+    const int v = lane + 32 * q;
+    if (v < vec) {
+      const uint4 wv = sw[v];
+      const uint32_t e4[4] = {u[q].x, u[q].y, u[q].z, u[q].w};
+      const uint32_t w4[4] = {wv.x, wv.y, wv.z, wv.w};
+      uint32_t o[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        o[e] = pack_bf16x2(bf16lo(e4[e]) * inv * bf16lo(w4[e]), bf16hi(e4[e]) * inv * bf16hi(w4[e]));
+      xr[v] = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+  }
+}
+
+// bf16 rows, 8 elements per 16-byte vector (any length).
 __global__ void rmsnorm_bf16_vec_kernel(const uint4* __restrict__ h, const uint4* __restrict__ w,
                                         int rows, int vec_per_row, float eps,
                                         uint4* __restrict__ x) {
@@ -401,8 +463,6 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ src, int N, int k, 
 //     pos_in[that row] -- the kept rows of the previous layer, already normed
 //     for the next layer's attention.
 // An index outside its range sets kStatusBadIndex and copies row 0.
-constexpr int kMaxVecPerLane = 16;
-
 __global__ void rows_norm_bf16_kernel(const uint4* __restrict__ src, const int32_t* __restrict__ tok,
                                       int vocab, int L, const int32_t* __restrict__ idx, int N,
                                       int k, const int32_t* __restrict__ pos_in, int rows, int vec,
@@ -411,10 +471,11 @@ __global__ void rows_norm_bf16_kernel(const uint4* __restrict__ src, const int32
                                       int32_t* __restrict__ pos_out, int* status,
                                       const int* __restrict__ cu_src, const int* __restrict__ cu_dst,
                                       int nseq) {
+  extern __shared__ uint4 sw[];
   pdl_trigger();
   const int r = blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
-  if (threadIdx.x < 32) prefetch_norm_weights(w, vec, lane);
+  stage_norm_weights(w, vec, sw);
   pdl_wait();
   if (r >= rows) return;
   size_t srow;
@@ -472,7 +533,7 @@ __global__ void rows_norm_bf16_kernel(const uint4* __restrict__ src, const int32
   for (int q = 0; q < kMaxVecPerLane; ++q) {
     const int v = lane + 32 * q;
     if (v < vec) {
-      const uint4 wv = __ldg(w + v);
+      const uint4 wv = sw[v];
       const uint32_t e4[4] = {u[q].x, u[q].y, u[q].z, u[q].w};
       const uint32_t w4[4] = {wv.x, wv.y, wv.z, wv.w};
       uint32_t o[4];
@@ -563,7 +624,11 @@ cudaError_t launch_embed(int dtype, const void* E, const int32_t* tok, int rows,
 
 cudaError_t launch_rmsnorm(int dtype, const void* h, const void* w, int rows, int d, float eps,
                            void* x, cudaStream_t s) {
-  if (dtype == ZSAA_BF16 && d % 8 == 0) {
+  if (dtype == ZSAA_BF16 && d % 8 == 0 && d / 8 <= 32 * kMaxVecPerLane) {
+    ZSAA_LAUNCH(rmsnorm_bf16_reg_kernel, dim3(row_blocks(rows)), dim3(32 * kWarpsPerBlock),
+                static_cast<size_t>(d / 8) * 16, s, static_cast<const uint4*>(h), static_cast<const uint4*>(w),
+                rows, d / 8, eps, static_cast<uint4*>(x));
+  } else if (dtype == ZSAA_BF16 && d % 8 == 0) {
     ZSAA_LAUNCH(rmsnorm_bf16_vec_kernel, dim3(row_blocks(rows)), dim3(32 * kWarpsPerBlock), 0, s, 
         static_cast<const uint4*>(h), static_cast<const uint4*>(w), rows, d / 8, eps,
         static_cast<uint4*>(x));
@@ -651,7 +716,8 @@ cudaError_t launch_rows_norm(const void* src, const int32_t* tok, int vocab, int
                              int d, const void* w, float eps, void* h_out, void* x_out,
                              int32_t* pos_out, int* status, cudaStream_t s, const int* cu_src,
                              const int* cu_dst, int nseq) {
-  ZSAA_LAUNCH(rows_norm_bf16_kernel, dim3(row_blocks(rows)), dim3(32 * kWarpsPerBlock), 0, s,
+  ZSAA_LAUNCH(rows_norm_bf16_kernel, dim3(row_blocks(rows)), dim3(32 * kWarpsPerBlock),
+              static_cast<size_t>(d / 8) * 16, s,
               static_cast<const uint4*>(src), tok, vocab, L, idx, N, k, pos_in, rows, d / 8,
               static_cast<const uint4*>(w), eps, static_cast<uint4*>(h_out),
               static_cast<uint4*>(x_out), pos_out, status, cu_src, cu_dst, nseq);
