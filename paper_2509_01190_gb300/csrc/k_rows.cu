@@ -274,20 +274,28 @@ __global__ void __launch_bounds__(THREADS)
     const float* pb = parts + static_cast<size_t>(b) * G * Ns;
     for (int j = tid; j < N; j += THREADS) {
       float acc = 0.f;
-      int t = 0;
+      const float* pj = pb + j;
+      int t = 0, g = 0;
+      size_t qoff = 0;  // qc * plane of partial t = qc * G + g
       for (; t + kSumBatch <= np; t += kSumBatch) {
         float v[kSumBatch];
 #pragma unroll
         for (int u = 0; u < kSumBatch; ++u) {
-          const int qc = (t + u) / G, g = t + u - qc * G;
-          v[u] = pb[qc * plane + static_cast<size_t>(g) * Ns + j];
+          v[u] = pj[qoff + static_cast<size_t>(g) * Ns];
+          if (++g == G) {
+            g = 0;
+            qoff += plane;
+          }
         }
 #pragma unroll
         for (int u = 0; u < kSumBatch; ++u) acc += v[u];
       }
       for (; t < np; ++t) {
-        const int qc = t / G, g = t - qc * G;
-        acc += pb[qc * plane + static_cast<size_t>(g) * Ns + j];
+        acc += pj[qoff + static_cast<size_t>(g) * Ns];
+        if (++g == G) {
+          g = 0;
+          qoff += plane;
+        }
       }
       sscore[j] = acc;
       if (scores_out != nullptr) scores_out[sc_row0 + j] = acc;
