@@ -1,16 +1,16 @@
 // bf16 GEMM on the sm_103a tensor cores: out = epi(A[M,K] W[N,K]^T), fp32
 // accumulation in tensor memory.
 //
-// Persistent stream-K kernels: one CTA per SM, or (gemm_pair_kernel, for
-// many rows) one CTA pair per TPC on the 2-SM MMA.  Tiles are 128 x BN (tiles
-// sharing a weight tile are adjacent, so weights stream from HBM once and are
-// re-read from L2).  All but the last one-to-two waves of tiles are handed out
-// whole, round robin; the k-iterations of the remaining tiles are split evenly
-// over all CTAs, so no SM idles in a ragged last wave.  A tile split across
-// CTAs is finished by the CTA holding its first k-block (its last item): the
-// other contributors (for whom it is their first item) write fp32 partials
-// and raise a per-warp flag; the finisher waits (bounded) and adds them in CTA
-// order before the epilogue -- deterministic, no extra launch, no atomics.
+// Persistent kernels: one CTA per SM, or (gemm_pair_kernel, for many rows)
+// one CTA pair per TPC on the 2-SM MMA.  Tiles are 128 x BN (tiles sharing a
+// weight tile are adjacent, so weights stream from HBM once and are re-read
+// from L2).  Whole waves of tiles are handed out round robin; with deep K the
+// tiles of a ragged last wave may instead be cut into S aligned k-parts, dealt
+// part-major so that the units of one round work on the same k-range of
+// neighbouring tiles.  The non-final parts write fp32 partials (one slot each)
+// and raise per-warp flags; the tile's last part waits (bounded) and adds them
+// in part order before the epilogue -- deterministic, no extra launch, no
+// atomics.
 // Warp-specialised roles:
 //   warp 0      TMA producer: 128B-swizzled A and W tiles (64 deep in K) into a
 //               STAGES-deep shared-memory ring ("full" mbarriers, expect-tx);
@@ -27,6 +27,7 @@
 // Every mbarrier wait is bounded (2 s); on expiry the kernel sets the status
 // word, the other roles stop waiting, in-flight copies are drained (bounded)
 // and TMEM is freed before the CTA exits.
+#include <algorithm>
 #include <cstdio>
 #include <cstdlib>
 #include <mutex>
@@ -54,68 +55,101 @@ struct TcMaps {
   CUtensorMap a, b0, b1, b2;
 };
 
-// Work split: tiles [0, dp_tiles) go whole to unit t % units; the k-iterations
-// of tiles [dp_tiles, total) (sk_iters of them, num_kb per tile) are cut into
-// `units` equal contiguous ranges.  Tile t -> (m tile t % m_tiles, n tile
-// t / m_tiles); the pair kernel's m tiles are 256 rows.
+// Work split: tiles [0, dp_tiles) go whole to unit t % units (whole waves).
+// The tiles after them are split in k in one of two ways:
+//   contiguous (sk_iters > 0): their sk_iters k-iterations are cut into
+//     `units` equal contiguous ranges, across tile boundaries;
+//   aligned (tail_R > 0): each of the tail_R tiles is cut into tail_S parts
+//     of equal length (part s: k-blocks [s KB / S, (s + 1) KB / S)); part
+//     q = s * tail_R + r (tile dp_tiles + r) goes to unit q % units, so the
+//     units of a round work on the same k-part of neighbouring tiles.
+// Tile t -> (m tile t % m_tiles, n tile t / m_tiles); the pair kernel's m
+// tiles are 256 rows.
 struct TileSched {
   int m_tiles, n_tiles, num_kb, total, dp_tiles;
   long long sk_iters;
-  float* ws;   // fp32 partial tiles, one BM x BN slot per CTA (slot = blockIdx.x)
-  int* flags;  // per CTA and epilogue warp: 1 while its partial is ready (reset by the reader)
+  int tail_R, tail_S;
+  float* ws;   // fp32 partials: one slot per contiguous unit or aligned non-final part
+  int* flags;  // per slot, CTA of the unit and epilogue warp: 1 while the partial is ready
 };
 
 // One unit of work of a CTA: k-blocks [kb0, kb1) of a tile.
 //   kind 0: the whole tile (epilogue directly);
-//   kind 1: a later part of a split tile (write the partial, raise the flags);
-//   kind 2: the first part of a split tile (add the partials of CTAs
-//           blockIdx.x+1 .. c_hi, then the epilogue).
+//   kind 1: a non-final part of a split tile (write the partial to slot
+//           `slot`, raise the flags);
+//   kind 2: the final part of a split tile (add the `count` partials in
+//           slots slot, slot + stride, ..., in that order; then the epilogue).
 struct Item {
-  int tile, kb0, kb1, kind, c_hi;
+  int tile, kb0, kb1, kind, slot, count, stride;
 };
 
 // Work of unit `unit` of `units` (a CTA of the one-CTA kernel, a CTA pair of
 // the pair kernel; both CTAs of a pair walk the same items).
 struct WorkIter {
-  int t_dp, units;
+  int t_dp, units, unit, q;
   long long it, end;
-  __device__ __forceinline__ void init(const TileSched& ts, int unit, int nunits) {
-    t_dp = unit;
+  __device__ __forceinline__ void init(const TileSched& ts, int u, int nunits) {
+    t_dp = u;
     units = nunits;
+    unit = u;
+    q = u;
     const long long G = nunits;
-    it = static_cast<long long>(unit) * ts.sk_iters / G;
-    end = static_cast<long long>(unit + 1) * ts.sk_iters / G;
+    it = static_cast<long long>(u) * ts.sk_iters / G;
+    end = static_cast<long long>(u + 1) * ts.sk_iters / G;
   }
   __device__ __forceinline__ bool next(const TileSched& ts, Item& w) {
+    w.slot = 0;
+    w.count = 0;
+    w.stride = 1;
     if (t_dp < ts.dp_tiles) {
       w.tile = t_dp;
       w.kb0 = 0;
       w.kb1 = ts.num_kb;
       w.kind = 0;
-      w.c_hi = 0;
       t_dp += units;
       return true;
     }
-    if (it >= end) return false;
     const int KB = ts.num_kb;
-    const long long u = it / KB;
-    const int a = static_cast<int>(it - u * KB);
-    const int b = static_cast<int>(min(static_cast<long long>(KB), a + (end - it)));
-    w.tile = ts.dp_tiles + static_cast<int>(u);
-    w.kb0 = a;
-    w.kb1 = b;
-    w.c_hi = 0;
-    if (a == 0 && b == KB) {
-      w.kind = 0;
-    } else if (a == 0) {
-      // the unit holding iteration x is floor(((x + 1) * units - 1) / sk_iters)
+    if (ts.sk_iters > 0) {
+      if (it >= end) return false;
+      const long long u = it / KB;
+      const int a = static_cast<int>(it - u * KB);
+      const int b = static_cast<int>(min(static_cast<long long>(KB), a + (end - it)));
+      w.tile = ts.dp_tiles + static_cast<int>(u);
+      w.kb0 = a;
+      w.kb1 = b;
+      if (a == 0 && b == KB) {
+        w.kind = 0;
+      } else if (a == 0) {
+        // the tile's later parts are the first items of units unit+1 .. c_hi
+        // (the unit holding iteration x is floor(((x + 1) * units - 1) / sk_iters))
+        w.kind = 2;
+        const long long G = units;
+        const int c_hi = static_cast<int>(((u + 1) * KB * G - 1) / ts.sk_iters);
+        w.slot = unit + 1;
+        w.count = c_hi - unit;
+      } else {
+        w.kind = 1;
+        w.slot = unit;
+      }
+      it += b - a;
+      return true;
+    }
+    if (q >= ts.tail_R * ts.tail_S) return false;
+    const int r = q % ts.tail_R, part = q / ts.tail_R, S = ts.tail_S;
+    w.tile = ts.dp_tiles + r;
+    w.kb0 = part * KB / S;
+    w.kb1 = (part + 1) * KB / S;
+    if (part == S - 1) {
       w.kind = 2;
-      const long long G = units;
-      w.c_hi = static_cast<int>(((u + 1) * KB * G - 1) / ts.sk_iters);
+      w.slot = r;  // parts 0 .. S-2 are in slots r, r + tail_R, ...
+      w.count = S - 1;
+      w.stride = ts.tail_R;
     } else {
       w.kind = 1;
+      w.slot = q;
     }
-    it += b - a;
+    q += units;
     return true;
   }
 };
@@ -543,30 +577,32 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       tc_fence_after();
       const uint32_t tbase = tmem + static_cast<uint32_t>(ab * BN) + (static_cast<uint32_t>(quad * 32) << 16);
+      constexpr size_t kSlot = static_cast<size_t>(BM) * BN;
       if (w.kind == 1) {
-        // a later part of a split tile: hand the partial to the tile's first CTA
-        write_partial<BN>(tbase, ts.ws + static_cast<size_t>(blockIdx.x) * BM * BN, rit);
+        // a non-final k-part of a tail tile: its partial to slot w.slot
+        write_partial<BN>(tbase, ts.ws + static_cast<size_t>(w.slot) * kSlot, rit);
         __threadfence();
         __syncwarp();
         if (lane == 0) {
-          int* f = ts.flags + blockIdx.x * 4 + quad;
+          int* f = ts.flags + w.slot * 4 + quad;
           asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(f), "r"(1) : "memory");
         }
       } else {
-        int c0 = 1, c1 = 0;  // no partials
+        int c1 = -1;  // partials 0 .. c1 (none for a whole tile)
         if (w.kind == 2) {
-          c0 = blockIdx.x + 1;
-          c1 = w.c_hi;
+          c1 = w.count - 1;
           bool got = true;
-          for (int c = c0; c <= c1; ++c)
-            got = got && wait_flag(ts.flags + c * 4 + quad, p.status, abort_flag);
-          if (!__all_sync(0xffffffffu, got)) c1 = c0 - 1;  // gave up: status already set
+          for (int c = 0; c <= c1; ++c)
+            got = got && wait_flag(ts.flags + (w.slot + c * w.stride) * 4 + quad, p.status, abort_flag);
+          if (!__all_sync(0xffffffffu, got)) c1 = -1;  // gave up: status already set
         }
-        tile_epilogue<BN, EPI>(tbase, row, row < p.M, nt * BN, p, ts.ws, static_cast<size_t>(BM) * BN, c0, c1, rit);
+        tile_epilogue<BN, EPI>(tbase, row, row < p.M, nt * BN, p,
+                               c1 >= 0 ? ts.ws + static_cast<size_t>(w.slot) * kSlot : nullptr,
+                               static_cast<size_t>(w.stride) * kSlot, 0, c1, rit);
         if (w.kind == 2) {
           __syncwarp();
           if (lane == 0)
-            for (int c = c0; c <= c1; ++c) ts.flags[c * 4 + quad] = 0;
+            for (int c = 0; c <= c1; ++c) ts.flags[(w.slot + c * w.stride) * 4 + quad] = 0;
         }
       }
       tc_fence_before();
@@ -619,6 +655,10 @@ constexpr uint32_t P_TMEM_COLS = 2 * P_BN;  // two accumulators
 constexpr double kPairTileCost = 0.9;
 // K of at least this many 64-deep k-blocks counts as deep in the tile plan.
 constexpr int kDeepKb = 64;
+// From this many k-blocks on (the 8B down projection, 224) a ragged last wave
+// may be cut into aligned k-parts; below it (1B down, 128; 64) the contiguous
+// stream-K split measured better, or no split at all.
+constexpr int kVeryDeepKb = 192;
 
 template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -790,32 +830,32 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       tc_fence_after();
       const uint32_t tbase = tmem + static_cast<uint32_t>(ab * P_BN) + (static_cast<uint32_t>(quad * 32) << 16);
+      // a pair's slot q holds CTA r's 128 rows at CTA slot 2q + r
       if (w.kind == 1) {
-        // a later part of a split tile: hand this CTA's rows to the tile's first pair
-        write_partial<P_BN>(tbase, ts.ws + static_cast<size_t>(blockIdx.x) * kSlot, rit);
+        // a non-final k-part of a tail tile: this CTA's rows to its slot
+        write_partial<P_BN>(tbase, ts.ws + static_cast<size_t>(2 * w.slot + rank) * kSlot, rit);
         __threadfence();
         __syncwarp();
         if (lane == 0) {
-          int* f = ts.flags + blockIdx.x * 4 + quad;
+          int* f = ts.flags + (2 * w.slot + rank) * 4 + quad;
           asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(f), "r"(1) : "memory");
         }
       } else {
-        int c0 = 1, c1 = 0;  // no partials
+        int c1 = -1;  // partials 0 .. c1 (none for a whole tile)
         if (w.kind == 2) {
-          c0 = pair + 1;
-          c1 = w.c_hi;
+          c1 = w.count - 1;
           bool got = true;
-          for (int c = c0; c <= c1; ++c)
-            got = got && wait_flag(ts.flags + (2 * c + rank) * 4 + quad, p.status, abort_flag);
-          if (!__all_sync(0xffffffffu, got)) c1 = c0 - 1;  // gave up: status already set
+          for (int c = 0; c <= c1; ++c)
+            got = got && wait_flag(ts.flags + (2 * (w.slot + c * w.stride) + rank) * 4 + quad, p.status, abort_flag);
+          if (!__all_sync(0xffffffffu, got)) c1 = -1;  // gave up: status already set
         }
-        // contributor pair c's rows of this CTA are in slot 2c + rank
-        const float* ws = c0 <= c1 ? ts.ws + rank * kSlot : nullptr;
-        tile_epilogue<P_BN, EPI>(tbase, row, row < p.M, nt * P_BN, p, ws, 2 * kSlot, c0, c1, rit);
+        const float* ws = c1 >= 0 ? ts.ws + static_cast<size_t>(2 * w.slot + rank) * kSlot : nullptr;
+        tile_epilogue<P_BN, EPI>(tbase, row, row < p.M, nt * P_BN, p, ws, 2 * static_cast<size_t>(w.stride) * kSlot,
+                                 0, c1, rit);
         if (w.kind == 2) {
           __syncwarp();
           if (lane == 0)
-            for (int c = c0; c <= c1; ++c) ts.flags[(2 * c + rank) * 4 + quad] = 0;
+            for (int c = 0; c <= c1; ++c) ts.flags[(2 * (w.slot + c * w.stride) + rank) * 4 + quad] = 0;
         }
       }
       tc_fence_before();
@@ -983,6 +1023,56 @@ bool bn_ok(int BN, int epi, const TcWeights& W, const GemmParams& p) {
   return true;
 }
 
+// Whether to cut the ragged last wave of a plan into aligned k-parts, from a
+// model fitted to GB300 measurements of forced plans on the 8B projections
+// (graph-timed, weights from HBM): with Tw the time of one full wave,
+//   whole: W Tw + Tw min(1, 0.25 + 4 R / units)  (only a nearly empty last
+//          wave runs faster: 8B down at 1204 rows spent about 25 us on its
+//          last 4 of 76 pair tiles, but 70-73 us on 20, 36 or 52 of them,
+//          as on a full wave);
+//   split: W Tw + Tw / S + 8 us + 5.5 us (S - 1), all R S parts in one round
+//          (one partial written, S - 1 read back by the tile's last part:
+//          17-31 us measured at S = 3..5 on 224 k-blocks; two rounds measured
+//          slower than predicted).
+// So the split pays only on deep K (8B down: 1536 rows 145.5 -> 114.3 us,
+// 5084 rows 397.2 -> 364.2 us); on 64 k-blocks it measured 3-37% slower.
+struct TailPlan {
+  int S;  // k-parts per remainder tile; 1: whole tiles only
+};
+TailPlan tail_plan(int total, int units, int kb, double step_us, bool can_split, int max_slots) {
+  const int W = total / units, R = total - W * units;
+  TailPlan tp{1};
+  if (!can_split || R == 0 || kb < kDeepKb) return tp;
+  const double tw = kb * step_us;
+  double best = tw * std::min(1.0, 0.25 + 4.0 * R / units);
+  for (int S = 2; S <= 8; ++S) {
+    if (kb / S < 8 || R * (S - 1) > max_slots || R * S > units) break;
+    const double t = tw / S + 8.0 + 5.5 * (S - 1);
+    if (t < best - 1e-9) {
+      best = t;
+      tp.S = S;
+    }
+  }
+  return tp;
+}
+
+// Fill t's work split from tail_plan; returns the grid in units.
+int apply_tail(TileSched& t, int units, const TailPlan& tp) {
+  t.sk_iters = 0;
+  if (tp.S <= 1) {
+    t.dp_tiles = t.total;
+    t.tail_R = 0;
+    t.tail_S = 1;
+    return t.total < units ? t.total : units;
+  }
+  const int W = t.total / units;
+  t.dp_tiles = W * units;
+  t.tail_R = t.total - t.dp_tiles;
+  t.tail_S = tp.S;
+  const int parts = t.tail_R * tp.S;
+  return W > 0 ? units : (parts < units ? parts : units);
+}
+
 }  // namespace
 
 cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
@@ -1001,34 +1091,50 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
   const int slots = (pairs_enabled() && bn_ok(P_BN, epi, W, p)) ? pair_slots_for(epi) : 0;
   int BN = 0;
   bool plan_pairs = false;
+  // Split-K workspace: slots of BM x 256 fp32 per CTA, four flags each.
+  const bool can_split = p.splitk_ws != nullptr && p.splitk_flags != nullptr;
+  const int cta_slots = can_split ? static_cast<int>(std::min<size_t>(p.splitk_ws_elems / (static_cast<size_t>(BM) * 256),
+                                                                       kSplitKFlags / 4))
+                                  : 0;
+  TailPlan plan_tp{1};
   if (num_kb >= kDeepKb) {
     // Deep K (>= 64 k-blocks: every 8B projection, the 1B down projection):
-    // the plan with the least waves x cost of one k-block step -- one-CTA
-    // tiles 128 or 256 wide, or 256 x 256 tiles on CTA pairs (only with two
-    // or more 128-row tiles: a lone one would leave half of each pair tile
-    // empty).  The step costs are GB300 graph-timed averages over the 1B and
-    // 8B pruned-forward shapes with every SM streaming: 0.27 us (128-wide)
+    // the plan with the least waves x cost of one k-block step
+    // -- one-CTA tiles 128 or 256 wide, or 256 x 256 tiles on CTA pairs (only
+    // with two or more 128-row tiles: a lone one would leave half of each pair
+    // tile empty); then its ragged last wave possibly cut into aligned k-parts
+    // (tail_plan).  The step costs are GB300 graph-timed averages over the 1B
+    // and 8B pruned-forward shapes with every SM streaming: 0.27 us (128-wide)
     // and 0.36 us (256-wide) per 64-deep k-block, 0.34 us per pair step.
     // Narrow tiles win only while they still fit one wave (8B QKV at 316
     // rows: 25.2 us against 30.1 on pairs); pairs win while they add no wave
     // (8B O at 744 rows: 27.7 us against 33.0 on the swapped kernel).
     double best = 1e30;
+    int best_tiles = 0;
     for (int cand : {128, 256}) {
       if (!bn_ok(cand, epi, W, p)) continue;
-      const long tiles = static_cast<long>(m_tiles) * ((vn + cand - 1) / cand);
+      const int tiles = m_tiles * ((vn + cand - 1) / cand);
       const double cost = static_cast<double>((tiles + sms - 1) / sms) * (cand == 256 ? 0.36 : 0.27);
       if (cost < best - 1e-9) {
         best = cost;
         BN = cand;
+        best_tiles = tiles;
       }
     }
     if (slots > 0 && m_tiles >= 2) {
-      const long ptiles = static_cast<long>((m_tiles + 1) / 2) * ((vn + P_BN - 1) / P_BN);
+      const int ptiles = ((m_tiles + 1) / 2) * ((vn + P_BN - 1) / P_BN);
       const double cost = static_cast<double>((ptiles + slots - 1) / slots) * 0.34;
       if (cost < best - 1e-9) {
         BN = P_BN;
         plan_pairs = true;
+        best_tiles = ptiles;
       }
+    }
+    if (BN != 0 && num_kb >= kVeryDeepKb) {
+      plan_tp = plan_pairs ? tail_plan(best_tiles, slots, num_kb, 0.34, can_split && 2 * slots <= kMaxGemmCtas,
+                                       cta_slots / 2)
+                           : tail_plan(best_tiles, sms, num_kb, BN == 256 ? 0.36 : 0.27,
+                                       can_split && sms <= kMaxGemmCtas, cta_slots);
     }
   }
   if (BN == 0) {
@@ -1052,23 +1158,29 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
   ts.total = ts.m_tiles * ts.n_tiles;
   ts.ws = p.splitk_ws;
   ts.flags = p.splitk_flags;
-  // Whole tiles, except with deep K and a ragged last wave of two or more:
-  // then stream-K over the last one-to-two waves (or over everything, for
-  // problems smaller than two waves), splitting k-blocks so no SM idles.
-  // Measured on GB300: the split pays at 128 and 224 k-blocks from a quarter
-  // of the last wave's SM-time idle (8B down at 1196 rows: 99.2 us split
-  // against 140.3 whole), but at 64 k-blocks only from 40% idle (8B QKV at
-  // 1732 rows, 26% idle: 79.3 split against 65.3 whole; 8B O at 1204 rows,
-  // 47% idle: 43.5 against 46.7), and never within one wave, where it only
-  // adds the partial hand-off (8B down at 744 rows: 81.5 against 74.6).
+  // Whole tiles, except with deep K and a ragged last wave:
+  //  - very deep K, where tail_plan found it cheaper: the last wave's tiles cut
+  //    into aligned k-parts (8B down at 1536 rows 145.5 -> 114.3 us, at 6456
+  //    rows 499.7 -> 461.3 us, against the rules below);
+  //  - else, from two waves on, stream-K over the last one-to-two waves (or
+  //    over everything, for problems smaller than two waves). Measured on
+  //    GB300: the contiguous split pays at 128 and 224 k-blocks from a quarter
+  //    of the last wave's SM-time idle (8B down at 1196 rows: 99.2 us split
+  //    against 140.3 whole), but at 64 k-blocks only from 40% idle (8B QKV
+  //    at 1732 rows, 26% idle: 79.3 split against 65.3 whole; 8B O at 1204
+  //    rows, 47% idle: 43.5 against 46.7), and never within one wave, where it
+  //    only adds the partial hand-off (8B down at 744 rows: 81.5 against 74.6).
   const double split_idle = num_kb >= 2 * kDeepKb ? 0.25 : 0.40;
   int grid;
-  {
+  if (!plan_pairs && plan_tp.S > 1) {
+    grid = apply_tail(ts, sms, plan_tp);
+  } else {
+    ts.tail_R = 0;
+    ts.tail_S = 1;
     const int waves = (ts.total + sms - 1) / sms;
     const double idle = 1.0 - static_cast<double>(ts.total) / (static_cast<double>(waves) * sms);
-    const bool can_split = p.splitk_ws != nullptr && p.splitk_flags != nullptr && sms <= kMaxGemmCtas &&
-                           static_cast<size_t>(sms) * BM * BN <= p.splitk_ws_elems;
-    if (plan_pairs || !can_split || num_kb < kDeepKb || waves < 2 || idle <= split_idle) {
+    const bool split_ok = can_split && sms <= kMaxGemmCtas && sms <= cta_slots;
+    if (plan_pairs || !split_ok || num_kb < kDeepKb || waves < 2 || idle <= split_idle) {
       ts.dp_tiles = ts.total;
       ts.sk_iters = 0;
       grid = ts.total < sms ? ts.total : sms;
@@ -1099,25 +1211,15 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
     ps.total = ps.m_tiles * ps.n_tiles;
     ps.ws = ts.ws;
     ps.flags = ts.flags;
+    ps.tail_R = 0;
+    ps.tail_S = 1;
     const int waves_pair = (ps.total + slots - 1) / slots;
     const double pair_idle = 1.0 - static_cast<double>(ps.total) / (static_cast<double>(waves_pair) * slots);
-    const bool pair_split_ok = 2 * slots <= kMaxGemmCtas &&
-                               static_cast<size_t>(2 * slots) * BM * P_BN <= p.splitk_ws_elems &&
-                               p.splitk_ws != nullptr && p.splitk_flags != nullptr;
-    bool whole = false, split = false;
-    if (plan_pairs) {
-      split = pair_split_ok && waves_pair >= 2 && pair_idle > split_idle;
-      whole = !split;
-    } else if (num_kb < kDeepKb) {
-      const int waves_one = (ts.total + sms - 1) / sms;
-      whole = waves_pair * kPairTileCost < waves_one && waves_one >= 2;
-    }
-    if (whole) {
-      ps.dp_tiles = ps.total;
-      ps.sk_iters = 0;
-      pairs = ps.total < slots ? ps.total : slots;
-    } else if (split) {
-      // deep K with a ragged last wave: the same stream-K split over the pairs
+    const bool pair_split_ok = can_split && 2 * slots <= kMaxGemmCtas && 2 * slots <= cta_slots;
+    if (plan_pairs && plan_tp.S > 1) {
+      pairs = apply_tail(ps, slots, plan_tp);
+    } else if (plan_pairs && pair_split_ok && waves_pair >= 2 && pair_idle > split_idle) {
+      // deep K with a ragged last wave: the contiguous stream-K split over the pairs
       pairs = slots;
       ps.dp_tiles = ps.total >= 2 * pairs ? (ps.total / pairs - 1) * pairs : 0;
       ps.sk_iters = static_cast<long long>(ps.total - ps.dp_tiles) * ps.num_kb;
@@ -1125,6 +1227,11 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
         const long long g = ps.sk_iters / 8;
         pairs = static_cast<int>(g < 1 ? 1 : (g < slots ? g : slots));
       }
+    } else if (plan_pairs) {
+      pairs = apply_tail(ps, slots, TailPlan{1});
+    } else if (num_kb < kDeepKb) {
+      const int waves_one = (ts.total + sms - 1) / sms;
+      if (waves_pair * kPairTileCost < waves_one && waves_one >= 2) pairs = apply_tail(ps, slots, TailPlan{1});
     }
   }
   TcMaps maps;

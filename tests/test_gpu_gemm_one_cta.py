@@ -19,10 +19,13 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 # (epilogue, M, N, K): whole tiles (two waves; 5000 x 2048 at K = 4096: 320
 # tiles, a full last wave), then deep K split over the CTAs where the last of
 # two or more waves is ragged (1204 rows: 160 tiles of 64 k-blocks; 1700 rows of
-# RoPE: 168; the 1B down projection at 3296 rows: 208 tiles of 128 k-blocks)
+# RoPE: 168; the 1B down projection at 3296 rows: 208 tiles of 128 k-blocks),
+# and with 192 k-blocks the last wave's tiles cut into aligned k-parts (5760 x
+# 1024: 180 tiles, the last 28 in four parts; SwiGLU 3072 x 1024: 40 in three)
 CASES = [("store", 2056, 2064, 512), ("swiglu", 2300, 1088, 512), ("rope", 2300, 3072, 512),
          ("store_f32", 1204, 4096, 4096), ("resid", 5000, 2048, 4096), ("swiglu", 1204, 2048, 4096),
-         ("rope", 1700, 3072, 4096), ("resid", 3296, 2048, 8192)]
+         ("rope", 1700, 3072, 4096), ("resid", 3296, 2048, 8192),
+         ("resid", 5760, 1024, 12288), ("swiglu", 3072, 1024, 12288)]
 
 
 def _run_cases():

@@ -107,6 +107,31 @@ def test_pair_streamk_down_1b(z):
     check_linear(out, ref, tol, "resid", "down M=3296")
 
 
+# Very deep K (>= 192 k-blocks, like the 8B down projection) with a ragged last
+# wave: the remainder tiles are cut into aligned k-parts (3072 rows x 2048
+# columns at K = 12288: 96 pair tiles, one whole wave, the last 20 tiles in
+# three parts of 64 k-blocks, the third adding the other two's partials).
+@pytest.mark.parametrize("epi,N", [("resid", 2048), ("store_f32", 2048), ("swiglu", 1024)])
+def test_pair_aligned_tail_split(z, epi, N):
+    out, ref, tol = linear_case(z, epi, 3072, N, 12288, 1600 + N)
+    check_linear(out, ref, tol, epi, f"{epi} M=3072 N={N} K=12288")
+
+
+def test_pair_aligned_tail_split_deterministic(z):
+    # the partials are added in part order: repeated calls agree bit for bit
+    M, N, K = 3072, 2048, 12288
+    A = rand_bf16((M, K), 31)
+    W = rand_bf16((N, K), 32, 0.05)
+    outs = []
+    for _ in range(3):
+        out = torch.empty(M, N, device="cuda", dtype=torch.float32)
+        z.zsaa_op_linear(A, W, None, None, out, M, N, K, z.ZSAA_BF16, z.EPI_STORE_F32)
+        outs.append(out)
+    torch.cuda.synchronize()
+    z.zsaa_device_status()
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
+
+
 # Deep-K plans of the pruned Llama-3.1-8B forward at a few hundred rows, one
 # wave each: whole pair tiles (down-like, 48 pair tiles of 128 k-blocks),
 # 128-wide one-CTA tiles (QKV + RoPE, hd 128, 144 tiles) and 256-wide one-CTA
