@@ -239,6 +239,8 @@ __device__ __forceinline__ uint32_t order_key(float f) {
 // the few hundred kept rows of the deep pruned layers).  Radix select (4 passes of 8 bits) finds the key T of
 // the need-th best candidate and how many candidates equal to T are taken;
 // then an index-ordered ballot/prefix scan writes the kept indices ascending.
+// Up to 256 candidates without marks take a shorter route to the same set:
+// each thread counts its candidate's rank against all others.
 // Ties (equal keys) keep lower indices first.  With force_last the last index
 // is kept and the other k-1 come from indices [0, N-1).
 // FROM_PARTS: the scores are first summed from column-mass partials
@@ -310,10 +312,41 @@ __global__ void __launch_bounds__(THREADS)
   const int n_cand = force_last ? N - 1 : N;
   const int need = force_last ? k - 1 : k;
 
-  __shared__ uint32_t hist[256];
+  __shared__ __align__(16) uint32_t hist[256];
   __shared__ uint32_t sh_digit, sh_remaining;
   __shared__ int wgt[nwarps], weq[nwarps];
   __shared__ int tile_gt, tile_eq;
+  const uint32_t lt_mask = (1u << lane) - 1u;
+
+  if (THREADS == 256 && al == nullptr && n_cand <= THREADS) {
+    // Short sequence, one candidate per thread: count the candidates ahead of
+    // candidate j in (key descending, index ascending) order directly.  Rank <
+    // need is the radix path's kept set (every key above the threshold, then
+    // equal keys lowest index first), without its four barrier-bound passes.
+    uint32_t* skey = hist;  // THREADS keys; the padding (key 0) never counts
+    const int j = tid;
+    const uint32_t kj = j < n_cand ? order_key(s[j]) : 0u;
+    skey[j] = kj;
+    __syncthreads();
+    int rank = 0;
+    const int n4 = (n_cand + 3) & ~3;
+    for (int i0 = 0; i0 < n4; i0 += 4) {
+      const uint4 k4 = *reinterpret_cast<const uint4*>(skey + i0);
+      rank += (k4.x > kj) + (k4.x == kj && i0 < j);
+      rank += (k4.y > kj) + (k4.y == kj && i0 + 1 < j);
+      rank += (k4.z > kj) + (k4.z == kj && i0 + 2 < j);
+      rank += (k4.w > kj) + (k4.w == kj && i0 + 3 < j);
+    }
+    const bool keep = j < n_cand && rank < need;
+    const uint32_t bk = __ballot_sync(0xffffffffu, keep);
+    if (lane == 0) wgt[warp] = __popc(bk);
+    __syncthreads();
+    int before = __popc(bk & lt_mask);
+    for (int w = 0; w < warp; ++w) before += wgt[w];
+    if (keep) out[before] = j;
+    if (force_last && tid == 0) out[k - 1] = N - 1;
+    return;
+  }
 
   uint32_t prefix = 0, mask = 0, remaining = static_cast<uint32_t>(need);
   if (need > 0) {
@@ -358,7 +391,6 @@ __global__ void __launch_bounds__(THREADS)
     }
   }
   const uint32_t T = prefix;
-  const uint32_t lt_mask = (1u << lane) - 1u;
   int base_gt = 0, base_eq = 0;
   for (int j0 = 0; j0 < n_cand && need > 0; j0 += THREADS) {
     const int j = j0 + tid;

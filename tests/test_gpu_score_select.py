@@ -36,7 +36,10 @@ def _select_oracle_f32(scores32, k, force_last):
     return np.stack([O.select_topk(s[b], k, force_last) for b in range(s.shape[0])])
 
 
-@pytest.mark.parametrize("B,L", [(3, 1), (2, 7), (4, 1000), (2, 1024), (1, 3001), (2, 8192)])
+# up to 256 candidates (L <= 256, or 257 with force-keep-last) take the rank-count
+# route, longer sequences the radix passes
+@pytest.mark.parametrize("B,L", [(3, 1), (2, 7), (2, 64), (3, 200), (2, 255), (2, 256), (2, 257), (4, 1000),
+                                 (2, 1024), (1, 3001), (2, 8192)])
 def test_selector_fed_scores_matches_oracle_exactly(z, B, L):
     rng = np.random.default_rng(L)
     cases = [rng.standard_normal((B, L)).astype(np.float32),
