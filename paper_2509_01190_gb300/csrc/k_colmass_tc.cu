@@ -304,8 +304,23 @@ __global__ void __launch_bounds__(CM_THREADS, 2)
             const int qc0 = half * 64 + c;
             const int q0 = qb * CM_BN + qc0;
             if ((!a.causal || q0 > key) && q0 + 32 <= n_b) {  // whole chunk inside the mask
+              // lse - s c for two columns in one packed FMA, then exp2 of its
+              // negation (the same rounding as s c - lse), summed in pairs:
+              // half the FMA-pipe instructions, which the MMA thread on the
+              // same SMSP competes with for issue slots
+              const uint64_t nc2 = f2pack(-a.scale_log2, -a.scale_log2);
+              uint64_t acc2 = f2pack(0.f, 0.f);
 #pragma unroll
-              for (int e = 0; e < 32; ++e) acc += ex2_ftz(__uint_as_float(r[e]) * a.scale_log2 - L[qc0 + e]);
+              for (int e = 0; e < 32; e += 2) {
+                const uint64_t u = ffma2(f2pack(__uint_as_float(r[e]), __uint_as_float(r[e + 1])), nc2,
+                                         *reinterpret_cast<const uint64_t*>(L + qc0 + e));
+                float u0, u1;
+                f2unpack(u, u0, u1);
+                acc2 = fadd2(acc2, f2pack(ex2_ftz(-u0), ex2_ftz(-u1)));
+              }
+              float a0, a1;
+              f2unpack(acc2, a0, a1);
+              acc += a0 + a1;
             } else {
 #pragma unroll
               for (int e = 0; e < 32; ++e) {
