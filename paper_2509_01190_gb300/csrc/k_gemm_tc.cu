@@ -185,41 +185,52 @@ __device__ __forceinline__ void store_bf16x16(bf16* dst, const float (&v)[16]) {
   d[1] = make_uint4(o[4], o[5], o[6], o[7]);
 }
 
-// Sum of the partial tiles of contributors c0..c1 (inclusive; none if
-// c0 > c1) at this thread's row, tile columns [col, col + 16), added to v.
-// Contributor c's slot starts at ws + c * cstride.  Partials are stored
-// column-major ([BN][BM] per slot) so a warp's loads are coalesced; up to four
-// contributors' loads are in flight together, then added in order.
+// Adds the fp32 partials of `count` contributors (slot c at ws + c * cstride,
+// column-major [BN][BM]: element (row, col) at slot[col * BM + row]) into this
+// thread's row of the TMEM accumulator, contributor by contributor and column
+// by column in increasing order, so each element is acc + p0 + p1 + ... in
+// that order.  Every partial load is an L2 round trip, so the loads run two
+// 32-column chunks ahead of the adds (a warp's loads of one column are one
+// coalesced 128-byte line).
 template <int BN>
-__device__ __forceinline__ void add_partials(float (&v)[16], const float* ws, size_t cstride, int c0,
-                                             int c1, int rit, int col) {
-  for (int c = c0; c <= c1; c += 4) {
-    float t[4][16];
+__device__ __forceinline__ void fold_partials(uint32_t tbase, const float* ws, size_t cstride, int count,
+                                              int rit) {
+  constexpr int NCH = BN / 32;
+  constexpr int DEPTH = NCH < 2 ? NCH : 2;
+#pragma unroll 1
+  for (int c = 0; c < count; ++c) {
+    const float* slot = ws + static_cast<size_t>(c) * cstride + rit;
+    float buf[DEPTH][32];
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      if (c + k <= c1) {
-        const float* q = ws + static_cast<size_t>(c + k) * cstride + static_cast<size_t>(col) * BM + rit;
+    for (int k = 0; k < DEPTH; ++k)
 #pragma unroll
-        for (int e = 0; e < 16; ++e) t[k][e] = __ldcg(q + e * BM);
+      for (int e = 0; e < 32; ++e) buf[k][e] = __ldcg(slot + static_cast<size_t>(32 * k + e) * BM);
+#pragma unroll
+    for (int ch = 0; ch < NCH; ++ch) {
+      uint32_t r[32];
+      __syncwarp();
+      tmem_ld16(tbase + 32 * ch, *reinterpret_cast<uint32_t(*)[16]>(r));
+      tmem_ld16(tbase + 32 * ch + 16, *reinterpret_cast<uint32_t(*)[16]>(r + 16));
+      tmem_ld_wait();
+#pragma unroll
+      for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) + buf[ch % DEPTH][e]);
+      tmem_st16(tbase + 32 * ch, *reinterpret_cast<const uint32_t(*)[16]>(r));
+      tmem_st16(tbase + 32 * ch + 16, *reinterpret_cast<const uint32_t(*)[16]>(r + 16));
+      if (ch + DEPTH < NCH) {
+#pragma unroll
+        for (int e = 0; e < 32; ++e)
+          buf[ch % DEPTH][e] = __ldcg(slot + static_cast<size_t>(32 * (ch + DEPTH) + e) * BM);
       }
     }
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      if (c + k <= c1) {
-#pragma unroll
-        for (int e = 0; e < 16; ++e) v[e] += t[k][e];
-      }
-    }
+    tmem_st_wait();  // this contributor's sums are in TMEM before the next pass reads them
   }
 }
 
-// Epilogue of one finished accumulator tile for this thread's row; the
-// partials of contributors c0..c1 (slots ws + c * cstride, if any) are added
-// to the accumulator first.
+// Epilogue of one finished accumulator tile for this thread's row (any
+// split-K partials are already folded into the accumulator).
 template <int BN, int EPI>
 __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_ok, int n0,
-                                              const GemmParams& p, const float* ws, size_t cstride,
-                                              int c0, int c1, int rit) {
+                                              const GemmParams& p) {
   if (EPI == kEpiSwiGLU) {
     bf16* out = static_cast<bf16*>(p.out);
     const int oc0 = n0 / 2;
@@ -237,8 +248,6 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
           gv[e] = __uint_as_float(g[e]);
           uv[e] = __uint_as_float(u[e]);
         }
-        add_partials<BN>(gv, ws, cstride, c0, c1, rit, c);
-        add_partials<BN>(uv, ws, cstride, c0, c1, rit, BN / 2 + c);
 #pragma unroll
         for (int e = 0; e < 16; ++e) v[e] = silu_f(gv[e]) * uv[e];
         store_bf16x16(out + static_cast<size_t>(row) * p.ldo + oc0 + c, v);
@@ -259,7 +268,6 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
           float v[16];
 #pragma unroll
           for (int e = 0; e < 16; ++e) v[e] = __uint_as_float(r[16 * h + e]);
-          add_partials<BN>(v, ws, cstride, c0, c1, rit, c + 16 * h);
           float4* dst = reinterpret_cast<float4*>(out + static_cast<size_t>(row) * p.ldo + n0 + c + 16 * h);
 #pragma unroll
           for (int q = 0; q < 4; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
@@ -298,8 +306,6 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
             a1[e] = __uint_as_float(x1[e]);
             a2[e] = __uint_as_float(x2[e]);
           }
-          add_partials<BN>(a1, ws, cstride, c0, c1, rit, hs + c);
-          add_partials<BN>(a2, ws, cstride, c0, c1, rit, hs + half + c);
           if (rot) {
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -369,7 +375,6 @@ __device__ __forceinline__ void tile_epilogue(uint32_t tbase, int row, bool row_
           float v[16];
 #pragma unroll
           for (int e = 0; e < 16; ++e) v[e] = __uint_as_float(r[16 * h + e]);
-          add_partials<BN>(v, ws, cstride, c0, c1, rit, c + 16 * h);
           if (EPI == kEpiResid) {
             const uint32_t rr[8] = {rc[2 * h].x, rc[2 * h].y, rc[2 * h].z, rc[2 * h].w,
                                     rc[2 * h + 1].x, rc[2 * h + 1].y, rc[2 * h + 1].z, rc[2 * h + 1].w};
@@ -596,9 +601,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             got = got && wait_flag(ts.flags + (w.slot + c * w.stride) * 4 + quad, p.status, abort_flag);
           if (!__all_sync(0xffffffffu, got)) c1 = -1;  // gave up: status already set
         }
-        tile_epilogue<BN, EPI>(tbase, row, row < p.M, nt * BN, p,
-                               c1 >= 0 ? ts.ws + static_cast<size_t>(w.slot) * kSlot : nullptr,
-                               static_cast<size_t>(w.stride) * kSlot, 0, c1, rit);
+        if (c1 >= 0)
+          fold_partials<BN>(tbase, ts.ws + static_cast<size_t>(w.slot) * kSlot, static_cast<size_t>(w.stride) * kSlot,
+                            c1 + 1, rit);
+        tile_epilogue<BN, EPI>(tbase, row, row < p.M, nt * BN, p);
         if (w.kind == 2) {
           __syncwarp();
           if (lane == 0)
@@ -849,9 +855,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             got = got && wait_flag(ts.flags + (2 * (w.slot + c * w.stride) + rank) * 4 + quad, p.status, abort_flag);
           if (!__all_sync(0xffffffffu, got)) c1 = -1;  // gave up: status already set
         }
-        const float* ws = c1 >= 0 ? ts.ws + static_cast<size_t>(2 * w.slot + rank) * kSlot : nullptr;
-        tile_epilogue<P_BN, EPI>(tbase, row, row < p.M, nt * P_BN, p, ws, 2 * static_cast<size_t>(w.stride) * kSlot,
-                                 0, c1, rit);
+        if (c1 >= 0)
+          fold_partials<P_BN>(tbase, ts.ws + static_cast<size_t>(2 * w.slot + rank) * kSlot,
+                              2 * static_cast<size_t>(w.stride) * kSlot, c1 + 1, rit);
+        tile_epilogue<P_BN, EPI>(tbase, row, row < p.M, nt * P_BN, p);
         if (w.kind == 2) {
           __syncwarp();
           if (lane == 0)
