@@ -57,11 +57,11 @@ TRAFFIC = {
     # profiles/gemm_gate_up_swiglu_8b_traffic.md: the first layer's MLP at accel 4
     ("gemm_gate_up_swiglu", "8b"): {
         "launch": "gate/up + SwiGLU, M=7272 rows (layer 1 of the accel-4 forward), N=2x14336, K=4096",
-        "bytes": 1322317568.0,
+        "bytes": 1343622912.0,
         "algorithmic_bytes": 502956032.0,
         "sources": {
-            "paper_2509_01190_gb300/csrc/k_gemm_tc.cu": "0252745b58d5e879bc6f057916a7ff378d83590e0119fea4bf4d9a38fa7b142f",
-            "paper_2509_01190_gb300/csrc/common.cuh": "04c1d919379eb70f1b19a49cf56ae7cba7f55c48cb1fcf4db130c293a8ab7625",
+            "paper_2509_01190_gb300/csrc/k_gemm_tc.cu": "bff0e75c635c6b3c7c3463f889db3f0a2fb19b883c7646720056df95af1dcbd2",
+            "paper_2509_01190_gb300/csrc/common.cuh": "9e474368fc0200765d2891a8fa691189a035962da12ffe00a8ef80d040644cbf",
             "paper_2509_01190_gb300/csrc/kernels.h": "388c8fccbdf54c8ab7761032c7012ee27e045ee27c2d3acaac223b7b2208d596",
         },
     },
