@@ -188,7 +188,9 @@ cudaError_t run_skinny(const bf16* A, int lda, const TcWeights& W, const GemmPar
   const int bands = p.N / 16;
   const int cap = 2 * sm_count();
   const int grid = bands < cap ? bands : cap;
-  constexpr int U = EPI == kEpiSwiGLU ? (MF == 1 ? 4 : 2) : (MF == 1 ? 6 : 4);
+  // chunks in flight per warp, as many as the registers allow: with 8 rows and
+  // one weight matrix, a K = 2048 band's whole share (8 chunks) per round trip
+  constexpr int U = EPI == kEpiSwiGLU ? (MF == 1 ? 4 : 2) : (MF == 1 ? 8 : 4);
   ZSAA_LAUNCH(skinny_gemm_kernel<EPI, MF, U>, dim3(grid), dim3(SK_THREADS), 0, s, A, lda, W, p,
               bands);
   return cudaSuccess;
