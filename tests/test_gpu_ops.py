@@ -31,8 +31,9 @@ def _np(t):
     return t.detach().float().cpu().numpy().astype(np.float64)
 
 
+# (3, 1024, 4096): the weight-streaming kernel's 16-warp form (K >= 4096, few bands)
 @pytest.mark.parametrize("M,N,K", [(1, 64, 64), (300, 384, 256), (128, 256, 128), (517, 1024, 512),
-                                   (40, 2048, 2048)])
+                                   (40, 2048, 2048), (3, 1024, 4096)])
 def test_linear_bf16_store_and_f32(z, M, N, K):
     A = _rand((M, K), 1)
     W = _rand((N, K), 2)
@@ -61,7 +62,8 @@ def test_linear_bf16_large_n_lm_head(z):
     assert np.all(np.abs(_np(out) - ref) <= accum_bound(_np(A), _np(W)) + 1e-6 * np.abs(ref))
 
 
-@pytest.mark.parametrize("M,N,K", [(200, 256, 128), (5, 512, 1024), (1000, 2048, 256)])
+# (8, 2048, 8192): a decode step's down projection (16-warp weight streaming)
+@pytest.mark.parametrize("M,N,K", [(200, 256, 128), (5, 512, 1024), (1000, 2048, 256), (8, 2048, 8192)])
 def test_linear_bf16_residual_in_place(z, M, N, K):
     A = _rand((M, K), 5, 0.1)
     W = _rand((N, K), 6, 0.1)
