@@ -60,9 +60,9 @@ TRAFFIC = {
         "bytes": 1343622912.0,
         "algorithmic_bytes": 502956032.0,
         "sources": {
-            "paper_2509_01190_gb300/csrc/k_gemm_tc.cu": "bff0e75c635c6b3c7c3463f889db3f0a2fb19b883c7646720056df95af1dcbd2",
+            "paper_2509_01190_gb300/csrc/k_gemm_tc.cu": "476652139b6316266382a408d78f0d679ecabad54bb26d64f2f15e01a1c5d7f0",
             "paper_2509_01190_gb300/csrc/common.cuh": "9e474368fc0200765d2891a8fa691189a035962da12ffe00a8ef80d040644cbf",
-            "paper_2509_01190_gb300/csrc/kernels.h": "388c8fccbdf54c8ab7761032c7012ee27e045ee27c2d3acaac223b7b2208d596",
+            "paper_2509_01190_gb300/csrc/kernels.h": "c895255d48b1cd8b7810c67d6c8082cc110807e30ffdb7a90ddc0a9faca5635b",
         },
     },
 }

@@ -375,6 +375,35 @@ zsaa_status zsaa_op_linear(const void* A, const void* W, const void* W2, const v
                            const int32_t* pos, int rope_cols, int rope_hd, float rope_theta,
                            zsaa_stream stream);
 
+/* The work decomposition of the persistent tiled GEMM (the kernel that
+ * zsaa_op_linear and the forward use beyond the weight-streaming and
+ * swapped-operand row ranges) for one call shape, computed on the host exactly
+ * as a launch computes it, without device work (no GPU needed).  The device
+ * is described by sms (one-CTA kernel CTAs resident at once, one per SM;
+ * >= 1), pair_slots (CTA pairs resident at once; 0: the pair kernel is not
+ * used) and split_slots (split-K partial slots of 128 x 256 fp32 in the
+ * workspace; 256 in the library's own workspaces, 0: no split).  One weight
+ * matrix [N, K]; epilogue as zsaa_op_linear, RoPE heads of hd dims (hd >= 32,
+ * a multiple of 32; other epilogues ignore hd).  K % 64 == 0, N % 16 == 0,
+ * M >= 1.
+ *   plan_out (host int32[12]): tile width, kernel (0 one CTA, 1 CTA pairs on
+ *     256-row tiles), units (CTAs or pairs launched), row tiles, column tiles,
+ *     64-deep k-blocks per tile, tiles, whole tiles dealt round robin first,
+ *     k-iterations of the contiguous split that follows them, tiles of the
+ *     aligned split (R) and their k-parts (S), 0.
+ *   items (host int32[cap][8], or NULL with cap 0): every unit's work items
+ *     in the order the unit runs them: unit, tile, first and end k-block, kind
+ *     (0 a whole tile; 1 a part whose fp32 partial goes to slot `slot`; 2 the
+ *     tile's final part, which waits for and adds the `count` partials in
+ *     slots slot, slot + stride, ... in that order), slot, count, stride.
+ *   *n_items (host) receives the number of items, including any past cap.
+ * Unsupported shapes return ZSAA_ERR_INVALID_ARG or ZSAA_ERR_UNSUPPORTED; so
+ * does a plan whose work items would outnumber its tiles' k-blocks (each item
+ * covers at least one), which no sound plan has. */
+zsaa_status zsaa_gemm_schedule(int epilogue, int M, int N, int K, int hd, int sms, int pair_slots,
+                               int split_slots, int32_t* plan_out, int32_t* items, int64_t cap,
+                               int64_t* n_items);
+
 /* zsaa_op_attention: causal grouped-query attention (Eq. 1) over a packed
  * qkv [B*N, (Hq + 2 Hkv) hd] buffer (per row: Hq query heads, then Hkv key
  * heads, then Hkv value heads).  out [B*N, Hq*hd]; lse float32 [B, Hq, N]

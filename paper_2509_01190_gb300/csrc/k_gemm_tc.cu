@@ -84,11 +84,12 @@ struct Item {
 };
 
 // Work of unit `unit` of `units` (a CTA of the one-CTA kernel, a CTA pair of
-// the pair kernel; both CTAs of a pair walk the same items).
+// the pair kernel; both CTAs of a pair walk the same items).  Plain integer
+// arithmetic, also run on the host to describe a plan (gemm_tc_schedule).
 struct WorkIter {
   int t_dp, units, unit, q;
   long long it, end;
-  __device__ __forceinline__ void init(const TileSched& ts, int u, int nunits) {
+  __host__ __device__ __forceinline__ void init(const TileSched& ts, int u, int nunits) {
     t_dp = u;
     units = nunits;
     unit = u;
@@ -97,7 +98,7 @@ struct WorkIter {
     it = static_cast<long long>(u) * ts.sk_iters / G;
     end = static_cast<long long>(u + 1) * ts.sk_iters / G;
   }
-  __device__ __forceinline__ bool next(const TileSched& ts, Item& w) {
+  __host__ __device__ __forceinline__ bool next(const TileSched& ts, Item& w) {
     w.slot = 0;
     w.count = 0;
     w.stride = 1;
@@ -114,7 +115,8 @@ struct WorkIter {
       if (it >= end) return false;
       const long long u = it / KB;
       const int a = static_cast<int>(it - u * KB);
-      const int b = static_cast<int>(min(static_cast<long long>(KB), a + (end - it)));
+      const long long rest = a + (end - it);
+      const int b = static_cast<int>(rest < KB ? rest : KB);
       w.tile = ts.dp_tiles + static_cast<int>(u);
       w.kb0 = a;
       w.kb1 = b;
@@ -1080,29 +1082,38 @@ int apply_tail(TileSched& t, int units, const TailPlan& tp) {
   return W > 0 ? units : (parts < units ? parts : units);
 }
 
-}  // namespace
+// What the tile plan needs besides the call's shape: how many CTAs (one per
+// SM) and CTA pairs the device runs at once for this epilogue, the split-K
+// workspace, and which tile widths the weight splits and RoPE heads allow.
+struct TilePlanIn {
+  int epi, M, N, K;
+  int sms;         // one-CTA kernel: CTAs resident at once
+  int slots;       // pair kernel: CTA pairs resident at once; 0: no pairs
+  bool can_split;  // a split-K workspace and flags were given
+  int cta_slots;   // its partial slots (BM x 256 fp32, four flags each)
+  bool bn64, bn128, bn256;
+  bool width_ok(int BN) const { return BN == 64 ? bn64 : (BN == 128 ? bn128 : (BN == 256 && bn256)); }
+};
 
-cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
-                           const GemmParams& p, cudaStream_t s) {
-  if (p.K % BK != 0 || p.N % 16 != 0 || lda % 8 != 0) return cudaErrorInvalidValue;
-  // a handful of rows: 128-row tiles would idle most of the tensor core and
-  // most SMs; stream the weights instead
-  if (skinny_supported(A, lda, W, epi, p)) return launch_gemm_skinny(A, lda, W, epi, p, s);
-  // a few hundred rows: weight band as the 128-row operand, K split over a cluster
-  if (swap_preferred(epi, p.M, p.N, p.K) && swap_supported(A, lda, W, epi, p))
-    return launch_gemm_swap(A, lda, W, epi, p, s);
-  const int sms = num_sms();
-  const int vn = epi == kEpiSwiGLU ? 2 * p.N : p.N;
-  const int m_tiles = (p.M + BM - 1) / BM;
-  const int num_kb = p.K / BK;
-  const int slots = (pairs_enabled() && bn_ok(P_BN, epi, W, p)) ? pair_slots_for(epi) : 0;
+// The plan: the one-CTA kernel's tile width, grid and work split, and, when
+// pairs > 0, the CTA-pair kernel's (which then runs instead).  The splits'
+// workspace pointers are left to the caller.
+struct TilePlanOut {
+  int BN, grid;
+  TileSched ts;
+  int pairs;
+  TileSched ps;
+};
+
+// Host only: no device calls.  False when no tile width fits.
+bool plan_tiles(const TilePlanIn& in, TilePlanOut& o) {
+  const int epi = in.epi, sms = in.sms, slots = in.slots, cta_slots = in.cta_slots;
+  const bool can_split = in.can_split;
+  const int vn = epi == kEpiSwiGLU ? 2 * in.N : in.N;
+  const int m_tiles = (in.M + BM - 1) / BM;
+  const int num_kb = in.K / BK;
   int BN = 0;
   bool plan_pairs = false;
-  // Split-K workspace: slots of BM x 256 fp32 per CTA, four flags each.
-  const bool can_split = p.splitk_ws != nullptr && p.splitk_flags != nullptr;
-  const int cta_slots = can_split ? static_cast<int>(std::min<size_t>(p.splitk_ws_elems / (static_cast<size_t>(BM) * 256),
-                                                                       kSplitKFlags / 4))
-                                  : 0;
   TailPlan plan_tp{1};
   if (num_kb >= kDeepKb) {
     // Deep K (>= 64 k-blocks: every 8B projection, the 1B down projection):
@@ -1119,7 +1130,7 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
     double best = 1e30;
     int best_tiles = 0;
     for (int cand : {128, 256}) {
-      if (!bn_ok(cand, epi, W, p)) continue;
+      if (!in.width_ok(cand)) continue;
       const int tiles = m_tiles * ((vn + cand - 1) / cand);
       const double cost = static_cast<double>((tiles + sms - 1) / sms) * (cand == 256 ? 0.36 : 0.27);
       if (cost < best - 1e-9) {
@@ -1153,18 +1164,16 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
     const long wide_tiles = static_cast<long>(m_tiles) * ((vn + 255) / 256);
     const int want = (epi == kEpiSwiGLU || wide_tiles >= 2L * sms)
                          ? 256
-                         : (p.M <= 256 ? 64 : (p.M <= 768 ? 128 : 256));
+                         : (in.M <= 256 ? 64 : (in.M <= 768 ? 128 : 256));
     for (int cand : {64, 128, 256})
-      if (bn_ok(cand, epi, W, p) && (BN == 0 || cand <= want)) BN = cand;
-    if (BN == 0) return cudaErrorInvalidValue;
+      if (in.width_ok(cand) && (BN == 0 || cand <= want)) BN = cand;
+    if (BN == 0) return false;
   }
   TileSched ts{};
   ts.m_tiles = m_tiles;
   ts.n_tiles = (vn + BN - 1) / BN;
   ts.num_kb = num_kb;
   ts.total = ts.m_tiles * ts.n_tiles;
-  ts.ws = p.splitk_ws;
-  ts.flags = p.splitk_flags;
   // Whole tiles, except with deep K and a ragged last wave:
   //  - very deep K, where tail_plan found it cheaper: the last wave's tiles cut
   //    into aligned k-parts (8B down at 1536 rows 145.5 -> 114.3 us, at 6456
@@ -1216,8 +1225,6 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
     ps.n_tiles = ts.n_tiles;
     ps.num_kb = ts.num_kb;
     ps.total = ps.m_tiles * ps.n_tiles;
-    ps.ws = ts.ws;
-    ps.flags = ts.flags;
     ps.tail_R = 0;
     ps.tail_S = 1;
     const int waves_pair = (ps.total + slots - 1) / slots;
@@ -1241,6 +1248,47 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
       if (waves_pair * kPairTileCost < waves_one && waves_one >= 2) pairs = apply_tail(ps, slots, TailPlan{1});
     }
   }
+  o.BN = BN;
+  o.grid = grid;
+  o.ts = ts;
+  o.pairs = pairs;
+  o.ps = ps;
+  return true;
+}
+
+}  // namespace
+
+cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
+                           const GemmParams& p, cudaStream_t s) {
+  if (p.K % BK != 0 || p.N % 16 != 0 || lda % 8 != 0) return cudaErrorInvalidValue;
+  // a handful of rows: 128-row tiles would idle most of the tensor core and
+  // most SMs; stream the weights instead
+  if (skinny_supported(A, lda, W, epi, p)) return launch_gemm_skinny(A, lda, W, epi, p, s);
+  // a few hundred rows: weight band as the 128-row operand, K split over a cluster
+  if (swap_preferred(epi, p.M, p.N, p.K) && swap_supported(A, lda, W, epi, p))
+    return launch_gemm_swap(A, lda, W, epi, p, s);
+  const int vn = epi == kEpiSwiGLU ? 2 * p.N : p.N;
+  TilePlanIn in;
+  in.epi = epi;
+  in.M = p.M;
+  in.N = p.N;
+  in.K = p.K;
+  in.sms = num_sms();
+  in.slots = (pairs_enabled() && bn_ok(P_BN, epi, W, p)) ? pair_slots_for(epi) : 0;
+  // Split-K workspace: slots of BM x 256 fp32 per CTA, four flags each.
+  in.can_split = p.splitk_ws != nullptr && p.splitk_flags != nullptr;
+  in.cta_slots = in.can_split ? static_cast<int>(std::min<size_t>(p.splitk_ws_elems / (static_cast<size_t>(BM) * 256),
+                                                                   kSplitKFlags / 4))
+                              : 0;
+  in.bn64 = bn_ok(64, epi, W, p);
+  in.bn128 = bn_ok(128, epi, W, p);
+  in.bn256 = bn_ok(256, epi, W, p);
+  TilePlanOut pl;
+  if (!plan_tiles(in, pl)) return cudaErrorInvalidValue;
+  const int BN = pl.BN, grid = pl.grid, pairs = pl.pairs;
+  TileSched ts = pl.ts, ps = pl.ps;
+  ts.ws = ps.ws = p.splitk_ws;
+  ts.flags = ps.flags = p.splitk_flags;
   TcMaps maps;
   memset(&maps, 0, sizeof(maps));
   const uint32_t brows = (pairs > 0 || epi == kEpiSwiGLU) ? BN / 2 : BN;
@@ -1269,6 +1317,59 @@ cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
     case 128: return dispatch_epi<128>(epi, maps, n1, n2, p, ts, grid, s);
     default: return dispatch_epi<64>(epi, maps, n1, n2, p, ts, grid, s);
   }
+}
+
+int gemm_tc_schedule(int epi, int M, int N, int K, int hd, int sms, int pair_slots, int split_slots,
+                     int* plan, int* items, long long cap, long long* n_items) {
+  TilePlanIn in;
+  in.epi = epi;
+  in.M = M;
+  in.N = N;
+  in.K = K;
+  in.sms = sms;
+  // one weight matrix (no weight splits); RoPE heads of hd dims in every column tile
+  auto width_ok = [&](int BN) { return epi != kEpiRope || BN % hd == 0; };
+  in.slots = width_ok(P_BN) ? pair_slots : 0;
+  in.can_split = split_slots > 0;
+  in.cta_slots = in.can_split ? std::min(split_slots, static_cast<int>(kSplitKFlags / 4)) : 0;
+  in.bn64 = width_ok(64);
+  in.bn128 = width_ok(128);
+  in.bn256 = width_ok(256);
+  TilePlanOut pl;
+  if (!plan_tiles(in, pl)) return -1;
+  const bool pairs = pl.pairs > 0;
+  const TileSched& ts = pairs ? pl.ps : pl.ts;
+  const int units = pairs ? pl.pairs : pl.grid;
+  if (ts.sk_iters > 0x7fffffffLL) return -1;
+  const int fields[12] = {pl.BN, pairs ? 1 : 0, units, ts.m_tiles, ts.n_tiles, ts.num_kb, ts.total,
+                          ts.dp_tiles, static_cast<int>(ts.sk_iters), ts.tail_R, ts.tail_S, 0};
+  for (int i = 0; i < 12; ++i) plan[i] = fields[i];
+  // every item of a sound plan covers at least one k-block: more items than
+  // tile k-blocks means a unit's iterator does not advance
+  const long long limit = static_cast<long long>(ts.total) * ts.num_kb;
+  long long n = 0;
+  for (int u = 0; u < units; ++u) {
+    WorkIter it;
+    it.init(ts, u, units);
+    Item w;
+    while (it.next(ts, w)) {
+      if (n >= limit) return -2;
+      if (items != nullptr && n < cap) {
+        int* o = items + 8 * n;
+        o[0] = u;
+        o[1] = w.tile;
+        o[2] = w.kb0;
+        o[3] = w.kb1;
+        o[4] = w.kind;
+        o[5] = w.slot;
+        o[6] = w.count;
+        o[7] = w.stride;
+      }
+      ++n;
+    }
+  }
+  *n_items = n;
+  return 0;
 }
 
 }  // namespace zsaa

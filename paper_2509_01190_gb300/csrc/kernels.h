@@ -102,6 +102,16 @@ struct TcWeights {
 // K (ZSAA_GEMM_PAIRS=0 in the environment keeps one CTA).
 cudaError_t launch_gemm_tc(const void* A, int lda, const TcWeights& W, int epi,
                            const GemmParams& p, cudaStream_t s);
+// The tiled kernels' plan for one call shape, computed on the host exactly as
+// launch_gemm_tc computes it, for a device running `sms` CTAs and
+// `pair_slots` CTA pairs at once and `split_slots` split-K partial slots
+// (one weight matrix; RoPE heads of hd dims).  plan[12] and, up to cap of
+// them, every unit's work items (8 ints each) in the order the unit runs
+// them; *n_items = their number.  Returns 0; -1 when no tile width fits;
+// -2 when the units' items outnumber the tiles' k-blocks (an iterator that
+// does not advance).
+int gemm_tc_schedule(int epi, int M, int N, int K, int hd, int sms, int pair_slots, int split_slots,
+                     int* plan, int* items, long long cap, long long* n_items);
 
 // Weight-streaming bf16 GEMM for M <= kSkinnyMaxM rows (k_skinny.cu): every
 // epilogue but RoPE; N % 16 == 0, K % 32 == 0, lda % 8 == 0, 16-byte aligned

@@ -1788,6 +1788,25 @@ zsaa_status zsaa_score_select_ex(const void* hidden, int B, int L, int d, int dt
                            gathered_out, reinterpret_cast<cudaStream_t>(stream));
 }
 
+zsaa_status zsaa_gemm_schedule(int epilogue, int M, int N, int K, int hd, int sms, int pair_slots,
+                               int split_slots, int32_t* plan_out, int32_t* items, int64_t cap,
+                               int64_t* n_items) {
+  if (plan_out == nullptr || n_items == nullptr) return fail(ZSAA_ERR_INVALID_ARG, "null argument");
+  if (items == nullptr && cap != 0) return fail(ZSAA_ERR_INVALID_ARG, "null items with cap > 0");
+  if (cap < 0) return fail(ZSAA_ERR_INVALID_ARG, "cap must be >= 0");
+  if (M < 1 || N < 16 || K < 64) return fail(ZSAA_ERR_INVALID_ARG, "M >= 1, N >= 16, K >= 64");
+  if (K % 64 || N % 16) return fail(ZSAA_ERR_UNSUPPORTED, "the tiled GEMM needs K %% 64 == 0 and N %% 16 == 0");
+  if (epilogue < 0 || epilogue > 4) return fail(ZSAA_ERR_INVALID_ARG, "bad epilogue");
+  if (epilogue == kEpiRope && (hd < 32 || hd % 32)) return fail(ZSAA_ERR_INVALID_ARG, "bad RoPE head size");
+  if (sms < 1 || pair_slots < 0 || split_slots < 0) return fail(ZSAA_ERR_INVALID_ARG, "bad device description");
+  long long n = 0;
+  const int r = gemm_tc_schedule(epilogue, M, N, K, hd, sms, pair_slots, split_slots, plan_out, items, cap, &n);
+  if (r == -1) return fail(ZSAA_ERR_UNSUPPORTED, "no tile plan for this shape");
+  if (r != 0) return fail(ZSAA_ERR_INVALID_ARG, "work items outnumber the tiles' k-blocks");
+  *n_items = n;
+  return ZSAA_OK;
+}
+
 zsaa_status zsaa_op_linear(const void* A, const void* W, const void* W2, const void* resid,
                            void* out, int M, int N, int K, int dtype, int epilogue,
                            const int32_t* pos, int rope_cols, int rope_hd, float rope_theta,

@@ -31,6 +31,7 @@ EXPORTED = [
     "zsaa_prefill", "zsaa_decode_step", "zsaa_cache_layer", "zsaa_cache_bytes",
     "zsaa_op_attention_ex", "zsaa_op_colmass_ex", "zsaa_plan_varlen_config", "zsaa_plan_varlen",
     "zsaa_forward_varlen", "zsaa_forward_masked", "zsaa_forward_marked", "zsaa_selftest_wait_timeout",
+    "zsaa_gemm_schedule",
 ]
 
 
@@ -93,6 +94,7 @@ def lib():
             "zsaa_score_select_noalloc": ([_P, _I, _I, _I, _I, _P, _P, _P], _I),
             "zsaa_model_set_graphs": ([_P, _I], _I),
             "zsaa_op_linear": ([_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _I, _I, C.c_float, _P], _I),
+            "zsaa_gemm_schedule": ([_I, _I, _I, _I, _I, _I, _I, _I, _P, _P, C.c_int64, C.POINTER(C.c_int64)], _I),
             "zsaa_op_attention": ([_P, _I, _I, _I, _I, _I, _I, _P, _P, _P], _I),
             "zsaa_op_colmass": ([_P, _P, _I, _I, _I, _I, _I, _I, _P, _P], _I),
             "zsaa_op_attention_ex": ([_P, _I, _I, _I, _I, _I, _I, _I, _P, _P, _P], _I),
@@ -440,6 +442,21 @@ def zsaa_op_linear(A, W, W2, resid, out, M: int, N: int, K: int, dtype: int, epi
     _check(lib().zsaa_op_linear(_ptr(A), _ptr(W), _ptr(W2), _ptr(resid), _ptr(out), M, N, K, dtype,
                                 epilogue, _ptr(pos), rope_cols, rope_hd, float(rope_theta),
                                 _stream(stream)))
+
+
+def zsaa_gemm_schedule(epilogue: int, M: int, N: int, K: int, hd: int, sms: int, pair_slots: int,
+                       split_slots: int):
+    """Host-side tile plan of the tiled GEMM: (plan: 12 ints, items: list of
+    8-int tuples (unit, tile, kb0, kb1, kind, slot, count, stride))."""
+    plan = (C.c_int32 * 12)()
+    n = C.c_int64()
+    _check(lib().zsaa_gemm_schedule(epilogue, M, N, K, hd, sms, pair_slots, split_slots, plan, None, 0,
+                                    C.byref(n)))
+    buf = (C.c_int32 * (8 * max(n.value, 1)))()
+    _check(lib().zsaa_gemm_schedule(epilogue, M, N, K, hd, sms, pair_slots, split_slots, plan, buf,
+                                    n.value, C.byref(n)))
+    flat = list(buf)
+    return list(plan), [tuple(flat[8 * i:8 * i + 8]) for i in range(n.value)]
 
 
 def zsaa_op_attention(qkv, B: int, N: int, Hq: int, Hkv: int, hd: int, dtype: int, out, lse,
