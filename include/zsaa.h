@@ -377,7 +377,9 @@ zsaa_status zsaa_op_linear(const void* A, const void* W, const void* W2, const v
 
 /* The work decomposition of the persistent tiled GEMM (the kernel that
  * zsaa_op_linear and the forward use beyond the weight-streaming and
- * swapped-operand row ranges) for one call shape, computed on the host exactly
+ * swapped-operand row ranges; the paper has no counterpart: this describes
+ * how the library splits the projections of Appendix A over the device's SMs)
+ * for one call shape, computed on the host exactly
  * as a launch computes it, without device work (no GPU needed).  The device
  * is described by sms (one-CTA kernel CTAs resident at once, one per SM;
  * >= 1), pair_slots (CTA pairs resident at once; 0: the pair kernel is not
