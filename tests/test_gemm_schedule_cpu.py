@@ -93,13 +93,12 @@ def check_schedule(z, epi, M, N, K, hd=64, sms=152, pair_slots=76, split_slots=2
     return plan, items
 
 
-def forward_shapes():
+def forward_shapes(z):
     """(epilogue, M, N, K, hd) of every GEMM of the bench's forwards."""
     out = set()
     for name in ("1b", "1b_cls", "8b"):
         wl = I.WORKLOADS[name]
         sh, B, L = wl["shape"], wl["B"], wl["L"]
-        from paper_2509_01190_gb300 import zsaa as z
         cfg = z.config_from_shape(sh)
         d, hd, F = sh.d_model, sh.head_dim, sh.ffn_dim
         qkv = (sh.n_heads + 2 * sh.n_kv_heads) * hd
@@ -121,7 +120,7 @@ def test_forward_gemm_schedules(zlib, device):
         dev["pair_slots"] = 0
     if device == "no_workspace":
         dev["split_slots"] = 0
-    shapes = forward_shapes()
+    shapes = forward_shapes(zlib)
     assert len(shapes) > 100
     kinds = set()
     for epi, M, N, K, hd in shapes:
