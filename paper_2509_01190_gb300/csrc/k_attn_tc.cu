@@ -427,15 +427,17 @@ __global__ void v_transpose_kernel(const bf16* __restrict__ qkv, int B, int N, i
   }
 }
 
+// SMs of the current device (kept per device).
 int attn_sms() {
-  static int n = 0;
-  if (n == 0) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-    if (n <= 0) n = 1;
+  static int cached[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  if (cached[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+    cached[dev] = n;
   }
-  return n;
+  return cached[dev];
 }
 
 bool encode(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t ld_elems,
