@@ -472,11 +472,6 @@ __global__ void colmass_f32_kernel(const float* __restrict__ qkv, const float* _
   if (lane == 0) parts[(static_cast<size_t>(b) * Hkv + g) * N + j] = acc;
 }
 
-template <typename Kern>
-cudaError_t set_smem(Kern k, int bytes) {
-  return cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-}
-
 }  // namespace
 
 cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, int Hkv, int hd,
@@ -493,13 +488,15 @@ cudaError_t launch_attention(int dtype, const void* qkv, int B, int N, int Hq, i
   dim3 grid((N + 63) / 64, Hq, B);
   if (hd == 64) {
     const int smem = 5 * 64 * 128;
-    static cudaError_t e = set_smem(attn_fwd_bf16_kernel<64>, smem);
+    static OncePerDevice once;
+    const cudaError_t e = set_smem_limit_once(once, attn_fwd_bf16_kernel<64>, smem);
     if (e != cudaSuccess) return e;
     ZSAA_LAUNCH(attn_fwd_bf16_kernel<64>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), N, Hq, Hkv,
                                                       static_cast<bf16*>(out), lse, scale_log2, causal, cu, key_alive);
   } else if (hd == 128) {
     const int smem = 5 * 64 * 256;
-    static cudaError_t e = set_smem(attn_fwd_bf16_kernel<128>, smem);
+    static OncePerDevice once;
+    const cudaError_t e = set_smem_limit_once(once, attn_fwd_bf16_kernel<128>, smem);
     if (e != cudaSuccess) return e;
     ZSAA_LAUNCH(attn_fwd_bf16_kernel<128>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), N, Hq, Hkv,
                                                        static_cast<bf16*>(out), lse, scale_log2, causal, cu, key_alive);
@@ -542,14 +539,16 @@ cudaError_t colmass_parts(int dtype, const void* qkv, const float* lse, const fl
   dim3 grid((N + 63) / 64, *n_qc, Hkv * B);
   if (hd == 64) {
     const int smem = 3 * 64 * 128 + 2 * 64 * 4;
-    static cudaError_t e = set_smem(colmass_bf16_kernel<64>, smem);
+    static OncePerDevice once;
+    const cudaError_t e = set_smem_limit_once(once, colmass_bf16_kernel<64>, smem);
     if (e != cudaSuccess) return e;
     ZSAA_LAUNCH(colmass_bf16_kernel<64>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), lse, N, Hq,
                                                      Hkv, B, kColmassQPer, weight_vnorm, parts,
                                                      scale_log2, causal);
   } else if (hd == 128) {
     const int smem = 3 * 64 * 256 + 2 * 64 * 4;
-    static cudaError_t e = set_smem(colmass_bf16_kernel<128>, smem);
+    static OncePerDevice once;
+    const cudaError_t e = set_smem_limit_once(once, colmass_bf16_kernel<128>, smem);
     if (e != cudaSuccess) return e;
     ZSAA_LAUNCH(colmass_bf16_kernel<128>, dim3(grid), dim3(128), smem, s, static_cast<const bf16*>(qkv), lse, N, Hq,
                                                       Hkv, B, kColmassQPer, weight_vnorm, parts,
