@@ -198,7 +198,10 @@ int* shared_status() {
   if (it != g_status_by_dev.end()) return it->second;
   int* p = nullptr;
   if (cudaMalloc(&p, sizeof(int)) != cudaSuccess) return nullptr;
-  if (cudaMemset(p, 0, sizeof(int)) != cudaSuccess) return nullptr;
+  if (cudaMemset(p, 0, sizeof(int)) != cudaSuccess) {
+    cudaFree(p);
+    return nullptr;
+  }
   g_status_by_dev[dev] = p;
   return p;
 }
@@ -216,8 +219,12 @@ bool op_splitk_ws(float** ws, int** flags) {
     float* p = nullptr;
     int* f = nullptr;
     if (cudaMalloc(&p, kSplitKWorkspaceElems * sizeof(float)) != cudaSuccess) return false;
-    if (cudaMalloc(&f, kSplitKFlags * sizeof(int)) != cudaSuccess) return false;
-    if (cudaMemset(f, 0, kSplitKFlags * sizeof(int)) != cudaSuccess) return false;
+    if (cudaMalloc(&f, kSplitKFlags * sizeof(int)) != cudaSuccess ||
+        cudaMemset(f, 0, kSplitKFlags * sizeof(int)) != cudaSuccess) {
+      cudaFree(p);
+      if (f != nullptr) cudaFree(f);
+      return false;
+    }
     it = g_op_ws.emplace(dev, std::make_pair(p, f)).first;
   }
   *ws = it->second.first;
@@ -256,10 +263,15 @@ bool op_rope_table(float theta, int hd, RopeTable* out) {
       sv[static_cast<size_t>(q) * half + i] = static_cast<float>(std::sin(a));
     }
   RopeTable t{nullptr, nullptr};
-  if (cudaMalloc(&t.cos_t, c.size() * 4) != cudaSuccess) return false;
-  if (cudaMalloc(&t.sin_t, c.size() * 4) != cudaSuccess) return false;
-  if (cudaMemcpy(t.cos_t, c.data(), c.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess) return false;
-  if (cudaMemcpy(t.sin_t, sv.data(), c.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess) return false;
+  const bool ok = cudaMalloc(&t.cos_t, c.size() * 4) == cudaSuccess &&
+                  cudaMalloc(&t.sin_t, c.size() * 4) == cudaSuccess &&
+                  cudaMemcpy(t.cos_t, c.data(), c.size() * 4, cudaMemcpyHostToDevice) == cudaSuccess &&
+                  cudaMemcpy(t.sin_t, sv.data(), c.size() * 4, cudaMemcpyHostToDevice) == cudaSuccess;
+  if (!ok) {
+    if (t.cos_t != nullptr) cudaFree(t.cos_t);
+    if (t.sin_t != nullptr) cudaFree(t.sin_t);
+    return false;
+  }
   g_rope_tables[key] = t;
   *out = t;
   return true;
