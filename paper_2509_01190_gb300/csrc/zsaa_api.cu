@@ -1811,6 +1811,9 @@ zsaa_status zsaa_gemm_schedule(int epilogue, int M, int N, int K, int hd, int sm
   if (epilogue < 0 || epilogue > 4) return fail(ZSAA_ERR_INVALID_ARG, "bad epilogue");
   if (epilogue == kEpiRope && (hd < 32 || hd % 32)) return fail(ZSAA_ERR_INVALID_ARG, "bad RoPE head size");
   if (sms < 1 || pair_slots < 0 || split_slots < 0) return fail(ZSAA_ERR_INVALID_ARG, "bad device description");
+  // tile counts are ints: at most 2^31 - 1 tiles of the narrowest plan (128 x 64)
+  if ((static_cast<long long>(M) + 127) / 128 * ((2LL * N + 63) / 64) > 0x7fffffffLL)
+    return fail(ZSAA_ERR_UNSUPPORTED, "shape too large for the tile plan");
   long long n = 0;
   const int r = gemm_tc_schedule(epilogue, M, N, K, hd, sms, pair_slots, split_slots, plan_out, items, cap, &n);
   if (r == -1) return fail(ZSAA_ERR_UNSUPPORTED, "no tile plan for this shape");

@@ -170,3 +170,5 @@ def test_schedule_rejects_bad_arguments(zlib):
         zlib.zsaa_gemm_schedule(0, 100, 256, 256, 0, 0, 76, 256)  # no SMs
     with pytest.raises(zlib.ZsaaError):
         zlib.zsaa_gemm_schedule(5, 100, 256, 256, 0, 152, 76, 256)  # epilogue
+    with pytest.raises(zlib.ZsaaError):
+        zlib.zsaa_gemm_schedule(0, 2 ** 31 - 1, 2 ** 30, 64, 0, 152, 76, 256)  # tile count
